@@ -1,0 +1,436 @@
+// SMAT simulated-merge transform: plain single-threaded CPU oracle.
+//
+// TEST INFRASTRUCTURE ONLY. This file is the correctness reference for the
+// CUDA path. Only tests/, the smoke check and the bench's CPU-baseline leg
+// may load it. It shares no source, header, table or helper with the CUDA
+// library: the Philox block, the stream layout, the bf16 rounding and the
+// transforms below are written out independently from their definitions.
+//
+// What it computes (paper: "SMAT: Simple and Efficient Merge-Aware Training"):
+//   forward   theta~ = theta0 + alpha * m (.) (theta - theta0) + eps
+//             Eq. smat-state (Sec. 4.1), Scale / Mask / Perturb (Sec. 4.1,
+//             Eq. smat-mask for m, uniform eps on [-sqrt3 sigma, sqrt3 sigma]).
+//   gradient  g = alpha * m (.) g~                  Eq. smat-gradient (Sec. 4.2)
+//   the mask is regenerated for the gradient, never stored (App. D,
+//   "Implementation details").
+//
+// The paper does not say how the random draws are produced. The counter-based
+// stream layout below is this project's specification; every reading of the
+// paper it relies on is listed in the design notes (readings R1-R15).
+//
+// Stream specification (both sides implement it; nothing here is shared):
+//   Philox-4x32-R block (Salmon et al., SC'11), R = 10 by default.
+//   key     = (seed mod 2^32, seed div 2^32)
+//   counter = (j mod 2^32, j div 2^32, (stream << 28) | tensor_id, step)
+//   W(stream, tid, j)[w] = word w of that block.
+//   streams: MASK = 0, NOISE = 1, ALPHA_E = 2, ALPHA_T = 3, MASK_LO = 4.
+//   gidx    = elem_offset + i  (global element index of local element i)
+//   u01(u)      = (u >> 8) * 2^-24          in [0, 1)
+//   u01_open(u) = ((u >> 8) + 1) * 2^-24    in (0, 1]
+//   sym(u)      = (2 (u >> 8) + 1 - 2^24) * 2^-24   odd multiples of 2^-24 in (-1, 1)
+//   Mask uniform U(gidx) in [0, 2^32):
+//     hi = byte (gidx & 3) of W(MASK, tid, gidx >> 4)[(gidx >> 2) & 3]
+//     lo = W(MASK_LO, tid, gidx >> 2)[gidx & 3] >> 8
+//     U  = hi * 2^24 + lo ;  kept  <=>  U < T,  T = floor(p_keep * 2^32)
+//   Noise word  n = W(NOISE, tid, gidx >> 2)[gidx & 3]
+//   Alpha:  per tensor  alpha = fma(amax - amin, u01(W(ALPHA_T, t_a, 0)[0]), amin)
+//           t_a = 0x0FFFFFFF (one alpha for all tensors) or the tensor id;
+//           per element alpha = fma(amax - amin, u01(W(ALPHA_E, tid, gidx >> 2)[gidx & 3]), amin)
+//
+// Build: g++ -O2 -ffp-contract=off -shared -fPIC (no fast-math: every float
+// operation below is one IEEE binary32 operation, round to nearest even).
+
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <vector>
+
+namespace {
+
+// ---------------------------------------------------------------- Philox ---
+// Philox-4x32-R as defined by Salmon, Moraes, Dror and Shaw, "Parallel Random
+// Numbers: As Easy as 1, 2, 3" (SC'11): each round multiplies words 0 and 2
+// by the two round multipliers, keeps both halves of the 64-bit products and
+// mixes the high halves with words 1 and 3 and the round key; the key is
+// bumped by the two Weyl increments between rounds.
+const uint32_t kMulA = 0xD2511F53u;   // multiplier applied to counter word 0
+const uint32_t kMulB = 0xCD9E8D57u;   // multiplier applied to counter word 2
+const uint32_t kWeylA = 0x9E3779B9u;  // key word 0 increment (golden ratio)
+const uint32_t kWeylB = 0xBB67AE85u;  // key word 1 increment (sqrt(3) - 1)
+
+void philox_block(const uint32_t ctr[4], uint32_t k0, uint32_t k1, int rounds,
+                  uint32_t out[4]) {
+  uint32_t x0 = ctr[0], x1 = ctr[1], x2 = ctr[2], x3 = ctr[3];
+  for (int r = 0; r < rounds; ++r) {
+    if (r > 0) {
+      k0 += kWeylA;
+      k1 += kWeylB;
+    }
+    const uint64_t prodA = (uint64_t)kMulA * (uint64_t)x0;
+    const uint64_t prodB = (uint64_t)kMulB * (uint64_t)x2;
+    const uint32_t hiA = (uint32_t)(prodA >> 32), loA = (uint32_t)prodA;
+    const uint32_t hiB = (uint32_t)(prodB >> 32), loB = (uint32_t)prodB;
+    const uint32_t n0 = hiB ^ x1 ^ k0;
+    const uint32_t n1 = loB;
+    const uint32_t n2 = hiA ^ x3 ^ k1;
+    const uint32_t n3 = loA;
+    x0 = n0; x1 = n1; x2 = n2; x3 = n3;
+  }
+  out[0] = x0; out[1] = x1; out[2] = x2; out[3] = x3;
+}
+
+enum { S_MASK = 0, S_NOISE = 1, S_ALPHA_E = 2, S_ALPHA_T = 3, S_MASK_LO = 4 };
+const uint32_t kGlobalAlphaId = 0x0FFFFFFFu;
+
+enum { ALPHA_GLOBAL = 0, ALPHA_PER_TENSOR = 1, ALPHA_PER_ELEMENT = 2 };
+enum { NOISE_UNIFORM = 0, NOISE_GAUSSIAN = 1 };
+enum { DT_F32 = 0, DT_BF16 = 1 };
+
+}  // namespace
+
+extern "C" {
+
+// Layout mirrored by the ctypes wrapper (oracle/__init__.py).
+struct OrcConfig {
+  uint64_t seed;
+  uint32_t step;
+  int32_t rounds;      // Philox rounds (10 by default)
+  int32_t alpha_mode;  // ALPHA_GLOBAL / ALPHA_PER_TENSOR / ALPHA_PER_ELEMENT
+  int32_t noise;       // NOISE_UNIFORM / NOISE_GAUSSIAN
+  float alpha_min;
+  float alpha_max;
+};
+
+struct OrcTensor {
+  uint32_t tensor_id;  // < 0x0FFFFFFF
+  int32_t dtype;       // parameter storage dtype
+  int64_t numel;
+  int64_t elem_offset;
+  float keep_prob;     // p_keep = 1 - p (paper's p is the drop probability)
+  float sigma;         // Perturb RMS when sigma_rel == 0
+  float sigma_rel;     // > 0: sigma_t = sigma_rel * std_pop(theta - theta0)
+};
+
+}  // extern "C"
+
+namespace {
+
+uint32_t stream_word(const OrcConfig& cfg, uint32_t stream, uint32_t tid,
+                     uint64_t j, unsigned w) {
+  uint32_t ctr[4] = {(uint32_t)(j & 0xFFFFFFFFu), (uint32_t)(j >> 32),
+                     (stream << 28) | tid, cfg.step};
+  uint32_t out[4];
+  philox_block(ctr, (uint32_t)(cfg.seed & 0xFFFFFFFFu), (uint32_t)(cfg.seed >> 32),
+               cfg.rounds, out);
+  return out[w];
+}
+
+const float kTwoPow24Inv = 5.9604644775390625e-08f;  // 2^-24, exact
+
+float u01(uint32_t u) { return (float)(u >> 8) * kTwoPow24Inv; }
+double u01_open_d(uint32_t u) { return (double)((u >> 8) + 1u) * 0x1p-24; }
+double u01_d(uint32_t u) { return (double)(u >> 8) * 0x1p-24; }
+float sym(uint32_t u) {
+  const int32_t k = (int32_t)(u >> 8);
+  return (float)(2 * k + 1 - (1 << 24)) * kTwoPow24Inv;
+}
+
+// ------------------------------------------------------------- bf16 I/O ---
+float bf16_bits_to_f32(uint16_t h) {
+  uint32_t b = (uint32_t)h << 16;
+  float f;
+  std::memcpy(&f, &b, 4);
+  return f;
+}
+
+// Round to nearest even; NaN stays NaN (quiet bit set); overflow rounds to inf.
+uint16_t f32_to_bf16_bits(float f) {
+  uint32_t b;
+  std::memcpy(&b, &f, 4);
+  if ((b & 0x7F800000u) == 0x7F800000u && (b & 0x007FFFFFu) != 0u)
+    return (uint16_t)((b >> 16) | 0x0040u);
+  const uint32_t lsb = (b >> 16) & 1u;
+  b += 0x7FFFu + lsb;
+  return (uint16_t)(b >> 16);
+}
+
+float load_elem(const void* p, int dtype, int64_t i) {
+  if (dtype == DT_BF16) return bf16_bits_to_f32(((const uint16_t*)p)[i]);
+  return ((const float*)p)[i];
+}
+
+void store_elem(void* p, int dtype, int64_t i, float v) {
+  if (dtype == DT_BF16)
+    ((uint16_t*)p)[i] = f32_to_bf16_bits(v);
+  else
+    ((float*)p)[i] = v;
+}
+
+uint32_t stored_bits(int dtype, float v) {
+  if (dtype == DT_BF16) return f32_to_bf16_bits(v);
+  uint32_t b;
+  std::memcpy(&b, &v, 4);
+  return b;
+}
+
+// ------------------------------------------------------ per-call scalars ---
+struct Scalars {
+  float alpha;        // per-tensor alpha (unused in per-element mode)
+  float inv_keep;     // 1 / p_keep  (Eq. smat-mask: 1 / (1 - p))
+  float c;            // alpha * inv_keep
+  uint64_t T;         // keep threshold on the 32-bit mask uniform
+  float sigma;        // Perturb RMS for this call
+  float noise_scale;  // sqrt(3) sigma (uniform) or sigma (Gaussian)
+};
+
+// Population mean and centred second moment of delta = theta - theta0 (each
+// delta one fp32 subtraction), two passes in double.
+void delta_moments(const OrcTensor& t, const void* th, const void* t0,
+                   double* mean_out, double* m2_out) {
+  if (t.numel <= 0) { *mean_out = 0.0; *m2_out = 0.0; return; }
+  double s = 0.0;
+  for (int64_t i = 0; i < t.numel; ++i) {
+    const float d = load_elem(th, t.dtype, i) - load_elem(t0, t.dtype, i);
+    s += (double)d;
+  }
+  const double mean = s / (double)t.numel;
+  double m2 = 0.0;
+  for (int64_t i = 0; i < t.numel; ++i) {
+    const float d = load_elem(th, t.dtype, i) - load_elem(t0, t.dtype, i);
+    const double e = (double)d - mean;
+    m2 += e * e;
+  }
+  *mean_out = mean;
+  *m2_out = m2;
+}
+
+float sigma_for(const OrcTensor& t, const void* th, const void* t0) {
+  if (!(t.sigma_rel > 0.0f)) return t.sigma;
+  if (t.numel <= 0) return 0.0f;
+  double mean, m2;
+  delta_moments(t, th, t0, &mean, &m2);
+  return (float)((double)t.sigma_rel * std::sqrt(m2 / (double)t.numel));
+}
+
+// Scale (Sec. 4.1): alpha ~ U[alpha_min, alpha_max); Mask (Eq. smat-mask):
+// keep with probability p_keep, rescale kept entries by 1 / p_keep; Perturb:
+// uniform on [-sqrt3 sigma, sqrt3 sigma] (Sec. 4.1) or N(0, sigma^2).
+Scalars make_scalars(const OrcConfig& cfg, const OrcTensor& t, float sigma) {
+  Scalars s;
+  const float width = cfg.alpha_max - cfg.alpha_min;
+  if (cfg.alpha_mode == ALPHA_PER_ELEMENT) {
+    s.alpha = 0.0f;
+  } else {
+    const uint32_t ta = (cfg.alpha_mode == ALPHA_GLOBAL) ? kGlobalAlphaId : t.tensor_id;
+    s.alpha = std::fma(width, u01(stream_word(cfg, S_ALPHA_T, ta, 0, 0)), cfg.alpha_min);
+  }
+  s.inv_keep = (t.keep_prob > 0.0f) ? (float)(1.0 / (double)t.keep_prob) : 0.0f;
+  s.c = s.alpha * s.inv_keep;
+  s.T = (uint64_t)std::floor((double)t.keep_prob * 4294967296.0);
+  s.sigma = sigma;
+  s.noise_scale = (cfg.noise == NOISE_UNIFORM) ? (float)(std::sqrt(3.0) * (double)sigma)
+                                               : sigma;
+  return s;
+}
+
+// ------------------------------------------------------- element values ---
+bool is_kept(const OrcConfig& cfg, const OrcTensor& t, const Scalars& s, uint64_t gidx) {
+  const uint32_t hw = stream_word(cfg, S_MASK, t.tensor_id, gidx >> 4, (unsigned)((gidx >> 2) & 3));
+  const uint32_t hi = (hw >> (8u * (unsigned)(gidx & 3))) & 0xFFu;
+  const uint32_t lo = stream_word(cfg, S_MASK_LO, t.tensor_id, gidx >> 2, (unsigned)(gidx & 3)) >> 8;
+  const uint64_t U = ((uint64_t)hi << 24) | (uint64_t)lo;
+  return U < s.T;
+}
+
+float element_c(const OrcConfig& cfg, const OrcTensor& t, const Scalars& s, uint64_t gidx) {
+  if (cfg.alpha_mode != ALPHA_PER_ELEMENT) return s.c;
+  const float width = cfg.alpha_max - cfg.alpha_min;
+  const uint32_t u = stream_word(cfg, S_ALPHA_E, t.tensor_id, gidx >> 2, (unsigned)(gidx & 3));
+  const float alpha = std::fma(width, u01(u), cfg.alpha_min);
+  return alpha * s.inv_keep;
+}
+
+// Standard-normal variate of element gidx: Box-Muller on the word pair
+// (2q, 2q+1) of its noise block, evaluated in double and rounded once.
+double gauss_z(const OrcConfig& cfg, const OrcTensor& t, uint64_t gidx) {
+  const unsigned w = (unsigned)(gidx & 3);
+  const unsigned q = w >> 1;
+  const uint32_t a = stream_word(cfg, S_NOISE, t.tensor_id, gidx >> 2, 2 * q);
+  const uint32_t b = stream_word(cfg, S_NOISE, t.tensor_id, gidx >> 2, 2 * q + 1);
+  const double rho = std::sqrt(-2.0 * std::log(u01_open_d(a)));
+  const double phi = 2.0 * M_PI * u01_d(b);
+  return (w & 1u) ? rho * std::sin(phi) : rho * std::cos(phi);
+}
+
+float noise_eps(const OrcConfig& cfg, const OrcTensor& t, const Scalars& s, uint64_t gidx) {
+  if (cfg.noise == NOISE_UNIFORM) {
+    const uint32_t n = stream_word(cfg, S_NOISE, t.tensor_id, gidx >> 2, (unsigned)(gidx & 3));
+    return s.noise_scale * sym(n);
+  }
+  return s.noise_scale * (float)gauss_z(cfg, t, gidx);
+}
+
+// Eq. smat-state for one element, fp32 arithmetic, before the storage rounding.
+float simulate_value(const OrcConfig& cfg, const OrcTensor& t, const Scalars& s,
+                     uint64_t gidx, float th, float t0) {
+  float x;
+  if (is_kept(cfg, t, s, gidx)) {
+    const float c = element_c(cfg, t, s, gidx);
+    const float d = th - t0;
+    x = (c == 1.0f) ? th : std::fma(c, d, t0);
+  } else {
+    x = t0;
+  }
+  if (s.sigma > 0.0f) x = x + noise_eps(cfg, t, s, gidx);
+  return x;
+}
+
+// Eq. smat-gradient for one element, fp32, before the storage rounding.
+float gradmap_value(const OrcConfig& cfg, const OrcTensor& t, const Scalars& s,
+                    uint64_t gidx, float gsim, int accumulate, float gold) {
+  float g = 0.0f;
+  if (is_kept(cfg, t, s, gidx)) g = element_c(cfg, t, s, gidx) * gsim;
+  if (accumulate) g = gold + g;
+  return g;
+}
+
+}  // namespace
+
+extern "C" {
+
+// One Philox-4x32-R block.
+void orc_philox(const uint32_t* ctr4, const uint32_t* key2, int32_t rounds, uint32_t* out4) {
+  philox_block(ctr4, key2[0], key2[1], rounds, out4);
+}
+
+// Raw stream word W(stream, tid, j)[w] for n (j, w) pairs.
+void orc_stream_words(const OrcConfig* cfg, uint32_t stream, uint32_t tid, const uint64_t* j,
+                      const uint32_t* w, int64_t n, uint32_t* out) {
+  for (int64_t i = 0; i < n; ++i) out[i] = stream_word(*cfg, stream, tid, j[i], w[i] & 3u);
+}
+
+// fp32 <-> bf16 bit conversions (storage rounding of the oracle).
+void orc_f32_to_bf16(const float* x, int64_t n, uint16_t* out) {
+  for (int64_t i = 0; i < n; ++i) out[i] = f32_to_bf16_bits(x[i]);
+}
+
+// Per-call scalars: out = {alpha, inv_keep, c, T, sigma_t, noise_scale}.
+// theta / theta0 are read only when sigma_rel > 0.
+void orc_scalars(const OrcConfig* cfg, const OrcTensor* t, const void* th, const void* t0,
+                 double* out6) {
+  const Scalars s = make_scalars(*cfg, *t, sigma_for(*t, th, t0));
+  out6[0] = s.alpha; out6[1] = s.inv_keep; out6[2] = s.c;
+  out6[3] = (double)s.T; out6[4] = s.sigma; out6[5] = s.noise_scale;
+}
+
+// delta statistics: out = {mean, M2, sigma_t}.
+void orc_delta_stats(const OrcTensor* t, const void* th, const void* t0, double* out3) {
+  double mean, m2;
+  delta_moments(*t, th, t0, &mean, &m2);
+  out3[0] = mean; out3[1] = m2; out3[2] = sigma_for(*t, th, t0);
+}
+
+// Forward over a whole tensor: out[i] = round_dtype(Eq. smat-state).
+void orc_simulate(const OrcConfig* cfg, const OrcTensor* t, const void* th, const void* t0,
+                  void* out) {
+  const Scalars s = make_scalars(*cfg, *t, sigma_for(*t, th, t0));
+  for (int64_t i = 0; i < t->numel; ++i) {
+    const uint64_t gidx = (uint64_t)(t->elem_offset + i);
+    const float v = simulate_value(*cfg, *t, s, gidx, load_elem(th, t->dtype, i),
+                                   load_elem(t0, t->dtype, i));
+    store_elem(out, t->dtype, i, v);
+  }
+}
+
+// Forward at sampled local indices with a given sigma_t; th_vals / t0_vals are
+// the fp32 values of theta / theta0 there. out_bits: stored bits (bf16 in the
+// low 16 bits); kept_out: 1 if the element was kept.
+void orc_simulate_at(const OrcConfig* cfg, const OrcTensor* t, float sigma_t, const int64_t* idx,
+                     int64_t n, const float* th_vals, const float* t0_vals, uint32_t* out_bits,
+                     uint8_t* kept_out) {
+  const Scalars s = make_scalars(*cfg, *t, sigma_t);
+  for (int64_t k = 0; k < n; ++k) {
+    const uint64_t gidx = (uint64_t)(t->elem_offset + idx[k]);
+    const float v = simulate_value(*cfg, *t, s, gidx, th_vals[k], t0_vals[k]);
+    out_bits[k] = stored_bits(t->dtype, v);
+    if (kept_out) kept_out[k] = is_kept(*cfg, *t, s, gidx) ? 1 : 0;
+  }
+}
+
+// Gradient map over a whole tensor: g_out[i] = round_gdtype(Eq. smat-gradient
+// [+ g_out[i] when accumulating]). g_out may equal g_sim when not accumulating.
+void orc_gradmap(const OrcConfig* cfg, const OrcTensor* t, int32_t gdtype, int32_t accumulate,
+                 const void* g_sim, void* g_out) {
+  const Scalars s = make_scalars(*cfg, *t, 0.0f);
+  for (int64_t i = 0; i < t->numel; ++i) {
+    const uint64_t gidx = (uint64_t)(t->elem_offset + i);
+    const float gold = accumulate ? load_elem(g_out, gdtype, i) : 0.0f;
+    const float v = gradmap_value(*cfg, *t, s, gidx, load_elem(g_sim, gdtype, i), accumulate, gold);
+    store_elem(g_out, gdtype, i, v);
+  }
+}
+
+// Gradient map at sampled local indices (values given in fp32).
+void orc_gradmap_at(const OrcConfig* cfg, const OrcTensor* t, int32_t gdtype, int32_t accumulate,
+                    const int64_t* idx, int64_t n, const float* gsim_vals, const float* gold_vals,
+                    uint32_t* out_bits) {
+  const Scalars s = make_scalars(*cfg, *t, 0.0f);
+  for (int64_t k = 0; k < n; ++k) {
+    const uint64_t gidx = (uint64_t)(t->elem_offset + idx[k]);
+    const float gold = accumulate ? gold_vals[k] : 0.0f;
+    out_bits[k] = stored_bits(gdtype, gradmap_value(*cfg, *t, s, gidx, gsim_vals[k], accumulate, gold));
+  }
+}
+
+// Packed keep bits: bit (i mod 32) of word i / 32, LSB first; unused high bits of
+// the last word are 0.
+void orc_mask_bits(const OrcConfig* cfg, const OrcTensor* t, uint32_t* bits) {
+  const Scalars s = make_scalars(*cfg, *t, 0.0f);
+  const int64_t nwords = (t->numel + 31) / 32;
+  for (int64_t w = 0; w < nwords; ++w) bits[w] = 0u;
+  for (int64_t i = 0; i < t->numel; ++i) {
+    const uint64_t gidx = (uint64_t)(t->elem_offset + i);
+    if (is_kept(*cfg, *t, s, gidx)) bits[i >> 5] |= (1u << (i & 31));
+  }
+}
+
+// Standard-normal variates z (before the sigma scaling) of the Gaussian mode.
+void orc_gauss_z(const OrcConfig* cfg, const OrcTensor* t, const uint64_t* gidx, int64_t n,
+                 double* z) {
+  for (int64_t k = 0; k < n; ++k) z[k] = gauss_z(*cfg, *t, gidx[k]);
+}
+
+// Real-arithmetic (double) evaluation of the same transform, for the
+// finite-difference check of Eq. smat-gradient. The draws and the per-call
+// scalars are those of the fp32 path; the arithmetic is double.
+void orc_simulate_f64(const OrcConfig* cfg, const OrcTensor* t, float sigma_t, const double* th,
+                      const double* t0, double* out) {
+  const Scalars s = make_scalars(*cfg, *t, sigma_t);
+  for (int64_t i = 0; i < t->numel; ++i) {
+    const uint64_t gidx = (uint64_t)(t->elem_offset + i);
+    double x = t0[i];
+    if (is_kept(*cfg, *t, s, gidx)) {
+      const double c = (double)element_c(*cfg, *t, s, gidx);
+      x = t0[i] + c * (th[i] - t0[i]);
+    }
+    if (s.sigma > 0.0f) {
+      if (cfg->noise == NOISE_UNIFORM) {
+        const uint32_t nw = stream_word(*cfg, S_NOISE, t->tensor_id, gidx >> 2, (unsigned)(gidx & 3));
+        x += (double)s.noise_scale * (double)sym(nw);
+      } else {
+        x += (double)s.noise_scale * gauss_z(*cfg, *t, gidx);
+      }
+    }
+    out[i] = x;
+  }
+}
+
+void orc_gradmap_f64(const OrcConfig* cfg, const OrcTensor* t, const double* gsim, double* out) {
+  const Scalars s = make_scalars(*cfg, *t, 0.0f);
+  for (int64_t i = 0; i < t->numel; ++i) {
+    const uint64_t gidx = (uint64_t)(t->elem_offset + i);
+    out[i] = is_kept(*cfg, *t, s, gidx) ? (double)element_c(*cfg, *t, s, gidx) * gsim[i] : 0.0;
+  }
+}
+
+}  // extern "C"

@@ -1,0 +1,543 @@
+"""Pins of the CPU oracle against facts fixed outside it.
+
+Each test checks the oracle against the paper's equations, a closed form, a
+statistical law, an independent library routine or brute force. None of them
+retypes the oracle's own formula. Chosen so that a plausible slip (a dropped
+term, a swapped theta/theta0, a wrong sign, a wrong stream index or word) fails
+at least one test.
+"""
+
+import json
+import math
+import os
+import subprocess
+import sys
+
+import numpy as np
+import pytest
+import torch
+from scipy import stats
+
+import oracle as O
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+
+
+def rng(seed):
+    return np.random.default_rng(seed)
+
+
+def f32(x):
+    return np.asarray(x, np.float32)
+
+
+# ----------------------------------------------------------------- Philox ---
+
+def _triton_philox(ctrs, seeds, rounds):
+    pytest.importorskip("triton")
+    req = json.dumps({"ctr": [[int(v) for v in c] for c in ctrs],
+                      "seed": [int(s) for s in seeds], "rounds": rounds})
+    p = subprocess.run([sys.executable, os.path.join(HERE, "_triton_philox.py")], input=req,
+                       capture_output=True, text=True, timeout=600)
+    if p.returncode != 0:
+        pytest.skip("triton interpreter unavailable: " + p.stderr[-300:])
+    return np.array(json.loads(p.stdout), dtype=np.uint64).astype(np.uint32)
+
+
+@pytest.mark.parametrize("rounds", [10, 7])
+def test_philox_block_matches_triton_library(rounds):
+    """Philox-4x32-R block (Salmon et al. SC'11) against Triton's Philox,
+    including counter words and keys with all bits set."""
+    r = rng(1)
+    ctrs = r.integers(0, 2**32, size=(48, 4), dtype=np.uint64)
+    ctrs[0] = 0
+    ctrs[1] = 2**32 - 1
+    seeds = r.integers(0, 2**63, size=48, dtype=np.uint64) * 2 + r.integers(0, 2, size=48, dtype=np.uint64)
+    seeds[0] = 0
+    seeds[1] = 2**64 - 1
+    ref = _triton_philox(ctrs, seeds, rounds)
+    for k in range(len(ctrs)):
+        s = int(seeds[k])
+        ours = O.philox(ctrs[k], [s & 0xFFFFFFFF, s >> 32], rounds)
+        assert np.array_equal(ours, ref[k]), (k, ours, ref[k])
+
+
+def test_stream_counter_layout_matches_triton_library():
+    """W(stream, tid, j)[w] is word w of the Philox block at counter
+    (j lo, j hi, stream << 28 | tid, step) under key (seed lo, seed hi)."""
+    r = rng(2)
+    seed, step = 0x0123456789ABCDEF, 77
+    cfg = O.config(seed=seed, step=step)
+    cases = []
+    for _ in range(24):
+        stream = int(r.integers(0, 5))
+        tid = int(r.integers(0, 0x0FFFFFFF))
+        j = int(r.integers(0, 2**40))
+        cases.append((stream, tid, j))
+    ref = _triton_philox([[j & 0xFFFFFFFF, j >> 32, (s << 28) | t, step] for s, t, j in cases],
+                         [seed] * len(cases), 10)
+    for k, (s, t, j) in enumerate(cases):
+        got = O.stream_words(cfg, s, t, [j] * 4, [0, 1, 2, 3])
+        assert np.array_equal(got, ref[k])
+
+
+def test_philox_avalanche():
+    """A one-bit counter change flips about half the output bits (a property of
+    the published block function; catches a dropped round or mixing term)."""
+    r = rng(3)
+    flips = []
+    for _ in range(400):
+        c = r.integers(0, 2**32, size=4, dtype=np.uint64).astype(np.uint32)
+        k = r.integers(0, 2**32, size=2, dtype=np.uint64).astype(np.uint32)
+        w = int(r.integers(0, 4))
+        b = int(r.integers(0, 32))
+        c2 = c.copy()
+        c2[w] ^= np.uint32(1 << b)
+        a1, a2 = O.philox(c, k), O.philox(c2, k)
+        flips.append(sum(bin(int(x ^ y)).count("1") for x, y in zip(a1, a2)))
+    m = np.mean(flips)
+    assert abs(m - 64.0) < 5 * 4.0 / math.sqrt(400) * 1.5, m
+
+
+# ------------------------------------------------------------------- bf16 ---
+
+def test_bf16_rounding_matches_torch():
+    """Storage rounding = round-to-nearest-even, as torch's CPU float->bfloat16."""
+    r = rng(4)
+    x = np.concatenate([
+        r.standard_normal(20000).astype(np.float32) * np.float32(0.02),
+        (r.integers(0, 2**32, size=20000, dtype=np.uint64).astype(np.uint32)).view(np.float32),
+        f32([0.0, -0.0, 1.0, -1.0, np.inf, -np.inf, 3.4028235e38, -3.4028235e38, 1e-45, -1e-45,
+             1.1754942e-38, 1.00390625, 1.01171875, 1.0078125 + 2**-24]),
+    ])
+    # exact ties: low 16 bits = 0x8000
+    ties = (r.integers(0, 2**16, size=2000, dtype=np.uint64).astype(np.uint32) << 16) | np.uint32(0x8000)
+    x = np.concatenate([x, ties.view(np.float32)])
+    ours = O.f32_to_bf16(x)
+    ref = torch.from_numpy(x.copy()).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    nan = np.isnan(x)
+    assert np.array_equal(ours[~nan], ref[~nan])
+    assert np.all(np.isnan(O.bf16_to_f32(ours[nan])))
+
+
+# ------------------------------------------------------------ identities ---
+
+@pytest.mark.parametrize("dtype", [O.F32, O.BF16])
+def test_identity_no_scale_mask_perturb(dtype):
+    """alpha = 1, p_keep = 1, sigma = 0: theta~ is theta bit for bit
+    (Eq. expert-displacement with alpha m = 1 and eps = 0)."""
+    r = rng(5)
+    n = 4099
+    th = r.standard_normal(n).astype(np.float32) * np.float32(3.0)
+    t0 = r.standard_normal(n).astype(np.float32) * np.float32(1e-3)
+    th[:4] = f32([0.0, -0.0, 1e30, -1e-40])
+    t0[:4] = f32([1e30, 5.0, -1e30, 7.0])
+    if dtype == O.BF16:
+        th, t0 = O.f32_to_bf16(th), O.f32_to_bf16(t0)
+    cfg = O.config(alpha_min=1.0, alpha_max=1.0, step=3)
+    t = O.tensor(11, n, dtype=dtype, keep_prob=1.0, sigma=0.0)
+    out = O.simulate(cfg, t, th, t0)
+    assert out.tobytes() == np.asarray(th).tobytes()
+
+
+@pytest.mark.parametrize("dtype", [O.F32, O.BF16])
+def test_all_dropped_without_noise_is_theta0(dtype):
+    """p_keep = 0, sigma = 0: every coordinate is masked, theta~ = theta0."""
+    r = rng(6)
+    n = 1000
+    th = r.standard_normal(n).astype(np.float32)
+    t0 = r.standard_normal(n).astype(np.float32)
+    if dtype == O.BF16:
+        th, t0 = O.f32_to_bf16(th), O.f32_to_bf16(t0)
+    t = O.tensor(3, n, dtype=dtype, keep_prob=0.0, sigma=0.0)
+    out = O.simulate(O.config(), t, th, t0)
+    assert out.tobytes() == np.asarray(t0).tobytes()
+
+
+def test_no_mask_closed_form():
+    """Mask off (p_keep = 1), fixed alpha = 0.75, no noise: theta~ = theta0 +
+    0.75 (theta - theta0) rounded once (Eq. smat-state), computed here in
+    float64 from the fp32 difference."""
+    r = rng(7)
+    n = 5000
+    th = r.standard_normal(n).astype(np.float32)
+    t0 = r.standard_normal(n).astype(np.float32)
+    cfg = O.config(alpha_min=0.75, alpha_max=0.75)
+    t = O.tensor(1, n, keep_prob=1.0)
+    out = O.simulate(cfg, t, th, t0)
+    d = (th - t0).astype(np.float64)
+    ref = (t0.astype(np.float64) + 0.75 * d).astype(np.float32)
+    assert np.array_equal(out, ref)
+
+
+def test_masked_closed_form_and_kept_set():
+    """alpha = 0.5, p_keep = 0.25 (rescale 4): kept coordinates are
+    theta0 + 2 (theta - theta0), dropped ones theta0 (Eq. smat-mask rescaling);
+    the kept set is the one mask_bits reports."""
+    r = rng(8)
+    n = 8192
+    th = r.standard_normal(n).astype(np.float32)
+    t0 = r.standard_normal(n).astype(np.float32)
+    cfg = O.config(alpha_min=0.5, alpha_max=0.5, step=9)
+    t = O.tensor(21, n, keep_prob=0.25)
+    out = O.simulate(cfg, t, th, t0)
+    kept = O.unpack_bits(O.mask_bits(cfg, t), n).astype(bool)
+    d = (th - t0).astype(np.float64)
+    ref = np.where(kept, (t0.astype(np.float64) + 2.0 * d).astype(np.float32), t0)
+    assert np.array_equal(out, ref)
+    assert 0.2 < kept.mean() < 0.3
+
+
+def test_scalars_inverse_keep_and_threshold():
+    """1 / p_keep is the Eq. smat-mask rescale 1 / (1 - p); the threshold is
+    floor(p_keep 2^32)."""
+    for pk in (0.0, 0.1, 0.3, 0.5, 0.7, 0.9, 1.0, 2.0**-20):
+        s = O.scalars(O.config(), O.tensor(5, 10, keep_prob=pk))
+        assert s["T"] == math.floor(float(np.float32(pk)) * 2**32)
+        if pk > 0:
+            assert s["inv_keep"] == float(np.float32(1.0 / float(np.float32(pk))))
+
+
+# ---------------------------------------------------------- Mask (Eq. 4) ---
+
+@pytest.mark.parametrize("pk", [0.1, 0.3, 0.5, 0.7, 0.9])
+def test_keep_rate_binomial(pk):
+    """Empirical keep rate within a 5-sigma binomial bound of p_keep."""
+    n = 200_000
+    t = O.tensor(1234, n, keep_prob=pk)
+    k = O.unpack_bits(O.mask_bits(O.config(seed=5, step=1), t), n).sum()
+    p = float(np.float32(pk))
+    assert abs(k - n * p) <= 5 * math.sqrt(n * p * (1 - p))
+
+
+def test_keep_threshold_low_24_bits_on_ties():
+    """kept <=> U < floor(p_keep 2^32) with U uniform on 32 bits: masks at nested
+    keep probabilities are nested (one uniform per coordinate), and between
+    p = 128/256 and p = 129/256 lie exactly the coordinates whose high byte is
+    128. At p = 1/2 + 2^-10 the low 24 bits of the threshold are 2^22, so a
+    quarter of those must be kept: treating the tie as always kept (rate 1) or
+    always dropped (rate 0) fails."""
+    n = 2_000_000
+    cfg = O.config(seed=11)
+
+    def kept(pk):
+        return O.unpack_bits(O.mask_bits(cfg, O.tensor(77, n, keep_prob=pk)), n).astype(bool)
+
+    lo, mid, hi = kept(0.5), kept(0.5 + 2.0**-10), kept(129 / 256)
+    assert np.all(lo <= mid) and np.all(mid <= hi)
+    ties = hi & ~lo
+    m = int(ties.sum())
+    assert abs(m - n / 256) < 5 * math.sqrt(n / 256)
+    rate = mid[ties].mean()
+    assert abs(rate - 0.25) < 5 * math.sqrt(0.25 * 0.75 / m)
+
+
+def test_mask_has_no_lag_correlation():
+    """Coordinates are masked independently (Eq. smat-mask): for lags inside and
+    across the 4- and 16-element draw groups, P(both kept) = p^2."""
+    n = 400_000
+    pk = 0.5
+    m = O.unpack_bits(O.mask_bits(O.config(seed=3), O.tensor(9, n, keep_prob=pk)), n).astype(np.float64)
+    for lag in (1, 2, 3, 4, 5, 8, 12, 15, 16, 17, 32, 64):
+        both = (m[:-lag] * m[lag:]).mean()
+        se = math.sqrt(0.25 * 0.75 / (n - lag))
+        assert abs(both - 0.25) < 6 * se, lag
+
+
+def test_masks_differ_across_tensors_steps_seeds():
+    n = 4096
+    base = O.mask_bits(O.config(seed=1, step=2), O.tensor(5, n, keep_prob=0.5))
+    for cfg, tid in ((O.config(seed=1, step=3), 5), (O.config(seed=2, step=2), 5), (O.config(seed=1, step=2), 6)):
+        other = O.mask_bits(cfg, O.tensor(tid, n, keep_prob=0.5))
+        agree = np.mean(O.unpack_bits(base, n) == O.unpack_bits(other, n))
+        assert 0.45 < agree < 0.55
+
+
+def test_mask_moments_over_steps():
+    """E[m_k] = 1 and E[m_k^2] = 1 / (1 - p_k) (proof of Prop. moments, App. C),
+    m = kept / p_keep, over many steps."""
+    n, steps, pk = 512, 600, 0.3
+    acc1 = np.zeros(n)
+    acc2 = np.zeros(n)
+    for s in range(steps):
+        kept = O.unpack_bits(O.mask_bits(O.config(seed=4, step=s), O.tensor(2, n, keep_prob=pk)), n)
+        m = kept / pk
+        acc1 += m
+        acc2 += m * m
+    tot = n * steps
+    e1, e2 = acc1.sum() / tot, acc2.sum() / tot
+    sd1 = math.sqrt((1 / pk - 1) / tot)
+    sd2 = math.sqrt((1 / pk**3 - 1 / pk**2) / tot)
+    assert abs(e1 - 1.0) < 5 * sd1
+    assert abs(e2 - 1 / pk) < 5 * sd2
+
+
+# ------------------------------------------------------- Scale and noise ---
+
+def test_alpha_uniform_per_tensor_and_global():
+    """Scale: alpha ~ U[alpha_min, alpha_max) (Sec. 4.1); one scalar for every
+    tensor in global mode, independent draws per tensor in per-tensor mode."""
+    amin, amax = 0.3, 1.0
+    al = []
+    for s in range(3000):
+        al.append(O.scalars(O.config(seed=8, step=s, alpha_min=amin, alpha_max=amax), O.tensor(4, 1))["alpha"])
+    al = np.array(al)
+    assert al.min() >= amin and al.max() < amax
+    assert stats.kstest((al - amin) / (amax - amin), "uniform").pvalue > 1e-4
+    g = O.config(seed=8, step=0, alpha_mode=O.ALPHA_GLOBAL)
+    ga = {O.scalars(g, O.tensor(tid, 1))["alpha"] for tid in range(20)}
+    assert len(ga) == 1
+    pt = O.config(seed=8, step=0, alpha_mode=O.ALPHA_PER_TENSOR)
+    pa = {O.scalars(pt, O.tensor(tid, 1))["alpha"] for tid in range(20)}
+    assert len(pa) == 20
+
+
+def test_uniform_noise_law():
+    """Perturb: eps ~ U[-sqrt3 sigma, sqrt3 sigma] (Sec. 4.1): with theta0 = 0 and
+    every coordinate dropped, theta~ = eps exactly; mean 0, variance sigma^2,
+    support inside the interval, KS against the uniform law."""
+    n, sigma = 200_000, 2e-3
+    t = O.tensor(8, n, keep_prob=0.0, sigma=sigma)
+    z = np.zeros(n, np.float32)
+    eps = O.simulate(O.config(seed=6, noise=O.NOISE_UNIFORM), t, z, z).astype(np.float64)
+    a = math.sqrt(3.0) * sigma
+    assert np.all(np.abs(eps) <= a * (1 + 1e-6))
+    assert abs(eps.mean()) < 5 * sigma / math.sqrt(n)
+    assert abs(eps.var() / sigma**2 - 1) < 5 * math.sqrt(0.8 / n)
+    assert stats.kstest(eps / a, "uniform", args=(-1, 2)).pvalue > 1e-4
+
+
+def test_gaussian_noise_law():
+    """Gaussian Perturb (eps ~ N(0, sigma^2)): KS against N(0, 1), unit
+    variance, and the two variates of each Box-Muller pair uncorrelated."""
+    n, sigma = 200_000, 1e-4
+    t = O.tensor(8, n, keep_prob=0.0, sigma=sigma)
+    z = np.zeros(n, np.float32)
+    eps = O.simulate(O.config(seed=6, noise=O.NOISE_GAUSSIAN), t, z, z).astype(np.float64) / sigma
+    assert stats.kstest(eps, "norm").pvalue > 1e-4
+    assert abs(eps.var() - 1) < 5 * math.sqrt(2.0 / n)
+    pairs = eps.reshape(-1, 2)
+    assert abs(np.corrcoef(pairs[:, 0], pairs[:, 1])[0, 1]) < 5 / math.sqrt(n / 2)
+    assert abs(np.corrcoef(eps[:-4], eps[4:])[0, 1]) < 5 / math.sqrt(n)
+
+
+def test_gaussian_z_matches_noise_of_simulate():
+    n = 64
+    t = O.tensor(8, n, keep_prob=0.0, sigma=1.0)
+    z = np.zeros(n, np.float32)
+    cfg = O.config(seed=9, noise=O.NOISE_GAUSSIAN)
+    eps = O.simulate(cfg, t, z, z)
+    zz = O.gauss_z(cfg, t, np.arange(n))
+    assert np.array_equal(eps, zz.astype(np.float32))
+
+
+# ------------------------------------------- Prop. moments (App. C) ---
+
+def test_state_moments_proposition():
+    """Prop. moments (App. C), global alpha: mean theta0 + abar Delta; covariance
+    v_a Delta Delta^T + s_a Diag(Delta^2 p/(1-p)) + sigma^2 I (p the drop
+    probability), checked coordinate-wise and on off-diagonal pairs."""
+    r = rng(10)
+    n, steps = 24, 6000
+    amin, pk, sigma = 0.2, 0.6, 0.05
+    t0 = r.standard_normal(n).astype(np.float32)
+    delta = (r.standard_normal(n) * 0.5 + np.sign(r.standard_normal(n))).astype(np.float32)
+    th = (t0 + delta).astype(np.float32)
+    D = (th - t0).astype(np.float64)
+    X = np.zeros((steps, n))
+    for s in range(steps):
+        cfg = O.config(seed=12, step=s, alpha_mode=O.ALPHA_GLOBAL, alpha_min=amin, alpha_max=1.0)
+        X[s] = O.simulate(cfg, O.tensor(3, n, keep_prob=pk, sigma=sigma), th, t0)
+    abar = (1 + amin) / 2
+    va = (1 - amin) ** 2 / 12
+    sa = abar**2 + va
+    p_drop = 1 - pk
+    mean_ref = t0 + abar * D
+    var_ref = va * D**2 + sa * D**2 * p_drop / (1 - p_drop) + sigma**2
+    mean = X.mean(0)
+    C = np.cov(X.T, bias=True)
+    assert np.all(np.abs(mean - mean_ref) < 5 * np.sqrt(var_ref / steps))
+    # variance: standard error of a sample variance <= sqrt((m4 - var^2) / steps)
+    m4 = ((X - mean) ** 4).mean(0)
+    assert np.all(np.abs(np.diag(C) - var_ref) < 5 * np.sqrt((m4 - np.diag(C) ** 2) / steps) + 1e-12)
+    # off-diagonal: only the shared alpha correlates coordinates
+    Xc = X - mean
+    for (k, l) in ((0, 1), (2, 7), (5, 19), (10, 11)):
+        prod = Xc[:, k] * Xc[:, l]
+        ref = va * D[k] * D[l]
+        assert abs(prod.mean() - ref) < 5 * prod.std() / math.sqrt(steps), (k, l)
+
+
+# ---------------------------------------------- gradient (Eq. smat-gradient) ---
+
+@pytest.mark.parametrize("mode", [O.ALPHA_PER_TENSOR, O.ALPHA_PER_ELEMENT])
+def test_gradient_map_matches_finite_differences(mode):
+    """With the draws fixed, the gradient of L(theta~(theta)) w.r.t. theta is
+    alpha m (.) grad L(theta~) (Eq. smat-gradient). L = 1/2 sum w theta~^2,
+    central differences in double."""
+    r = rng(13)
+    n = 61
+    th = r.standard_normal(n)
+    t0 = r.standard_normal(n)
+    w = r.standard_normal(n)
+    cfg = O.config(seed=21, step=4, alpha_mode=mode, alpha_min=0.2, alpha_max=1.0, noise=O.NOISE_GAUSSIAN)
+    t = O.tensor(6, n, keep_prob=0.7, sigma=0.01)
+
+    def loss(x):
+        y = O.simulate_f64(cfg, t, 0.01, x, t0)
+        return 0.5 * np.sum(w * y * y)
+
+    y = O.simulate_f64(cfg, t, 0.01, th, t0)
+    g = O.gradmap_f64(cfg, t, w * y)
+    h = 1e-6
+    fd = np.zeros(n)
+    for k in range(n):
+        e = np.zeros(n)
+        e[k] = h
+        fd[k] = (loss(th + e) - loss(th - e)) / (2 * h)
+    assert np.allclose(g, fd, rtol=1e-6, atol=1e-8)
+    kept = O.unpack_bits(O.mask_bits(O.config(seed=21, step=4, alpha_mode=mode), t), n).astype(bool)
+    assert np.all(g[~kept] == 0.0) and np.all(g[kept] != 0.0)
+
+
+def test_gradient_fp32_agrees_with_real_arithmetic():
+    r = rng(14)
+    n = 3000
+    gs = r.standard_normal(n).astype(np.float32)
+    cfg = O.config(seed=2, step=1, alpha_mode=O.ALPHA_PER_ELEMENT, alpha_min=0.0, alpha_max=1.0)
+    t = O.tensor(4, n, keep_prob=0.3)
+    g32 = O.gradmap(cfg, t, gs).astype(np.float64)
+    g64 = O.gradmap_f64(cfg, t, gs.astype(np.float64))
+    assert np.allclose(g32, g64, rtol=2 * 2**-24, atol=0)
+
+
+def test_gradient_zero_when_alpha_zero():
+    """alpha = 0: no coordinate contributes, the mapped gradient is 0 (Sec. 4.2)."""
+    n = 777
+    gs = rng(15).standard_normal(n).astype(np.float32)
+    cfg = O.config(alpha_min=0.0, alpha_max=0.0)
+    out = O.gradmap(cfg, O.tensor(1, n, keep_prob=0.5), gs)
+    assert np.all(out == 0.0)
+
+
+def test_gradient_of_ones_is_rescaled_mask():
+    """g~ = 1 maps to c on kept coordinates and 0 elsewhere, c = alpha / p_keep."""
+    n = 5000
+    cfg = O.config(seed=3, step=5)
+    t = O.tensor(17, n, keep_prob=0.7)
+    g = O.gradmap(cfg, t, np.ones(n, np.float32))
+    c = O.scalars(cfg, t)["c"]
+    kept = O.unpack_bits(O.mask_bits(cfg, t), n).astype(bool)
+    assert np.all(g[kept] == np.float32(c)) and np.all(g[~kept] == 0.0)
+
+
+def test_gradient_accumulate_adds():
+    r = rng(16)
+    n = 1000
+    gs = r.standard_normal(n).astype(np.float32)
+    go = r.standard_normal(n).astype(np.float32)
+    cfg = O.config(seed=3)
+    t = O.tensor(2, n, keep_prob=0.5)
+    plain = O.gradmap(cfg, t, gs)
+    acc = O.gradmap(cfg, t, gs, accumulate=True, g_old=go)
+    assert np.array_equal(acc, (go + plain).astype(np.float32))
+
+
+# ---------------------------------------------------- consistency checks ---
+
+def test_forward_kept_set_equals_gradient_kept_set():
+    """The gradient map regenerates the forward's mask (App. D): the kept flags of
+    the forward are exactly the nonzero pattern of the mapped ones."""
+    n = 3000
+    r = rng(17)
+    th = r.standard_normal(n).astype(np.float32)
+    t0 = r.standard_normal(n).astype(np.float32)
+    cfg = O.config(seed=5, step=2, noise=O.NOISE_GAUSSIAN)
+    t = O.tensor(99, n, keep_prob=0.4, sigma=1e-3)
+    _, kept = O.simulate_at(cfg, t, 1e-3, np.arange(n), th, t0)
+    g = O.gradmap(cfg, t, np.ones(n, np.float32))
+    assert np.array_equal(kept.astype(bool), g != 0)
+
+
+@pytest.mark.parametrize("split", [1, 15, 16, 17, 1000, 2999])
+def test_shard_invariance(split):
+    """Element offsets make any contiguous sharding produce the same bits."""
+    n = 3000
+    r = rng(18)
+    th = r.standard_normal(n).astype(np.float32)
+    t0 = r.standard_normal(n).astype(np.float32)
+    cfg = O.config(seed=7, step=1, alpha_mode=O.ALPHA_PER_ELEMENT, noise=O.NOISE_GAUSSIAN)
+    full = O.simulate(cfg, O.tensor(4, n, keep_prob=0.6, sigma=1e-2), th, t0)
+    a = O.simulate(cfg, O.tensor(4, split, keep_prob=0.6, sigma=1e-2), th[:split], t0[:split])
+    b = O.simulate(cfg, O.tensor(4, n - split, keep_prob=0.6, sigma=1e-2, elem_offset=split),
+                   th[split:], t0[split:])
+    assert np.array_equal(full, np.concatenate([a, b]))
+
+
+def test_simulate_at_matches_full_tensor():
+    n = 2000
+    r = rng(19)
+    th = O.f32_to_bf16(r.standard_normal(n).astype(np.float32) * 0.02)
+    t0 = O.f32_to_bf16(r.standard_normal(n).astype(np.float32) * 0.02)
+    cfg = O.config(seed=5, noise=O.NOISE_GAUSSIAN)
+    t = O.tensor(12, n, dtype=O.BF16, keep_prob=0.7, sigma_rel=0.1)
+    full = O.simulate(cfg, t, th, t0)
+    sig = O.delta_stats(t, th, t0)["sigma"]
+    idx = r.choice(n, 300, replace=False)
+    bits, _ = O.simulate_at(cfg, t, sig, idx, O.bf16_to_f32(th[idx]), O.bf16_to_f32(t0[idx]))
+    assert np.array_equal(bits.astype(np.uint16), full[idx])
+
+
+def test_delta_stats_match_numpy():
+    """sigma_t = sigma_rel * population std of theta - theta0."""
+    r = rng(20)
+    n = 100_003
+    t0 = O.f32_to_bf16(r.standard_normal(n).astype(np.float32) * 0.02)
+    d = r.standard_normal(n).astype(np.float32) * 3e-4 + 1e-4
+    th = O.f32_to_bf16(O.bf16_to_f32(t0) + d)
+    t = O.tensor(1, n, dtype=O.BF16, sigma_rel=0.1)
+    s = O.delta_stats(t, th, t0)
+    dd = (O.bf16_to_f32(th) - O.bf16_to_f32(t0)).astype(np.float64)
+    assert math.isclose(s["mean"], dd.mean(), rel_tol=1e-12)
+    assert math.isclose(s["sigma"], float(np.float32(0.1 * dd.std())), rel_tol=1e-6)
+
+
+def test_paper_default_settings_fixture():
+    """The paper's stated SMAT settings (tests/golden/paper_settings.json) give
+    the intended Mask keep rate and Perturb RMS."""
+    with open(os.path.join(HERE, "golden", "paper_settings.json")) as f:
+        gold = json.load(f)
+    for name, s in gold["settings"].items():
+        pk = 1.0 - s["mask_drop_p"]
+        n = 100_000
+        t = O.tensor(1, n, keep_prob=pk, sigma=s["perturb_rms"])
+        cfg = O.config(seed=1, alpha_min=s["alpha_min"], alpha_max=1.0, noise=O.NOISE_UNIFORM)
+        k = O.unpack_bits(O.mask_bits(cfg, t), n).sum()
+        assert abs(k - n * pk) <= 5 * math.sqrt(n * pk * (1 - pk)), name
+        z = np.zeros(n, np.float32)
+        eps = O.simulate(cfg, O.tensor(1, n, keep_prob=0.0, sigma=s["perturb_rms"]), z, z)
+        assert abs(np.sqrt(np.mean(eps.astype(np.float64) ** 2)) / s["perturb_rms"] - 1) < 0.01, name
+
+
+def test_oracle_regression_fixture():
+    """The oracle still reproduces its committed outputs (guards against an
+    unintended change of the stream specification)."""
+    with open(os.path.join(HERE, "golden", "oracle_regression.json")) as f:
+        doc = json.load(f)
+    for c in doc["cases"]:
+        cfg = O.OrcConfig(**c["config"])
+        t = O.OrcTensor(**c["tensor"])
+        pd = np.uint16 if t.dtype == O.BF16 else np.uint32
+        gd = np.uint16 if c["gdtype"] == O.BF16 else np.uint32
+        th = np.array(c["theta_bits"], pd)
+        t0 = np.array(c["theta0_bits"], pd)
+        gs = np.array(c["gsim_bits"], gd)
+        if t.dtype == O.F32:
+            th, t0 = th.view(np.float32), t0.view(np.float32)
+        if c["gdtype"] == O.F32:
+            gs = gs.view(np.float32)
+        sim = np.asarray(O.simulate(cfg, t, th, t0)).view(pd)
+        g = np.asarray(O.gradmap(cfg, t, gs, gdtype=c["gdtype"])).view(gd)
+        assert sim.tolist() == c["sim_bits"], c["name"]
+        assert g.tolist() == c["g_bits"], c["name"]
+        assert O.mask_bits(cfg, t).tolist() == c["mask_words"], c["name"]
