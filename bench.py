@@ -1,0 +1,456 @@
+#!/usr/bin/env python
+"""Benchmark of the SMAT simulated-merge hot path on GB300.
+
+One step = one SMAT simulated-loss step's worth of the hot path over the
+whole parameter list: delta statistics (sigma_t = 0.1 std(delta) per tensor),
+per-call scalars, the fused forward theta~ = theta0 + alpha m (.) (theta -
+theta0) + eps, the storage swap, the gradient map g = alpha m (.) g~ and the
+swap back. Workload: the 7B Llama-style list in bf16 (291 tensors,
+6,738,415,616 elements, bf16 gradients), Gaussian eps, per-tensor alpha ~
+U[0.3, 1), p_keep 0.7 on attention/MLP linears.
+
+Metric: algorithmic HBM bytes of the step / step time (GB/s), plus params/s.
+Algorithmic bytes per element: 2b (statistics: theta, theta0) + 3b (forward:
+theta, theta0 in, theta~ out) + 2gb (gradient: g~ in, g out) = 14 B in bf16.
+
+N > 1 (torchrun): each rank runs its own expert's full list (independent
+problems, weak scaling, no collective on the data path); value is the bytes
+of all ranks over the slowest rank's time.
+
+--impl reference runs the CPU oracle (the reference arm of this benchmark)
+on a bounded sample of the same workload, on the host cores, rank 0 only.
+"""
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from paper_2609_33437_gb300 import workloads as W  # noqa: E402
+
+METRIC = "simulated-merge fwd+grad-map HBM GB/s (fraction of GB300 peak); params/sec"
+UNIT = "GB/s"
+FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 8000.0
+KERNEL_SOURCES = [os.path.join(ROOT, "paper_2609_33437_gb300", "csrc", f)
+                  for f in ("smat_kernels.cu", "smat_internal.h")]
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["smat", "reference"], default="smat")
+    ap.add_argument("--workload", default="llama_7b", choices=["llama_7b", "dec_0p5b", "vl_7b", "tiny_flat"])
+    ap.add_argument("--noise", choices=["gaussian", "uniform"], default="gaussian")
+    ap.add_argument("--scale", type=int, default=0, help="cut the list to about this many elements (profiling)")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    return ap.parse_args()
+
+
+def workload(args) -> W.Workload:
+    if args.workload == "llama_7b":
+        w = W.llama_7b(noise=1 if args.noise == "gaussian" else 0)
+    else:
+        w = W.WORKLOADS[args.workload]()
+        if args.noise == "uniform":
+            w.noise = 0
+    if args.scale:
+        w = W.scaled(w, args.scale)
+    return w
+
+
+def step_bytes(w: W.Workload) -> dict:
+    b = 2 if w.dtype == W.BF16 else 4
+    gb = 2 if w.gdtype == W.BF16 else 4
+    n_rel = sum(t.numel for t in w.tensors if t.sigma_rel > 0)
+    return {"delta_stats": 2 * b * n_rel, "simulate": 3 * b * w.numel, "gradmap": 2 * gb * w.numel}
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_hash():
+    import hashlib
+    h = hashlib.sha256()
+    for p in KERNEL_SOURCES:
+        with open(p, "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str, wname: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel source (else None)."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        rec = d.get(kernel, {}).get(wname)
+        if rec and rec.get("kernel_hash") == kernel_hash():
+            return rec
+    except Exception:
+        pass
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during a region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.samples = []
+        self.proc = None
+        self.marks = []
+        try:
+            uuid = "GPU-" + str(torch.cuda.get_device_properties(device_index).uuid)
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", uuid, f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.perf_counter(), line.strip()))
+
+    def mark(self):
+        self.marks.append(time.perf_counter())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        t0, t1 = (self.marks + [0, 0])[:2]
+        rows = [s for t, s in self.samples if t0 <= t <= t1 + 0.15] or [s for _, s in self.samples[-3:]]
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            f = [x.strip() for x in r.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx.append(float(f[1]))
+            except ValueError:
+                continue
+            for name, v in zip(names, f[4:8]):
+                if v.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(local)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ------------------------------------------------------------ CPU oracle ---
+
+def oracle_run(w: W.Workload, max_elems: int, step: int = 0):
+    """Oracle forward + gradient map over a sample of w: every tensor of w
+    scaled so the sample totals about max_elems (all shapes and settings
+    kept). Returns (seconds, algorithmic bytes, elements, sample name)."""
+    import oracle as O
+    s = W.scaled(w, max_elems)
+    gen = torch.Generator().manual_seed(99)
+    cfg = O.config(seed=w.seed, step=step, alpha_mode=w.alpha_mode, noise=w.noise, alpha_min=w.alpha_min,
+                   alpha_max=w.alpha_max)
+    secs = 0.0
+    for k, spec in enumerate(s.tensors):
+        n = spec.numel
+        t0f = torch.randn(n, generator=gen) * w.theta0_std
+        thf = t0f + torch.randn(n, generator=gen) * w.delta_std
+        gf = torch.randn(n, generator=gen)
+
+        def host(x, dt):
+            x = x.to(W.torch_dtype(dt))
+            return x.view(torch.int16).numpy().view(np.uint16) if dt == W.BF16 else x.numpy()
+
+        th, t0, g = host(thf, w.dtype), host(t0f, w.dtype), host(gf, w.gdtype)
+        t = O.tensor(k, n, dtype=w.dtype, keep_prob=spec.keep_prob, sigma=spec.sigma, sigma_rel=spec.sigma_rel)
+        a = time.perf_counter()
+        O.simulate(cfg, t, th, t0)
+        O.gradmap(cfg, t, g, gdtype=w.gdtype)
+        secs += time.perf_counter() - a
+    nbytes = sum(step_bytes(s).values())
+    return secs, nbytes, s.numel, f"{s.name}: {len(s.tensors)} tensors, {s.numel} elements"
+
+
+def run_reference(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    w = workload(args)
+    per_step = int(min(8_000_000, max(200_000, 150.0 / max(1, args.steps + args.warmup) / 250e-9)))
+    for _ in range(args.warmup):
+        oracle_run(w, per_step)
+    tot_s, tot_b, tot_n = 0.0, 0, 0
+    sample = ""
+    for _ in range(args.steps):
+        s, b, n, sample = oracle_run(w, per_step)
+        tot_s += s
+        tot_b += b
+        tot_n += n
+    value = tot_b / tot_s / 1e9
+    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_s / args.steps,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+           "data": "synthetic", "params_per_s": tot_n / tot_s,
+           "config": {"workload": w.name, "elements_per_step_sample": tot_n // args.steps,
+                      "noise": "gaussian" if w.noise == 1 else "uniform"},
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                            "sample": f"each step: {sample} (single-threaded C++ oracle, forward + gradient map)"},
+           "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out))
+    return 0
+
+
+# ------------------------------------------------------------- GPU path ---
+
+def host_available_bytes():
+    try:
+        return os.sysconf("SC_AVPHYS_PAGES") * os.sysconf("SC_PAGE_SIZE")
+    except Exception:
+        return 0
+
+
+def e2e_run(w, sess_factory, steps, warmup, world):
+    """The same step through the public API with host inputs: pinned host
+    theta, theta0 and g~ are copied in and theta~ and g copied out every
+    step, inside the timed region."""
+    dev = torch.device("cuda")
+    tdt, gdt = W.torch_dtype(w.dtype), W.torch_dtype(w.gdtype)
+    n = w.numel
+    h_th = torch.empty(n, dtype=tdt, pin_memory=True)
+    h_t0 = torch.empty(n, dtype=tdt, pin_memory=True)
+    h_gs = torch.empty(n, dtype=gdt, pin_memory=True)
+    h_sim = torch.empty(n, dtype=tdt, pin_memory=True)
+    h_go = torch.empty(n, dtype=gdt, pin_memory=True)
+    offs = np.cumsum([0] + [t.numel for t in w.tensors])
+    d_th, d_t0, d_sim, d_gs, d_go = [], [], [], [], []
+    for k in range(len(w.tensors)):
+        th, t0, g = W.generate_tensor(w, k, dev)
+        a, b = int(offs[k]), int(offs[k + 1])
+        h_th[a:b].copy_(th)
+        h_t0[a:b].copy_(t0)
+        h_gs[a:b].copy_(g)
+        d_th.append(th)
+        d_t0.append(t0)
+        d_gs.append(g)
+        d_sim.append(torch.empty_like(th))
+        d_go.append(torch.empty_like(g))
+    sess = sess_factory(d_th, d_t0, d_sim)
+    hv = lambda h: [h[int(offs[k]):int(offs[k + 1])] for k in range(len(w.tensors))]  # noqa: E731
+    hth, ht0, hgs, hsim, hgo = hv(h_th), hv(h_t0), hv(h_gs), hv(h_sim), hv(h_go)
+
+    def one(step):
+        for k in range(len(w.tensors)):
+            d_th[k].copy_(hth[k], non_blocking=True)
+            d_t0[k].copy_(ht0[k], non_blocking=True)
+            d_gs[k].copy_(hgs[k], non_blocking=True)
+        sess.simulate_multi(step)
+        sess.swap()
+        sess.grad_map_multi(step, d_gs, d_go)
+        sess.swap()
+        for k in range(len(w.tensors)):
+            hsim[k].copy_(d_sim[k], non_blocking=True)
+            hgo[k].copy_(d_go[k], non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+
+    for s in range(warmup):
+        one(s)
+    barrier(world)
+    torch.cuda.synchronize()
+    a = time.perf_counter()
+    for s in range(steps):
+        one(1000 + s)
+    torch.cuda.synchronize()
+    el = max_over_ranks(time.perf_counter() - a, world)
+    bytes_step = sum(step_bytes(w).values())
+    h2d = 2 * h_th.element_size() * n + h_gs.element_size() * n
+    d2h = h_sim.element_size() * n + h_go.element_size() * n
+    sess.close()
+    return {"value": world * bytes_step * steps / el / 1e9, "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": 1e3 * el / steps, "workload": w.name}
+
+
+def run_smat(args):
+    world, rank, local = dist_setup(args)
+    from paper_2609_33437_gb300 import smat as S
+    S.load_library()
+    dev = torch.device("cuda", local)
+    w = workload(args)
+    w.seed = rank  # each rank: an independent expert
+    w.data_seed = w.data_seed + 1000 * rank
+
+    def make_session(th, t0, sim):
+        return S.SmatSession(th, t0, sim, [t.keep_prob for t in w.tensors], [t.sigma for t in w.tensors],
+                             [t.sigma_rel for t in w.tensors], seed=w.seed, alpha_min=w.alpha_min,
+                             alpha_max=w.alpha_max, alpha_mode=w.alpha_mode, noise=w.noise)
+
+    th, t0, sim, gs, go = W.generate(w, device=dev)
+    sess = make_session(th, t0, sim)
+
+    def step(s):
+        sess.simulate_multi(s)
+        sess.swap()
+        sess.grad_map_multi(s, gs, go)
+        sess.swap()
+
+    for s in range(args.warmup):
+        step(s)
+    torch.cuda.synchronize()
+    clocks = None if args.no_clocks else ClockSampler(local)
+    if clocks:
+        time.sleep(0.3)
+    barrier(world)
+    torch.cuda.synchronize()
+    sess.timing_enable(True)
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if clocks:
+        clocks.mark()
+    e0.record(stream)
+    for s in range(args.steps):
+        step(100 + s)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if clocks:
+        clocks.mark()
+    barrier(world)
+    ms = e0.elapsed_time(e1)
+    kern = sess.timing_read()
+    sess.timing_enable(False)
+    clk = clocks.stop() if clocks else None
+    ms_step = max_over_ranks(ms / args.steps, world)
+
+    nb = step_bytes(w)
+    bytes_step = sum(nb.values())
+    value = world * bytes_step / (ms_step * 1e-3) / 1e9
+    peak, peak_kind = measured_peaks()
+    sim_ms, sim_n = kern["simulate"]
+    sim_avg = sim_ms / max(1, sim_n)
+    achieved = nb["simulate"] / (sim_avg * 1e-3) / 1e9
+    traffic = recorded_traffic("simulate", w.name)
+    per_kernel = {}
+    for k, (kms, kn) in kern.items():
+        if kn == 0:
+            continue
+        per_kernel[k] = {"avg_ms": kms / kn, "launches": kn, "share": kms / max(1e-9, sum(v[0] for v in kern.values()))}
+        if k in nb and nb[k]:
+            per_kernel[k]["gbs"] = nb[k] / (kms / kn * 1e-3) / 1e9
+            per_kernel[k]["frac_of_measured_peak"] = per_kernel[k]["gbs"] / peak
+    launches = int(sum(v[1] for v in kern.values()))
+    del sess
+    out = None
+    if rank == 0:
+        out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+               "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+               "vs_baseline": None, "dtype": "bf16" if w.dtype == W.BF16 else "f32",
+               "data": "synthetic (seeded torch draws shaped like a 7B Llama-style parameter list)",
+               "params_per_s": world * w.numel / (ms_step * 1e-3),
+               "frac_of_measured_peak": value / peak, "frac_of_nominal_8tbs": value / NOMINAL_HBM_GBS,
+               "config": {"workload": w.name, "tensors": len(w.tensors), "elements": w.numel,
+                          "param_dtype": "bf16" if w.dtype == W.BF16 else "f32",
+                          "grad_dtype": "bf16" if w.gdtype == W.BF16 else "f32",
+                          "noise": "gaussian" if w.noise == 1 else "uniform", "alpha": f"per-tensor U[{w.alpha_min}, {w.alpha_max})",
+                          "bytes_per_step": bytes_step, "l2": "inputs larger than L2 (no flush needed)",
+                          "parallelism": f"{world} independent experts (one per GPU)"},
+               "kernels": per_kernel,
+               "roofline": {"bound": "hbm", "kernel": "simulate", "achieved": achieved, "peak": peak,
+                            "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
+                            "traffic": traffic["dram_bytes_per_launch"] if traffic else None,
+                            "algorithmic_bytes_per_launch": nb["simulate"]},
+               "clocks": clk, "gpu_launches": launches}
+    if not args.no_e2e:
+        need = 5 * 2 * w.numel
+        avail = host_available_bytes() / max(1, world)
+        ew = w
+        if need > 0.5 * avail:
+            ew = W.scaled(w, int(0.5 * avail / 10))
+        del th, t0, sim, gs, go
+        torch.cuda.empty_cache()
+        e2e = e2e_run(ew, make_session, steps=max(1, min(args.steps, 3)), warmup=1, world=world)
+        if out is not None:
+            out["e2e"] = e2e
+    if out is not None and not args.no_cpu_baseline and world == 1:
+        secs, b, n, sample = oracle_run(w, 48_000_000)
+        out["cpu_baseline"] = {"value": b / secs / 1e9, "unit": UNIT, "cores": 1, "kind": "oracle",
+                               "sample": f"{sample} (single-threaded C++ oracle, forward + gradient map, "
+                                         f"{secs:.1f} s)", "params_per_s": n / secs}
+    if out is not None:
+        print(json.dumps(out))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_smat(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,198 @@
+/*
+ * smat.h — C ABI of the SMAT simulated-merge library (libsmat.so), GB300 / sm_103a.
+ *
+ * The library implements the data-parallel hot path of SMAT merge-aware
+ * training ("SMAT: Simple and Efficient Merge-Aware Training"):
+ *
+ *   forward   theta~ = theta0 + alpha * m (.) (theta - theta0) + eps
+ *             Eq. smat-state (Sec. 4.1) with Scale (alpha ~ U[alpha_min, 1]),
+ *             Mask (Eq. smat-mask: m_k = 0 w.p. p_k, 1/(1-p_k) otherwise) and
+ *             Perturb (eps uniform on [-sqrt3 sigma, sqrt3 sigma], Sec. 4.1;
+ *             a Gaussian N(0, sigma^2) variant is also provided);
+ *   gradient  g = alpha * m (.) g~          Eq. smat-gradient (Sec. 4.2), with
+ *             the mask regenerated rather than stored (App. D, implementation
+ *             details);
+ *   swap      which of theta / theta~ the model reads (Sec. 4.3, parameter
+ *             storage switching; App. E).
+ *
+ * Random draws come from counter-based Philox-4x32 streams keyed by
+ * (seed, step, tensor id, element index), so any element can be regenerated
+ * and the result does not depend on launch geometry or sharding.
+ *
+ * Conventions for every entry point:
+ *   - All device memory (parameters, outputs, gradients, the workspace) is
+ *     allocated and owned by the caller. The library never allocates device
+ *     memory; it owns only the host-side context object.
+ *   - Work is enqueued asynchronously on the caller's stream (`smat_stream_t`
+ *     is the CUDA runtime's cudaStream_t; NULL means the legacy default
+ *     stream). All calls on one context must be ordered on the device by the
+ *     caller (same stream, or explicit synchronisation).
+ *   - Every function returns a status code; none aborts or throws. Arguments
+ *     are validated on the host before anything is enqueued. A failed launch
+ *     returns SMAT_ERR_CUDA; an asynchronous device fault surfaces at the
+ *     caller's next synchronisation. smat_last_error() returns a message
+ *     describing the last failure on the calling thread.
+ *   - Alignment: every pointer must be aligned to its element size
+ *     (SMAT_ERR_ALIGNMENT otherwise). Tensors whose pointers are 32-byte
+ *     aligned and whose elem_offset is a multiple of 16 take the vectorised
+ *     (256-bit) path; any other tensor takes a per-element path with
+ *     identical results.
+ */
+#ifndef SMAT_H
+#define SMAT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SMAT_ABI_VERSION 1
+
+typedef struct CUstream_st* smat_stream_t; /* == cudaStream_t */
+typedef struct smat_ctx smat_ctx;          /* opaque host-side context */
+
+typedef enum {
+  SMAT_OK = 0,
+  SMAT_ERR_INVALID_ARG = 1, /* null pointer, bad size or out-of-range parameter */
+  SMAT_ERR_UNSUPPORTED = 2, /* unsupported dtype, mode or Philox round count */
+  SMAT_ERR_ALIGNMENT = 3,   /* pointer not aligned to its element size */
+  SMAT_ERR_WORKSPACE = 4,   /* workspace null, too small or misaligned */
+  SMAT_ERR_STATE = 5,       /* call not allowed in the context's current state */
+  SMAT_ERR_CUDA = 6         /* a CUDA runtime call or kernel launch failed */
+} smat_status;
+
+typedef enum { SMAT_F32 = 0, SMAT_BF16 = 1 } smat_dtype;
+
+/* Perturb law. Uniform on [-sqrt3 sigma, sqrt3 sigma] is the paper's (Sec. 4.1). */
+typedef enum { SMAT_NOISE_UNIFORM = 0, SMAT_NOISE_GAUSSIAN = 1 } smat_noise;
+
+/* Scale granularity. The paper shares one alpha across all coordinates
+ * (Sec. 4.1, App. A): SMAT_ALPHA_GLOBAL. Per tensor and per element are
+ * finer-grained variants. */
+typedef enum {
+  SMAT_ALPHA_GLOBAL = 0,
+  SMAT_ALPHA_PER_TENSOR = 1,
+  SMAT_ALPHA_PER_ELEMENT = 2
+} smat_alpha_mode;
+
+/* One trainable tensor. theta (the expert's parameters, read), theta0 (the
+ * shared initialisation, read) and sim (theta~, written) are device pointers
+ * of `numel` elements of `dtype`, contiguous; they must stay valid from
+ * smat_init to smat_destroy. sim must not overlap theta or theta0. */
+typedef struct {
+  const void* theta;
+  const void* theta0;
+  void* sim;
+  int64_t numel;       /* >= 0, < 2^40 */
+  int64_t elem_offset; /* global index of element 0 within the full tensor (sharding); >= 0 */
+  uint32_t tensor_id;  /* < 0x0FFFFFFF, unique within the context, stable across calls */
+  int32_t dtype;       /* smat_dtype of theta, theta0 and sim */
+  float keep_prob;     /* p_keep = 1 - p in [0, 1] (Eq. smat-mask); 1 = outside the masked set */
+  float sigma;         /* Perturb RMS >= 0 (used when sigma_rel == 0) */
+  float sigma_rel;     /* >= 0; if > 0, sigma_t = sigma_rel * std(theta - theta0) at each call */
+} smat_tensor_desc;
+
+typedef struct {
+  uint64_t seed;         /* Philox key */
+  float alpha_min;       /* Scale: alpha ~ U[alpha_min, alpha_max); paper: alpha_max = 1 */
+  float alpha_max;       /* alpha_min <= alpha_max, both finite */
+  int32_t alpha_mode;    /* smat_alpha_mode */
+  int32_t noise;         /* smat_noise */
+  int32_t philox_rounds; /* 10 (default) or 7 */
+} smat_config;
+
+/* Bytes of device workspace smat_init needs for this tensor list (0 on
+ * invalid arguments). The workspace holds the device tensor table, the chunk
+ * table, per-call scalars, statistics partials and the gradient pointer table. */
+size_t smat_workspace_bytes(const smat_tensor_desc* tensors, int32_t n_tensors,
+                            const smat_config* cfg);
+
+/* Validate the list, build the tables and upload them into d_workspace on
+ * `stream`. d_workspace: caller-owned device memory of at least
+ * smat_workspace_bytes(...) bytes, 256-byte aligned, untouched by the caller
+ * until smat_destroy. On success *out receives a new context, initially with
+ * the original storage (theta) active. */
+smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n_tensors,
+                      const smat_config* cfg, void* d_workspace, size_t workspace_bytes,
+                      smat_stream_t stream);
+
+/* Forward (Eq. smat-state) for every tensor at SMAT step `step`: computes the
+ * per-call scalars (and, for sigma_rel tensors, the delta statistics first)
+ * and writes theta~ into each tensor's `sim`. Requires the original storage to
+ * be active (SMAT_ERR_STATE otherwise): the simulated state is rebuilt only
+ * while the model reads theta. */
+smat_status smat_simulate_multi(smat_ctx* ctx, uint32_t step, smat_stream_t stream);
+
+/* Gradient map (Eq. smat-gradient) at step `step`: for tensor k,
+ * g_out[k][i] = alpha m_i g_sim[k][i] (rounded to gdtype), or
+ * g_out[k][i] + alpha m_i g_sim[k][i] when accumulate != 0. g_sim and g_out are
+ * HOST arrays of n_tensors DEVICE pointers (numel elements of gdtype each,
+ * same order as the descriptors; an entry may be NULL only if numel == 0).
+ * g_out[k] may equal g_sim[k] (in place). The pointer table is uploaded only
+ * when it differs from the previous call's. The mask is regenerated from the
+ * stream, never stored. */
+smat_status smat_grad_map_multi(smat_ctx* ctx, uint32_t step, const void* const* g_sim,
+                                void* const* g_out, int32_t gdtype, int32_t accumulate,
+                                smat_stream_t stream);
+
+/* Parameter storage switch (Sec. 4.3): flips the active storage and returns
+ * it in *active_out (0 = theta, the original storage; 1 = sim, theta~).
+ * Host only: no device work, no copy. */
+smat_status smat_swap(smat_ctx* ctx, int32_t* active_out);
+
+/* Which storage is active (0 = theta, 1 = sim). */
+smat_status smat_active(const smat_ctx* ctx, int32_t* active_out);
+
+/* Test hook: packed keep bits of tensor `tensor_index` at `step` into the
+ * device buffer d_bits of ceil(numel / 32) uint32 words; bit (i mod 32) of
+ * word i / 32 is 1 iff local element i is kept (LSB first; high bits of the
+ * last word 0). */
+smat_status smat_mask_bits(smat_ctx* ctx, uint32_t step, int32_t tensor_index, uint32_t* d_bits,
+                           smat_stream_t stream);
+
+/* Test hook: per-call scalars at `step` into the device buffer d_out of
+ * 4 * n_tensors floats: {alpha_t, c_t = alpha_t / p_keep, sigma_t,
+ * noise scale} per tensor (alpha_t and c_t are 0 in per-element mode).
+ * Computes the delta statistics first for sigma_rel tensors. */
+smat_status smat_tensor_scalars(smat_ctx* ctx, uint32_t step, float* d_out, smat_stream_t stream);
+
+/* Release the host context (the caller still owns and frees the workspace
+ * once the stream's work has finished). NULL is accepted. */
+smat_status smat_destroy(smat_ctx* ctx);
+
+/* Test hook: evaluate n Philox-4x32 blocks on the device. d_ctr: device array
+ * of 4 n uint32 counters; d_out: 4 n uint32 words from this library's Philox
+ * with `rounds` rounds and key (seed mod 2^32, seed div 2^32); d_out_ref (may
+ * be NULL, rounds must then be any supported value): 4 n words from cuRAND's
+ * curand_Philox4x32_10 on the same inputs (requires rounds == 10). */
+smat_status smat_debug_philox(const uint32_t* d_ctr, int64_t n, uint64_t seed, int32_t rounds,
+                              uint32_t* d_out, uint32_t* d_out_ref, smat_stream_t stream);
+
+/* Per-kernel timing (for measurement): while enabled, every kernel this
+ * context launches is bracketed by two CUDA events recorded on the launching
+ * stream. Kinds: 0 delta statistics (a2), 1 per-call scalars (a1),
+ * 2 forward (a3), 3 gradient map (a5). Enabling clears the totals. Host-side
+ * events only; no device memory is allocated. */
+smat_status smat_timing_enable(smat_ctx* ctx, int32_t enable);
+
+/* Wait for the recorded events and return, per kind, the summed kernel time
+ * in milliseconds (ms_out[4]) and the number of launches (launches_out[4])
+ * since timing was enabled. Either output may be NULL. */
+smat_status smat_timing_read(smat_ctx* ctx, double* ms_out, int64_t* launches_out);
+
+/* Static description of a status code. */
+const char* smat_status_string(smat_status s);
+
+/* Message describing the last failure on the calling thread ("" if none). */
+const char* smat_last_error(void);
+
+/* SMAT_ABI_VERSION of the loaded library. */
+int32_t smat_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SMAT_H */

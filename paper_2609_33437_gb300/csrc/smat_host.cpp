@@ -1,0 +1,550 @@
+// Host side of libsmat: argument validation, device tables, launches.
+// The C ABI is declared in include/smat.h.
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <unordered_set>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "smat.h"
+#include "smat_internal.h"
+
+using namespace smat;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+smat_status fail(smat_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  std::vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return s;
+}
+
+smat_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(SMAT_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+constexpr size_t kAlign = 256;
+size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+size_t elem_size(int32_t dt) { return dt == SMAT_BF16 ? 2 : 4; }
+constexpr int64_t kMaxNumel = int64_t(1) << 40;
+
+struct Layout {
+  size_t tensors, chunks, scal, partials, grads, total;
+};
+
+int64_t chunks_of(int64_t numel) { return (numel + kChunkElems - 1) / kChunkElems; }
+
+Layout layout_for(int32_t n, int64_t n_chunks, bool any_sigma_rel) {
+  Layout L;
+  size_t off = 0;
+  L.tensors = off; off = align_up(off + sizeof(DevTensor) * (size_t)n);
+  L.chunks = off;  off = align_up(off + sizeof(Chunk) * (size_t)n_chunks);
+  L.scal = off;    off = align_up(off + sizeof(DevScalars) * (size_t)n);
+  L.partials = off; off = align_up(off + (any_sigma_rel ? sizeof(StatPartial) * (size_t)n_chunks : 0));
+  L.grads = off;   off = align_up(off + sizeof(GradPtr) * (size_t)n);
+  L.total = off;
+  return L;
+}
+
+bool finite(float x) { return std::isfinite(x); }
+
+smat_status check_config(const smat_config* cfg) {
+  if (!cfg) return fail(SMAT_ERR_INVALID_ARG, "cfg is NULL");
+  if (cfg->alpha_mode < SMAT_ALPHA_GLOBAL || cfg->alpha_mode > SMAT_ALPHA_PER_ELEMENT)
+    return fail(SMAT_ERR_UNSUPPORTED, "alpha_mode %d not supported", cfg->alpha_mode);
+  if (cfg->noise != SMAT_NOISE_UNIFORM && cfg->noise != SMAT_NOISE_GAUSSIAN)
+    return fail(SMAT_ERR_UNSUPPORTED, "noise %d not supported", cfg->noise);
+  if (cfg->philox_rounds != 0 && cfg->philox_rounds != 7 && cfg->philox_rounds != 10)
+    return fail(SMAT_ERR_UNSUPPORTED, "philox_rounds %d not supported (7 or 10)", cfg->philox_rounds);
+  if (!finite(cfg->alpha_min) || !finite(cfg->alpha_max) || cfg->alpha_min > cfg->alpha_max)
+    return fail(SMAT_ERR_INVALID_ARG, "alpha range [%g, %g) invalid", cfg->alpha_min, cfg->alpha_max);
+  return SMAT_OK;
+}
+
+bool overlaps(const void* a, size_t abytes, const void* b, size_t bbytes) {
+  const uintptr_t x = (uintptr_t)a, y = (uintptr_t)b;
+  return x < y + bbytes && y < x + abytes;
+}
+
+smat_status check_tensors(const smat_tensor_desc* t, int32_t n, int64_t* n_chunks, bool* any_rel) {
+  if (n < 0) return fail(SMAT_ERR_INVALID_ARG, "n_tensors %d < 0", n);
+  if (n > 0 && !t) return fail(SMAT_ERR_INVALID_ARG, "tensors is NULL");
+  std::unordered_set<uint32_t> ids;
+  int64_t nc = 0;
+  bool rel = false;
+  for (int32_t k = 0; k < n; ++k) {
+    const smat_tensor_desc& d = t[k];
+    if (d.numel < 0 || d.numel >= kMaxNumel)
+      return fail(SMAT_ERR_INVALID_ARG, "tensor %d: numel %lld out of range", k, (long long)d.numel);
+    if (d.elem_offset < 0 || d.elem_offset >= (int64_t(1) << 62) - d.numel)
+      return fail(SMAT_ERR_INVALID_ARG, "tensor %d: elem_offset %lld out of range", k, (long long)d.elem_offset);
+    if (d.tensor_id >= kGlobalAlphaTensor)
+      return fail(SMAT_ERR_INVALID_ARG, "tensor %d: tensor_id %u >= 0x0FFFFFFF", k, d.tensor_id);
+    if (!ids.insert(d.tensor_id).second)
+      return fail(SMAT_ERR_INVALID_ARG, "tensor %d: duplicate tensor_id %u", k, d.tensor_id);
+    if (d.dtype != SMAT_F32 && d.dtype != SMAT_BF16)
+      return fail(SMAT_ERR_UNSUPPORTED, "tensor %d: dtype %d not supported", k, d.dtype);
+    if (!(d.keep_prob >= 0.0f && d.keep_prob <= 1.0f))
+      return fail(SMAT_ERR_INVALID_ARG, "tensor %d: keep_prob %g not in [0, 1]", k, d.keep_prob);
+    if (!finite(d.sigma) || d.sigma < 0.0f)
+      return fail(SMAT_ERR_INVALID_ARG, "tensor %d: sigma %g invalid", k, d.sigma);
+    if (!finite(d.sigma_rel) || d.sigma_rel < 0.0f)
+      return fail(SMAT_ERR_INVALID_ARG, "tensor %d: sigma_rel %g invalid", k, d.sigma_rel);
+    if (d.numel > 0) {
+      if (!d.theta || !d.theta0 || !d.sim)
+        return fail(SMAT_ERR_INVALID_ARG, "tensor %d: NULL data pointer", k);
+      const size_t es = elem_size(d.dtype);
+      if ((uintptr_t)d.theta % es || (uintptr_t)d.theta0 % es || (uintptr_t)d.sim % es)
+        return fail(SMAT_ERR_ALIGNMENT, "tensor %d: pointer not aligned to %zu bytes", k, es);
+      const size_t bytes = es * (size_t)d.numel;
+      if (overlaps(d.sim, bytes, d.theta, bytes) || overlaps(d.sim, bytes, d.theta0, bytes))
+        return fail(SMAT_ERR_INVALID_ARG, "tensor %d: sim overlaps theta or theta0", k);
+    }
+    nc += chunks_of(d.numel);
+    rel = rel || d.sigma_rel > 0.0f;
+  }
+  if (nc >= (int64_t(1) << 31)) return fail(SMAT_ERR_INVALID_ARG, "too many chunks (%lld)", (long long)nc);
+  *n_chunks = nc;
+  *any_rel = rel;
+  return SMAT_OK;
+}
+
+RoundKeys make_keys(uint64_t seed) {
+  RoundKeys k;
+  uint32_t a = (uint32_t)(seed & 0xFFFFFFFFu), b = (uint32_t)(seed >> 32);
+  for (int r = 0; r < kMaxRounds; ++r) {
+    k.k0[r] = a;
+    k.k1[r] = b;
+    a += 0x9E3779B9u;  // Weyl increments of the Philox key schedule
+    b += 0xBB67AE85u;
+  }
+  return k;
+}
+
+}  // namespace
+
+struct smat_ctx {
+  std::vector<smat_tensor_desc> desc;
+  smat_config cfg;
+  int rounds = 10;
+  std::vector<DevTensor> h_tensors;
+  std::vector<Chunk> h_chunks;
+  int64_t range_begin[2] = {0, 0};  // chunk range per dtype (F32, BF16)
+  int64_t range_end[2] = {0, 0};
+  bool any_sigma_rel = false;
+  DevTensor* d_tensors = nullptr;
+  Chunk* d_chunks = nullptr;
+  DevScalars* d_scal = nullptr;
+  StatPartial* d_partials = nullptr;
+  GradPtr* d_grads = nullptr;
+  RoundKeys keys;
+  int sm_count = 1;
+  int32_t active = 0;
+  int64_t scalars_step = -1;  // step whose scalars the table holds
+  bool scalars_sigma = false; // the table's sigma_t are current
+  std::vector<GradPtr> h_grads;
+  bool grads_uploaded = false;
+  // optional per-kernel timing
+  bool timing = false;
+  struct Mark { int kind; cudaEvent_t start, stop; };
+  std::vector<Mark> marks;
+  std::vector<cudaEvent_t> event_pool;
+  double ms[4] = {0, 0, 0, 0};
+  int64_t launches[4] = {0, 0, 0, 0};
+  ~smat_ctx() {
+    for (auto& m : marks) { event_pool.push_back(m.start); event_pool.push_back(m.stop); }
+    for (cudaEvent_t e : event_pool) cudaEventDestroy(e);
+  }
+};
+
+namespace {
+
+cudaEvent_t take_event(smat_ctx* c) {
+  if (!c->event_pool.empty()) {
+    cudaEvent_t e = c->event_pool.back();
+    c->event_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+// Bracket one launch with events on its stream when timing is enabled.
+struct Timed {
+  smat_ctx* c;
+  int kind;
+  cudaStream_t s;
+  cudaEvent_t start = nullptr;
+  Timed(smat_ctx* c_, int kind_, cudaStream_t s_) : c(c_), kind(kind_), s(s_) {
+    if (c->timing && (start = take_event(c)) != nullptr) cudaEventRecord(start, s);
+  }
+  void done() {
+    if (!start) return;
+    cudaEvent_t stop = take_event(c);
+    if (!stop) { c->event_pool.push_back(start); return; }
+    cudaEventRecord(stop, s);
+    c->marks.push_back({kind, start, stop});
+  }
+};
+
+KArgs base_args(const smat_ctx* c, uint32_t step) {
+  KArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.tensors = c->d_tensors;
+  a.chunks = c->d_chunks;
+  a.scal = c->d_scal;
+  a.partials = c->d_partials;
+  a.grads = c->d_grads;
+  a.key = c->keys;
+  a.step = step;
+  a.n_tensors = (int32_t)c->desc.size();
+  a.alpha_min = c->cfg.alpha_min;
+  a.alpha_width = c->cfg.alpha_max - c->cfg.alpha_min;
+  a.alpha_mode = c->cfg.alpha_mode;
+  return a;
+}
+
+int grid_for(const smat_ctx* c, int64_t chunks, int dtype) {
+  const int64_t resident = (int64_t)c->sm_count *
+                           streaming_ctas_per_sm(dtype, c->cfg.noise, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT, c->rounds);
+  return (int)(chunks < resident ? chunks : resident);
+}
+
+// Rows a2 + a1: delta statistics (if needed) then the per-call scalars.
+smat_status run_scalars(smat_ctx* c, uint32_t step, bool with_sigma, cudaStream_t s) {
+  KArgs a = base_args(c, step);
+  cudaError_t e;
+  const bool stats = with_sigma && c->any_sigma_rel;
+  if (stats) {
+    for (int dt = 0; dt < 2; ++dt) {
+      a.chunk_begin = c->range_begin[dt];
+      a.chunk_end = c->range_end[dt];
+      if (a.chunk_end <= a.chunk_begin) continue;
+      Timed t(c, 0, s);
+      e = launch_delta_stats(a, grid_for(c, a.chunk_end - a.chunk_begin, dt), dt, s);
+      t.done();
+      if (e != cudaSuccess) return cuda_fail(e, "delta statistics launch");
+    }
+  }
+  a.chunk_begin = 0;
+  a.chunk_end = 0;
+  a.with_sigma = stats ? 1 : 0;
+  if (a.n_tensors == 0) return SMAT_OK;
+  Timed t(c, 1, s);
+  e = launch_scalars(a, c->cfg.noise, c->rounds, s);
+  t.done();
+  if (e != cudaSuccess) return cuda_fail(e, "scalars launch");
+  c->scalars_step = step;
+  c->scalars_sigma = with_sigma;
+  return SMAT_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t smat_workspace_bytes(const smat_tensor_desc* tensors, int32_t n_tensors, const smat_config* cfg) {
+  if (check_config(cfg) != SMAT_OK) return 0;
+  int64_t nc = 0;
+  bool rel = false;
+  if (check_tensors(tensors, n_tensors, &nc, &rel) != SMAT_OK) return 0;
+  return layout_for(n_tensors, nc, rel).total;
+}
+
+smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n_tensors,
+                      const smat_config* cfg, void* d_workspace, size_t workspace_bytes,
+                      smat_stream_t stream) {
+  if (!out) return fail(SMAT_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  smat_status st = check_config(cfg);
+  if (st != SMAT_OK) return st;
+  int64_t nc = 0;
+  bool rel = false;
+  st = check_tensors(tensors, n_tensors, &nc, &rel);
+  if (st != SMAT_OK) return st;
+  const Layout L = layout_for(n_tensors, nc, rel);
+  if (!d_workspace) return fail(SMAT_ERR_WORKSPACE, "workspace is NULL");
+  if ((uintptr_t)d_workspace % kAlign) return fail(SMAT_ERR_WORKSPACE, "workspace not 256-byte aligned");
+  if (workspace_bytes < L.total)
+    return fail(SMAT_ERR_WORKSPACE, "workspace %zu bytes < %zu needed", workspace_bytes, L.total);
+
+  smat_ctx* c = new smat_ctx();
+  c->desc.assign(tensors, tensors + n_tensors);
+  c->cfg = *cfg;
+  c->rounds = cfg->philox_rounds == 7 ? 7 : 10;
+  c->any_sigma_rel = rel;
+  c->keys = make_keys(cfg->seed);
+  char* ws = static_cast<char*>(d_workspace);
+  c->d_tensors = reinterpret_cast<DevTensor*>(ws + L.tensors);
+  c->d_chunks = reinterpret_cast<Chunk*>(ws + L.chunks);
+  c->d_scal = reinterpret_cast<DevScalars*>(ws + L.scal);
+  c->d_partials = rel ? reinterpret_cast<StatPartial*>(ws + L.partials) : nullptr;
+  c->d_grads = reinterpret_cast<GradPtr*>(ws + L.grads);
+
+  c->h_tensors.resize(n_tensors);
+  c->h_chunks.reserve((size_t)nc);
+  for (int dt = 0; dt < 2; ++dt) {
+    c->range_begin[dt] = (int64_t)c->h_chunks.size();
+    for (int32_t k = 0; k < n_tensors; ++k) {
+      const smat_tensor_desc& d = tensors[k];
+      if (d.dtype != dt) continue;
+      DevTensor& T = c->h_tensors[k];
+      std::memset(&T, 0, sizeof(T));
+      T.theta = d.theta;
+      T.theta0 = d.theta0;
+      T.sim = d.sim;
+      T.numel = d.numel;
+      T.elem_offset = d.elem_offset;
+      T.tid = d.tensor_id;
+      T.dtype = d.dtype;
+      T.sigma = d.sigma;
+      T.sigma_rel = d.sigma_rel;
+      // Eq. smat-mask: keep with probability p_keep = 1 - p, rescale by 1 / p_keep.
+      const uint64_t thr = (uint64_t)std::floor((double)d.keep_prob * 4294967296.0);
+      T.inv_keep = d.keep_prob > 0.0f ? (float)(1.0 / (double)d.keep_prob) : 0.0f;
+      uint32_t flags = 0;
+      if (thr < (uint64_t(1) << 32)) {
+        flags |= TF_MASK;
+        T.t_hi = (uint32_t)(thr >> 24);
+        T.t_lo = (uint32_t)(thr & 0xFFFFFFu);
+      }
+      // 256-bit vector accesses need 32-byte aligned addresses; groups of 16
+      // elements start at multiples of 16 elements from the base pointer.
+      if (((uintptr_t)d.theta % 32 == 0) && ((uintptr_t)d.theta0 % 32 == 0) &&
+          ((uintptr_t)d.sim % 32 == 0) && (d.elem_offset % 16 == 0))
+        flags |= TF_VEC;
+      if (d.sigma_rel > 0.0f) flags |= TF_SIGMA_REL;
+      T.flags = flags;
+      T.chunk_first = (int32_t)c->h_chunks.size();
+      const int64_t m = chunks_of(d.numel);
+      T.n_chunks = (int32_t)m;
+      for (int64_t j = 0; j < m; ++j) {
+        Chunk ch;
+        ch.tensor = k;
+        ch.pad = 0;
+        ch.begin = j * kChunkElems;
+        ch.end = (j + 1) * kChunkElems < d.numel ? (j + 1) * kChunkElems : d.numel;
+        c->h_chunks.push_back(ch);
+      }
+    }
+    c->range_end[dt] = (int64_t)c->h_chunks.size();
+  }
+
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&c->sm_count, cudaDevAttrMultiProcessorCount, dev);
+  if (e == cudaSuccess && n_tensors > 0)
+    e = cudaMemcpyAsync(c->d_tensors, c->h_tensors.data(), sizeof(DevTensor) * (size_t)n_tensors,
+                        cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess && nc > 0)
+    e = cudaMemcpyAsync(c->d_chunks, c->h_chunks.data(), sizeof(Chunk) * (size_t)nc,
+                        cudaMemcpyHostToDevice, stream);
+  // The host vectors are pageable: the copies above have been staged when
+  // they return, but keep the data in the context anyway for its lifetime.
+  if (e != cudaSuccess) {
+    delete c;
+    return cuda_fail(e, "smat_init upload");
+  }
+  *out = c;
+  return SMAT_OK;
+}
+
+smat_status smat_simulate_multi(smat_ctx* c, uint32_t step, smat_stream_t stream) {
+  if (!c) return fail(SMAT_ERR_INVALID_ARG, "ctx is NULL");
+  if (c->active != 0)
+    return fail(SMAT_ERR_STATE, "simulate called while the simulated storage is active; swap back first");
+  smat_status st = run_scalars(c, step, true, stream);
+  if (st != SMAT_OK) return st;
+  KArgs a = base_args(c, step);
+  for (int dt = 0; dt < 2; ++dt) {
+    a.chunk_begin = c->range_begin[dt];
+    a.chunk_end = c->range_end[dt];
+    if (a.chunk_end <= a.chunk_begin) continue;
+    Timed t(c, 2, stream);
+    const cudaError_t e = launch_simulate(a, grid_for(c, a.chunk_end - a.chunk_begin, dt), dt, c->cfg.noise,
+                                          c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT, c->rounds, stream);
+    t.done();
+    if (e != cudaSuccess) return cuda_fail(e, "simulate launch");
+  }
+  return SMAT_OK;
+}
+
+smat_status smat_grad_map_multi(smat_ctx* c, uint32_t step, const void* const* g_sim, void* const* g_out,
+                                int32_t gdtype, int32_t accumulate, smat_stream_t stream) {
+  if (!c) return fail(SMAT_ERR_INVALID_ARG, "ctx is NULL");
+  if (gdtype != SMAT_F32 && gdtype != SMAT_BF16)
+    return fail(SMAT_ERR_UNSUPPORTED, "gradient dtype %d not supported", gdtype);
+  const int32_t n = (int32_t)c->desc.size();
+  if (n > 0 && (!g_sim || !g_out)) return fail(SMAT_ERR_INVALID_ARG, "gradient pointer arrays are NULL");
+  const size_t es = elem_size(gdtype);
+  std::vector<GradPtr> g((size_t)n);
+  for (int32_t k = 0; k < n; ++k) {
+    const smat_tensor_desc& d = c->desc[k];
+    GradPtr& p = g[k];
+    std::memset(&p, 0, sizeof(p));
+    p.g_sim = g_sim[k];
+    p.g_out = g_out[k];
+    if (d.numel > 0) {
+      if (!p.g_sim || !p.g_out) return fail(SMAT_ERR_INVALID_ARG, "tensor %d: NULL gradient pointer", k);
+      if ((uintptr_t)p.g_sim % es || (uintptr_t)p.g_out % es)
+        return fail(SMAT_ERR_ALIGNMENT, "tensor %d: gradient pointer not aligned to %zu bytes", k, es);
+      const size_t bytes = es * (size_t)d.numel;
+      if (p.g_sim != p.g_out && overlaps(p.g_sim, bytes, p.g_out, bytes))
+        return fail(SMAT_ERR_INVALID_ARG, "tensor %d: g_out partially overlaps g_sim", k);
+    }
+    p.vec = ((uintptr_t)p.g_sim % 32 == 0 && (uintptr_t)p.g_out % 32 == 0 && d.elem_offset % 16 == 0) ? 1u : 0u;
+  }
+  if (!c->grads_uploaded || g.size() != c->h_grads.size() ||
+      (n > 0 && std::memcmp(g.data(), c->h_grads.data(), sizeof(GradPtr) * (size_t)n) != 0)) {
+    c->h_grads.swap(g);
+    if (n > 0) {
+      const cudaError_t e = cudaMemcpyAsync(c->d_grads, c->h_grads.data(), sizeof(GradPtr) * (size_t)n,
+                                            cudaMemcpyHostToDevice, stream);
+      if (e != cudaSuccess) return cuda_fail(e, "gradient table upload");
+    }
+    c->grads_uploaded = true;
+  }
+  if (c->scalars_step != (int64_t)step) {
+    const smat_status st = run_scalars(c, step, false, stream);
+    if (st != SMAT_OK) return st;
+  }
+  KArgs a = base_args(c, step);
+  a.chunk_begin = 0;
+  a.chunk_end = (int64_t)c->h_chunks.size();
+  const int64_t resident = (int64_t)c->sm_count *
+                           gradmap_ctas_per_sm(gdtype, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT, accumulate != 0, c->rounds);
+  const int grid = (int)(a.chunk_end < resident ? a.chunk_end : resident);
+  if (a.chunk_end <= 0) return SMAT_OK;
+  Timed t(c, 3, stream);
+  const cudaError_t e = launch_gradmap(a, grid, gdtype, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT,
+                                       accumulate != 0, c->rounds, stream);
+  t.done();
+  if (e != cudaSuccess) return cuda_fail(e, "gradient map launch");
+  return SMAT_OK;
+}
+
+smat_status smat_swap(smat_ctx* c, int32_t* active_out) {
+  if (!c) return fail(SMAT_ERR_INVALID_ARG, "ctx is NULL");
+  c->active ^= 1;
+  if (active_out) *active_out = c->active;
+  return SMAT_OK;
+}
+
+smat_status smat_active(const smat_ctx* c, int32_t* active_out) {
+  if (!c || !active_out) return fail(SMAT_ERR_INVALID_ARG, "NULL argument");
+  *active_out = c->active;
+  return SMAT_OK;
+}
+
+smat_status smat_mask_bits(smat_ctx* c, uint32_t step, int32_t tensor_index, uint32_t* d_bits,
+                           smat_stream_t stream) {
+  if (!c) return fail(SMAT_ERR_INVALID_ARG, "ctx is NULL");
+  if (tensor_index < 0 || tensor_index >= (int32_t)c->desc.size())
+    return fail(SMAT_ERR_INVALID_ARG, "tensor_index %d out of range", tensor_index);
+  const int64_t numel = c->desc[tensor_index].numel;
+  if (numel == 0) return SMAT_OK;
+  if (!d_bits) return fail(SMAT_ERR_INVALID_ARG, "d_bits is NULL");
+  if ((uintptr_t)d_bits % 4) return fail(SMAT_ERR_ALIGNMENT, "d_bits not 4-byte aligned");
+  KArgs a = base_args(c, step);
+  a.bits = d_bits;
+  a.tensor_index = tensor_index;
+  const cudaError_t e = launch_mask_bits(a, numel, c->rounds, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "mask bits launch");
+  return SMAT_OK;
+}
+
+smat_status smat_tensor_scalars(smat_ctx* c, uint32_t step, float* d_out, smat_stream_t stream) {
+  if (!c) return fail(SMAT_ERR_INVALID_ARG, "ctx is NULL");
+  const size_t n = c->desc.size();
+  if (n == 0) return SMAT_OK;
+  if (!d_out) return fail(SMAT_ERR_INVALID_ARG, "d_out is NULL");
+  if ((uintptr_t)d_out % 4) return fail(SMAT_ERR_ALIGNMENT, "d_out not 4-byte aligned");
+  const smat_status st = run_scalars(c, step, true, stream);
+  if (st != SMAT_OK) return st;
+  const cudaError_t e = cudaMemcpyAsync(d_out, c->d_scal, sizeof(DevScalars) * n, cudaMemcpyDeviceToDevice, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "scalars copy");
+  return SMAT_OK;
+}
+
+smat_status smat_timing_enable(smat_ctx* c, int32_t enable) {
+  if (!c) return fail(SMAT_ERR_INVALID_ARG, "ctx is NULL");
+  for (auto& m : c->marks) {
+    c->event_pool.push_back(m.start);
+    c->event_pool.push_back(m.stop);
+  }
+  c->marks.clear();
+  for (int k = 0; k < 4; ++k) {
+    c->ms[k] = 0.0;
+    c->launches[k] = 0;
+  }
+  c->timing = enable != 0;
+  return SMAT_OK;
+}
+
+smat_status smat_timing_read(smat_ctx* c, double* ms_out, int64_t* launches_out) {
+  if (!c) return fail(SMAT_ERR_INVALID_ARG, "ctx is NULL");
+  for (auto& m : c->marks) {
+    cudaError_t e = cudaEventSynchronize(m.stop);
+    float ms = 0.0f;
+    if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, m.start, m.stop);
+    if (e != cudaSuccess) return cuda_fail(e, "timing event");
+    c->ms[m.kind] += ms;
+    c->launches[m.kind] += 1;
+    c->event_pool.push_back(m.start);
+    c->event_pool.push_back(m.stop);
+  }
+  c->marks.clear();
+  for (int k = 0; k < 4; ++k) {
+    if (ms_out) ms_out[k] = c->ms[k];
+    if (launches_out) launches_out[k] = c->launches[k];
+  }
+  return SMAT_OK;
+}
+
+smat_status smat_destroy(smat_ctx* c) {
+  delete c;
+  return SMAT_OK;
+}
+
+smat_status smat_debug_philox(const uint32_t* d_ctr, int64_t n, uint64_t seed, int32_t rounds,
+                              uint32_t* d_out, uint32_t* d_out_ref, smat_stream_t stream) {
+  if (n < 0) return fail(SMAT_ERR_INVALID_ARG, "n < 0");
+  if (n == 0) return SMAT_OK;
+  if (!d_ctr || !d_out) return fail(SMAT_ERR_INVALID_ARG, "NULL pointer");
+  if (rounds != 7 && rounds != 10) return fail(SMAT_ERR_UNSUPPORTED, "rounds %d not supported", rounds);
+  if (d_out_ref && rounds != 10) return fail(SMAT_ERR_UNSUPPORTED, "cuRAND reference needs 10 rounds");
+  const cudaError_t e = launch_debug_philox(d_ctr, n, make_keys(seed), rounds, d_out, d_out_ref, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "philox launch");
+  return SMAT_OK;
+}
+
+const char* smat_status_string(smat_status s) {
+  switch (s) {
+    case SMAT_OK: return "SMAT_OK";
+    case SMAT_ERR_INVALID_ARG: return "SMAT_ERR_INVALID_ARG";
+    case SMAT_ERR_UNSUPPORTED: return "SMAT_ERR_UNSUPPORTED";
+    case SMAT_ERR_ALIGNMENT: return "SMAT_ERR_ALIGNMENT";
+    case SMAT_ERR_WORKSPACE: return "SMAT_ERR_WORKSPACE";
+    case SMAT_ERR_STATE: return "SMAT_ERR_STATE";
+    case SMAT_ERR_CUDA: return "SMAT_ERR_CUDA";
+  }
+  return "SMAT_ERR_UNKNOWN";
+}
+
+const char* smat_last_error(void) { return g_last_error.c_str(); }
+
+int32_t smat_abi_version(void) { return SMAT_ABI_VERSION; }
+
+}  // extern "C"

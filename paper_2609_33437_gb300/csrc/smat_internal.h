@@ -1,0 +1,112 @@
+// Internal layout shared by the host side of libsmat and its kernels.
+// (The CPU oracle has its own, independent definitions.)
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+namespace smat {
+
+// Philox sub-streams (counter word 2 = stream << 28 | tensor id).
+enum : uint32_t { S_MASK = 0, S_NOISE = 1, S_ALPHA_E = 2, S_ALPHA_T = 3, S_MASK_LO = 4 };
+constexpr uint32_t kGlobalAlphaTensor = 0x0FFFFFFFu;
+
+// Elements per work chunk of the multi-tensor launch (a multiple of 16, so a
+// chunk never splits a 16-element mask draw group of an aligned tensor).
+constexpr int64_t kChunkElems = int64_t(1) << 16;
+constexpr int kMaxRounds = 10;
+
+enum : uint32_t {
+  TF_MASK = 1u,       // T = floor(p_keep 2^32) < 2^32: the mask stream is consulted
+  TF_VEC = 2u,        // 32-byte aligned pointers and elem_offset % 16 == 0
+  TF_SIGMA_REL = 4u,  // sigma_t from delta statistics
+};
+
+struct DevTensor {  // 80 bytes
+  const void* theta;
+  const void* theta0;
+  void* sim;
+  int64_t numel;
+  int64_t elem_offset;
+  uint32_t tid;
+  uint32_t flags;
+  uint32_t t_hi;  // keep threshold T >> 24, in [0, 255] when TF_MASK
+  uint32_t t_lo;  // T & 0xFFFFFF
+  float inv_keep; // fl(1 / p_keep), 0 when p_keep == 0
+  float sigma;
+  float sigma_rel;
+  int32_t dtype;
+  int32_t chunk_first;
+  int32_t n_chunks;
+};
+
+struct Chunk {  // 24 bytes
+  int32_t tensor;
+  int32_t pad;
+  int64_t begin;  // local element range [begin, end) of the tensor
+  int64_t end;
+};
+
+struct DevScalars {  // per-call scalars (row a1)
+  float alpha;
+  float c;
+  float sigma;
+  float noise_scale;
+};
+
+struct StatPartial {  // per-chunk delta sums (row a2)
+  double sum;
+  double sumsq;
+};
+
+struct GradPtr {
+  const void* g_sim;
+  void* g_out;
+  uint32_t vec;  // both 32-byte aligned and elem_offset % 16 == 0
+  uint32_t pad;
+};
+
+// Philox round keys, precomputed from the seed on the host.
+struct RoundKeys {
+  uint32_t k0[kMaxRounds];
+  uint32_t k1[kMaxRounds];
+};
+
+struct KArgs {
+  const DevTensor* tensors;
+  const Chunk* chunks;
+  DevScalars* scal;
+  StatPartial* partials;
+  const GradPtr* grads;
+  uint32_t* bits;        // mask_bits output
+  int64_t chunk_begin;   // chunk-table range handled by this launch
+  int64_t chunk_end;
+  RoundKeys key;
+  uint32_t step;
+  int32_t n_tensors;
+  float alpha_min;
+  float alpha_width;     // fl(alpha_max - alpha_min)
+  int32_t alpha_mode;
+  int32_t tensor_index;  // mask_bits: the tensor
+  int32_t with_sigma;    // scalars: 1 = derive sigma_t from the delta-statistics partials
+};
+
+// Kernel launchers (smat_kernels.cu). Each returns the launch's error code.
+cudaError_t launch_delta_stats(const KArgs& a, int grid, int dtype, cudaStream_t s);
+cudaError_t launch_scalars(const KArgs& a, int noise, int rounds, cudaStream_t s);
+cudaError_t launch_simulate(const KArgs& a, int grid, int dtype, int noise, bool per_elem_alpha,
+                            int rounds, cudaStream_t s);
+cudaError_t launch_gradmap(const KArgs& a, int grid, int gdtype, bool per_elem_alpha, bool accumulate,
+                           int rounds, cudaStream_t s);
+cudaError_t launch_mask_bits(const KArgs& a, int64_t numel, int rounds, cudaStream_t s);
+cudaError_t launch_debug_philox(const uint32_t* ctr, int64_t n, const RoundKeys& key, int rounds,
+                                uint32_t* out, uint32_t* out_ref, cudaStream_t s);
+// Resident CTAs per SM of the streaming kernels (for grid sizing).
+int streaming_ctas_per_sm(int dtype, int noise, bool per_elem_alpha, int rounds);
+int gradmap_ctas_per_sm(int gdtype, bool per_elem_alpha, bool accumulate, int rounds);
+
+constexpr int kBlock = 256;
+
+}  // namespace smat

@@ -1,0 +1,293 @@
+"""Thin Python binding of libsmat (include/smat.h).
+
+Argument marshalling only: PyTorch provides device memory and streams, every
+step of the simulated-merge path runs in the library's CUDA kernels. There is
+no CPU fallback: if the library cannot be loaded the calls raise.
+
+Names follow the C ABI: smat_init -> SmatSession(...), smat_simulate_multi ->
+SmatSession.simulate_multi, smat_grad_map_multi -> SmatSession.grad_map_multi,
+smat_swap -> SmatSession.swap, smat_mask_bits -> SmatSession.mask_bits,
+smat_tensor_scalars -> SmatSession.tensor_scalars.
+"""
+
+import ctypes
+import os
+from typing import List, Optional, Sequence
+
+import torch
+
+from . import build as _build
+
+SMAT_F32, SMAT_BF16 = 0, 1
+SMAT_NOISE_UNIFORM, SMAT_NOISE_GAUSSIAN = 0, 1
+SMAT_ALPHA_GLOBAL, SMAT_ALPHA_PER_TENSOR, SMAT_ALPHA_PER_ELEMENT = 0, 1, 2
+
+EXPORTED = ("smat_workspace_bytes", "smat_init", "smat_simulate_multi", "smat_grad_map_multi",
+            "smat_swap", "smat_active", "smat_mask_bits", "smat_tensor_scalars", "smat_destroy",
+            "smat_debug_philox", "smat_timing_enable", "smat_timing_read", "smat_status_string",
+            "smat_last_error", "smat_abi_version")
+
+
+class SmatError(RuntimeError):
+    def __init__(self, func, status, detail):
+        super().__init__(f"{func} failed: {status} ({detail})")
+        self.status = status
+        self.detail = detail
+
+
+class TensorDesc(ctypes.Structure):
+    _fields_ = [("theta", ctypes.c_void_p), ("theta0", ctypes.c_void_p), ("sim", ctypes.c_void_p),
+                ("numel", ctypes.c_int64), ("elem_offset", ctypes.c_int64),
+                ("tensor_id", ctypes.c_uint32), ("dtype", ctypes.c_int32),
+                ("keep_prob", ctypes.c_float), ("sigma", ctypes.c_float), ("sigma_rel", ctypes.c_float)]
+
+
+class Config(ctypes.Structure):
+    _fields_ = [("seed", ctypes.c_uint64), ("alpha_min", ctypes.c_float), ("alpha_max", ctypes.c_float),
+                ("alpha_mode", ctypes.c_int32), ("noise", ctypes.c_int32), ("philox_rounds", ctypes.c_int32)]
+
+
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
+    """Load the in-tree libsmat.so (building it with nvcc if it is missing)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(_build.LIB) or not _build.up_to_date():
+        if not build_if_missing:
+            raise ImportError("libsmat.so is not built; run paper_2609_33437_gb300/build.py")
+        _build.build()
+    L = ctypes.CDLL(_build.LIB)
+    P, I32, I64, U32, U64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32, ctypes.c_uint64
+    L.smat_workspace_bytes.argtypes = [P, I32, P]
+    L.smat_workspace_bytes.restype = ctypes.c_size_t
+    L.smat_init.argtypes = [ctypes.POINTER(P), P, I32, P, P, ctypes.c_size_t, P]
+    L.smat_simulate_multi.argtypes = [P, U32, P]
+    L.smat_grad_map_multi.argtypes = [P, U32, P, P, I32, I32, P]
+    L.smat_swap.argtypes = [P, ctypes.POINTER(I32)]
+    L.smat_active.argtypes = [P, ctypes.POINTER(I32)]
+    L.smat_mask_bits.argtypes = [P, U32, I32, P, P]
+    L.smat_tensor_scalars.argtypes = [P, U32, P, P]
+    L.smat_destroy.argtypes = [P]
+    L.smat_debug_philox.argtypes = [P, I64, U64, I32, P, P, P]
+    L.smat_timing_enable.argtypes = [P, I32]
+    L.smat_timing_read.argtypes = [P, P, P]
+    L.smat_status_string.argtypes = [I32]
+    L.smat_status_string.restype = ctypes.c_char_p
+    L.smat_last_error.argtypes = []
+    L.smat_last_error.restype = ctypes.c_char_p
+    L.smat_abi_version.restype = I32
+    for name in ("smat_init", "smat_simulate_multi", "smat_grad_map_multi", "smat_swap", "smat_active",
+                 "smat_mask_bits", "smat_tensor_scalars", "smat_destroy", "smat_debug_philox",
+                 "smat_timing_enable", "smat_timing_read"):
+        getattr(L, name).restype = I32
+    _lib = L
+    return L
+
+
+def check(func: str, status: int):
+    if status != 0:
+        L = load_library()
+        raise SmatError(func, L.smat_status_string(status).decode(), L.smat_last_error().decode())
+
+
+def dtype_code(dt: torch.dtype) -> int:
+    if dt == torch.float32:
+        return SMAT_F32
+    if dt == torch.bfloat16:
+        return SMAT_BF16
+    raise TypeError(f"unsupported dtype {dt} (float32 or bfloat16)")
+
+
+def _stream_handle(stream: Optional[torch.cuda.Stream]):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+class SmatSession:
+    """One smat_ctx over a list of trainable tensors.
+
+    thetas / theta0s / sims: lists of contiguous CUDA tensors (theta read,
+    theta0 read, sim = theta~ written), same dtype and numel per position.
+    keep_probs, sigmas, sigma_rels: per-tensor p_keep (Eq. smat-mask, 1 - p),
+    Perturb RMS, relative Perturb RMS. The workspace is allocated here with
+    torch and handed to the library.
+    """
+
+    def __init__(self, thetas: Sequence[torch.Tensor], theta0s: Sequence[torch.Tensor],
+                 sims: Sequence[torch.Tensor], keep_probs: Sequence[float], sigmas: Sequence[float],
+                 sigma_rels: Optional[Sequence[float]] = None, tensor_ids: Optional[Sequence[int]] = None,
+                 elem_offsets: Optional[Sequence[int]] = None, seed: int = 0, alpha_min: float = 0.0,
+                 alpha_max: float = 1.0, alpha_mode: int = SMAT_ALPHA_GLOBAL,
+                 noise: int = SMAT_NOISE_UNIFORM, philox_rounds: int = 10,
+                 stream: Optional[torch.cuda.Stream] = None):
+        self._L = load_library()
+        n = len(thetas)
+        if not (len(theta0s) == n and len(sims) == n and len(keep_probs) == n and len(sigmas) == n):
+            raise ValueError("per-tensor lists differ in length")
+        sigma_rels = sigma_rels if sigma_rels is not None else [0.0] * n
+        tensor_ids = tensor_ids if tensor_ids is not None else list(range(n))
+        elem_offsets = elem_offsets if elem_offsets is not None else [0] * n
+        self.n = n
+        self.numels = []
+        descs = (TensorDesc * max(n, 1))()
+        for k in range(n):
+            th, t0, sm = thetas[k], theta0s[k], sims[k]
+            for t in (th, t0, sm):
+                if not t.is_cuda or not t.is_contiguous():
+                    raise ValueError(f"tensor {k}: must be a contiguous CUDA tensor")
+            if th.dtype != t0.dtype or th.dtype != sm.dtype or th.numel() != t0.numel() or th.numel() != sm.numel():
+                raise ValueError(f"tensor {k}: theta / theta0 / sim differ in dtype or numel")
+            d = descs[k]
+            d.theta, d.theta0, d.sim = th.data_ptr(), t0.data_ptr(), sm.data_ptr()
+            d.numel = th.numel()
+            d.elem_offset = int(elem_offsets[k])
+            d.tensor_id = int(tensor_ids[k])
+            d.dtype = dtype_code(th.dtype)
+            d.keep_prob = float(keep_probs[k])
+            d.sigma = float(sigmas[k])
+            d.sigma_rel = float(sigma_rels[k])
+            self.numels.append(th.numel())
+        self._descs = descs
+        self.config = Config(int(seed) & (2**64 - 1), float(alpha_min), float(alpha_max), int(alpha_mode),
+                             int(noise), int(philox_rounds))
+        self.device = thetas[0].device if n else torch.device("cuda", torch.cuda.current_device())
+        nbytes = self._L.smat_workspace_bytes(ctypes.byref(descs), n, ctypes.byref(self.config))
+        if nbytes == 0 and n > 0:
+            # size query failed: let smat_init report the reason
+            nbytes = 256
+        self.workspace = torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=self.device)
+        self._keep = (list(thetas), list(theta0s), list(sims))  # the library holds raw pointers
+        ctx = ctypes.c_void_p()
+        check("smat_init", self._L.smat_init(ctypes.byref(ctx), ctypes.byref(descs), n, ctypes.byref(self.config),
+                                             ctypes.c_void_p(self.workspace.data_ptr()), self.workspace.numel(),
+                                             _stream_handle(stream)))
+        self._ctx = ctx
+        self._gkeep = None
+
+    # -- hot path ------------------------------------------------------------
+    def simulate_multi(self, step: int, stream: Optional[torch.cuda.Stream] = None):
+        check("smat_simulate_multi", self._L.smat_simulate_multi(self._ctx, int(step), _stream_handle(stream)))
+
+    def grad_map_multi(self, step: int, g_sims: Sequence[torch.Tensor], g_outs: Optional[Sequence[torch.Tensor]] = None,
+                       accumulate: bool = False, stream: Optional[torch.cuda.Stream] = None):
+        g_outs = g_sims if g_outs is None else g_outs
+        if len(g_sims) != self.n or len(g_outs) != self.n:
+            raise ValueError("one gradient per tensor expected")
+        gd = None
+        ins = (ctypes.c_void_p * max(self.n, 1))()
+        outs = (ctypes.c_void_p * max(self.n, 1))()
+        for k in range(self.n):
+            a, b = g_sims[k], g_outs[k]
+            if a.numel() != self.numels[k] or b.numel() != self.numels[k] or a.dtype != b.dtype:
+                raise ValueError(f"gradient {k}: numel or dtype mismatch")
+            if not (a.is_cuda and b.is_cuda and a.is_contiguous() and b.is_contiguous()):
+                raise ValueError(f"gradient {k}: must be contiguous CUDA tensors")
+            code = dtype_code(a.dtype)
+            if gd is None:
+                gd = code
+            elif gd != code:
+                raise ValueError("all gradients must share one dtype")
+            ins[k], outs[k] = a.data_ptr(), b.data_ptr()
+        self._gkeep = (list(g_sims), list(g_outs))
+        check("smat_grad_map_multi",
+              self._L.smat_grad_map_multi(self._ctx, int(step), ins, outs, SMAT_F32 if gd is None else gd,
+                                          int(bool(accumulate)), _stream_handle(stream)))
+
+    def swap(self) -> int:
+        a = ctypes.c_int32()
+        check("smat_swap", self._L.smat_swap(self._ctx, ctypes.byref(a)))
+        return a.value
+
+    @property
+    def active(self) -> int:
+        a = ctypes.c_int32()
+        check("smat_active", self._L.smat_active(self._ctx, ctypes.byref(a)))
+        return a.value
+
+    # -- test hooks ----------------------------------------------------------
+    def mask_bits(self, step: int, k: int, stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:
+        words = (self.numels[k] + 31) // 32
+        out = torch.zeros(max(words, 1), dtype=torch.int32, device=self.device)
+        check("smat_mask_bits", self._L.smat_mask_bits(self._ctx, int(step), int(k), ctypes.c_void_p(out.data_ptr()),
+                                                       _stream_handle(stream)))
+        return out[:words]
+
+    def tensor_scalars(self, step: int, stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:
+        out = torch.zeros(max(self.n, 1), 4, dtype=torch.float32, device=self.device)
+        check("smat_tensor_scalars", self._L.smat_tensor_scalars(self._ctx, int(step), ctypes.c_void_p(out.data_ptr()),
+                                                                 _stream_handle(stream)))
+        return out[:self.n]
+
+    def timing_enable(self, enable: bool = True):
+        check("smat_timing_enable", self._L.smat_timing_enable(self._ctx, int(bool(enable))))
+
+    TIMING_KINDS = ("delta_stats", "scalars", "simulate", "gradmap")
+
+    def timing_read(self):
+        """{kind: (total kernel ms, launches)} since timing_enable()."""
+        ms = (ctypes.c_double * 4)()
+        n = (ctypes.c_int64 * 4)()
+        check("smat_timing_read", self._L.smat_timing_read(self._ctx, ms, n))
+        return {k: (ms[i], n[i]) for i, k in enumerate(self.TIMING_KINDS)}
+
+    def close(self):
+        if getattr(self, "_ctx", None):
+            self._L.smat_destroy(self._ctx)
+            self._ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def debug_philox(ctr: torch.Tensor, seed: int, rounds: int = 10, with_curand: bool = True,
+                 stream: Optional[torch.cuda.Stream] = None):
+    """Device Philox blocks for counters ctr (int32 CUDA tensor [n, 4]); also
+    cuRAND's curand_Philox4x32_10 on the same inputs when with_curand."""
+    L = load_library()
+    ctr = ctr.contiguous()
+    n = ctr.shape[0]
+    out = torch.zeros_like(ctr)
+    ref = torch.zeros_like(ctr) if with_curand else None
+    check("smat_debug_philox", L.smat_debug_philox(ctypes.c_void_p(ctr.data_ptr()), n, int(seed) & (2**64 - 1), rounds,
+                                                   ctypes.c_void_p(out.data_ptr()),
+                                                   ctypes.c_void_p(ref.data_ptr() if ref is not None else 0),
+                                                   _stream_handle(stream)))
+    return out, ref
+
+
+class SmatParameters:
+    """Parameter storage switching for a list of torch Parameters (Sec. 4.3):
+    keeps theta0 and one reusable simulated-weight buffer per parameter and
+    rebinds each parameter's storage between theta and theta~ on swap(), with
+    no copy. The optimizer must run with the original storage active."""
+
+    def __init__(self, params: List[torch.nn.Parameter], theta0s: Sequence[torch.Tensor],
+                 keep_probs: Sequence[float], sigmas: Sequence[float], **cfg):
+        self.params = list(params)
+        self.theta = [p.data for p in self.params]
+        self.sims = [torch.empty_like(p.data) for p in self.params]
+        self.session = SmatSession(self.theta, list(theta0s), self.sims, keep_probs, sigmas, **cfg)
+
+    def simulate(self, step: int):
+        self.session.simulate_multi(step)
+
+    def swap(self) -> int:
+        active = self.session.swap()
+        src = self.sims if active == 1 else self.theta
+        for p, t in zip(self.params, src):
+            p.data = t
+        return active
+
+    def grad_map(self, step: int, accumulate: bool = False):
+        gs = [p.grad for p in self.params]
+        self.session.grad_map_multi(step, gs, gs, accumulate=accumulate)

@@ -1,0 +1,154 @@
+"""CPU-only checks of the C ABI: the library loads, exports every function
+include/smat.h declares, sizes its workspace and rejects invalid arguments on
+the host before touching the GPU. No kernel is launched here."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2609_33437_gb300 import smat as S
+from paper_2609_33437_gb300 import workloads as W
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def header_functions():
+    src = open(os.path.join(ROOT, "include", "smat.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(smat_[a-z_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    return S.load_library()
+
+
+def test_library_exports_every_declared_function(L):
+    names = header_functions()
+    assert len(names) >= 13
+    for n in names:
+        assert hasattr(L, n), n
+    assert set(names) == set(S.EXPORTED)
+    assert L.smat_abi_version() == 1
+
+
+def desc(numel=1024, tid=0, dtype=S.SMAT_BF16, keep=0.5, sigma=0.0, rel=0.0, off=0, base=0x10000000):
+    es = 2 if dtype == S.SMAT_BF16 else 4
+    d = S.TensorDesc()
+    d.theta = base
+    d.theta0 = base + 0x1000000 * es
+    d.sim = base + 0x2000000 * es
+    d.numel = numel
+    d.elem_offset = off
+    d.tensor_id = tid
+    d.dtype = dtype
+    d.keep_prob = keep
+    d.sigma = sigma
+    d.sigma_rel = rel
+    return d
+
+
+def cfg(**kw):
+    c = S.Config(0, 0.2, 1.0, S.SMAT_ALPHA_PER_TENSOR, S.SMAT_NOISE_GAUSSIAN, 10)
+    for k, v in kw.items():
+        setattr(c, k, v)
+    return c
+
+
+def arr(*ds):
+    a = (S.TensorDesc * len(ds))()
+    for i, d in enumerate(ds):
+        a[i] = d
+    return a
+
+
+def ws_bytes(L, ds, c):
+    return L.smat_workspace_bytes(ctypes.byref(arr(*ds)), len(ds), ctypes.byref(c))
+
+
+def test_workspace_size_scales_with_chunks(L):
+    small = ws_bytes(L, [desc(1000)], cfg())
+    big = ws_bytes(L, [desc(1 << 24)], cfg())
+    rel = ws_bytes(L, [desc(1 << 24, rel=0.1)], cfg())
+    assert 0 < small < big < rel
+    assert small % 256 == 0 and big % 256 == 0
+    # empty list is valid
+    assert L.smat_workspace_bytes(None, 0, ctypes.byref(cfg())) >= 0
+
+
+@pytest.mark.parametrize("bad,code", [
+    (dict(keep=1.5), 1), (dict(keep=-0.1), 1), (dict(keep=float("nan")), 1), (dict(sigma=-1.0), 1),
+    (dict(rel=float("inf")), 1), (dict(numel=-1), 1), (dict(numel=1 << 40), 1), (dict(tid=0x0FFFFFFF), 1),
+    (dict(dtype=7), 2), (dict(off=-16), 1), (dict(base=0x10000001), 3),
+])
+def test_init_rejects_invalid_tensor(L, bad, code):
+    ctx = ctypes.c_void_p()
+    d = desc(**bad)
+    st = L.smat_init(ctypes.byref(ctx), ctypes.byref(arr(d)), 1, ctypes.byref(cfg()), ctypes.c_void_p(0x7000000),
+                     1 << 20, None)
+    assert st == code, L.smat_last_error()
+    assert ctx.value is None
+    assert L.smat_last_error()
+
+
+@pytest.mark.parametrize("bad,code", [
+    (dict(alpha_mode=3), 2), (dict(noise=2), 2), (dict(philox_rounds=8), 2),
+    (dict(alpha_min=0.9, alpha_max=0.5), 1), (dict(alpha_min=float("nan")), 1),
+])
+def test_init_rejects_invalid_config(L, bad, code):
+    ctx = ctypes.c_void_p()
+    st = L.smat_init(ctypes.byref(ctx), ctypes.byref(arr(desc())), 1, ctypes.byref(cfg(**bad)),
+                     ctypes.c_void_p(0x7000000), 1 << 20, None)
+    assert st == code
+
+
+def test_init_rejects_duplicate_ids_overlap_and_workspace(L):
+    ctx = ctypes.c_void_p()
+    c = cfg()
+    st = L.smat_init(ctypes.byref(ctx), ctypes.byref(arr(desc(tid=3), desc(tid=3, base=0x20000000))), 2,
+                     ctypes.byref(c), ctypes.c_void_p(0x7000000), 1 << 20, None)
+    assert st == 1
+    d = desc()
+    d.sim = d.theta + 64  # overlaps theta
+    assert L.smat_init(ctypes.byref(ctx), ctypes.byref(arr(d)), 1, ctypes.byref(c), ctypes.c_void_p(0x7000000),
+                       1 << 20, None) == 1
+    need = ws_bytes(L, [desc()], c)
+    assert L.smat_init(ctypes.byref(ctx), ctypes.byref(arr(desc())), 1, ctypes.byref(c), ctypes.c_void_p(0), need,
+                       None) == 4
+    assert L.smat_init(ctypes.byref(ctx), ctypes.byref(arr(desc())), 1, ctypes.byref(c),
+                       ctypes.c_void_p(0x7000000 + 16), need, None) == 4
+    assert L.smat_init(ctypes.byref(ctx), ctypes.byref(arr(desc())), 1, ctypes.byref(c), ctypes.c_void_p(0x7000000),
+                       need - 256, None) == 4
+    assert L.smat_init(None, ctypes.byref(arr(desc())), 1, ctypes.byref(c), ctypes.c_void_p(0x7000000), need,
+                       None) == 1
+
+
+def test_null_context_calls_fail_cleanly(L):
+    assert L.smat_simulate_multi(None, 0, None) == 1
+    assert L.smat_grad_map_multi(None, 0, None, None, 0, 0, None) == 1
+    a = ctypes.c_int32()
+    assert L.smat_swap(None, ctypes.byref(a)) == 1
+    assert L.smat_mask_bits(None, 0, 0, None, None) == 1
+    assert L.smat_tensor_scalars(None, 0, None, None) == 1
+    assert L.smat_destroy(None) == 0
+    assert L.smat_debug_philox(None, -1, 0, 10, None, None, None) == 1
+    assert L.smat_debug_philox(None, 4, 0, 9, ctypes.c_void_p(16), None, None) == 1
+    assert L.smat_status_string(6) == b"SMAT_ERR_CUDA"
+
+
+def test_workload_inventory():
+    """The synthetic lists have the stated tensor counts and element counts."""
+    assert (len(W.dec_0p5b().tensors), W.dec_0p5b().numel) == (218, 494_005_120)
+    assert (len(W.llama_7b().tensors), W.llama_7b().numel) == (291, 6_738_415_616)
+    assert (len(W.vl_7b().tensors), W.vl_7b().numel) == (590, 7_062_575_104)
+    assert W.tiny_flat().numel == 1 << 20
+    vit = [t for t in W.vl_7b().tensors if t.name.startswith("vit.")]
+    assert (len(vit), sum(t.numel for t in vit)) == (295, 303_179_776)
+    proj = [t for t in W.vl_7b().tensors if t.name.startswith("proj.")]
+    assert sum(t.numel for t in proj) == 20_979_712
+    # mask set: attention/MLP linears only (Sec. 4.1)
+    for w in (W.dec_0p5b(), W.llama_7b(), W.vl_7b()):
+        for t in w.tensors:
+            assert (t.keep_prob < 1.0) == (t.kind == "linear")

@@ -1,0 +1,92 @@
+"""Full-size parity: the 0.5B, 7B and vision-language lists at their stated
+sizes, in the launch configuration the bench times, checked at sampled
+elements against the CPU oracle (which evaluates elements one by one), and
+through properties that hold at any size (binomial keep rate per tensor,
+sigma_t against the oracle's two-pass statistics)."""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2609_33437_gb300 import workloads as W
+
+from _parity import compare, f32_of, orc_config, orc_tensor, session_for, to_host
+
+pytestmark = pytest.mark.gpu
+
+SAMPLES = 768
+
+
+def _popcount(words: torch.Tensor) -> int:
+    w = words.to(torch.int64) & 0xFFFFFFFF
+    c = torch.zeros_like(w)
+    for b in range(32):
+        c += (w >> b) & 1
+    return int(c.sum())
+
+
+def _check_workload(w: W.Workload, step: int = 0):
+    dev = torch.device("cuda")
+    free, total = torch.cuda.mem_get_info()
+    need = (2 if w.dtype == O.BF16 else 4) * w.numel * 3 + (2 if w.gdtype == O.BF16 else 4) * w.numel * 2
+    if need > free * 0.9:
+        pytest.skip(f"needs {need / 1e9:.1f} GB of device memory, {free / 1e9:.1f} GB free")
+    th, t0, sim, gs, go = W.generate(w, device=dev)
+    sess = session_for(w, th, t0, sim)
+    sess.simulate_multi(step)
+    sess.swap()
+    sess.grad_map_multi(step, gs, go)
+    sess.swap()
+    scal = sess.tensor_scalars(step).cpu().numpy()
+    torch.cuda.synchronize()
+    cfg = orc_config(w, step)
+    rng = np.random.default_rng(77)
+    for k, spec in enumerate(w.tensors):
+        n = spec.numel
+        idx = np.unique(np.concatenate([np.arange(min(n, 16)), np.arange(max(0, n - 16), n),
+                                        rng.integers(0, n, size=min(n, SAMPLES))]))
+        it = torch.from_numpy(idx).to(dev)
+        t = orc_tensor(w, k)
+        if spec.sigma_rel > 0:
+            sig = O.delta_stats(t, to_host(th[k]), to_host(t0[k]))["sigma"]
+            assert abs(float(scal[k, 2]) - sig) <= 1e-5 * sig, f"tensor {k} sigma"
+        else:
+            sig = spec.sigma
+        thv = f32_of(to_host(th[k][it]))
+        t0v = f32_of(to_host(t0[k][it]))
+        ref, kept = O.simulate_at(cfg, t, sig, idx, thv, t0v)
+        mode = O.NOISE_GAUSSIAN if spec.sigma_rel > 0 else w.noise
+        compare(to_host(sim[k][it]), ref, w.dtype, mode, thv, t0v, what=f"{w.name} tensor {k} ({spec.name})")
+        gref = O.gradmap_at(cfg, t, idx, f32_of(to_host(gs[k][it])), gdtype=w.gdtype)
+        gv = np.uint16 if w.gdtype == O.BF16 else np.uint32
+        assert np.array_equal(to_host(go[k][it]).view(gv), gref.astype(gv)), f"tensor {k} gradmap"
+        words = sess.mask_bits(step, k)
+        wh = words.cpu().numpy().view(np.uint32)
+        gbits = (wh[idx >> 5] >> (idx & 31).astype(np.uint32)) & 1
+        assert np.array_equal(gbits.astype(np.uint8), kept), f"tensor {k} mask bits"
+        p = float(np.float32(spec.keep_prob))
+        if 0.0 < p < 1.0:
+            kcount = _popcount(words)
+            assert abs(kcount - n * p) <= 5 * math.sqrt(n * p * (1 - p)) + 1, f"tensor {k} keep rate"
+    sess.close()
+    del th, t0, sim, gs, go
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("name", ["dec_0p5b", "llama_7b", "vl_7b"])
+def test_full_size_list_sampled(name):
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    _check_workload(W.WORKLOADS[name]())
+
+
+def test_flat_2_32_plus_ragged_bf16_sampled():
+    """2^32 + 17 elements in one tensor: 64-bit element indexing end to end."""
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    w = W.flat_sweep(32, O.BF16, 0.3, 2, 1e-4)
+    w.tensors[0].shape = ((1 << 32) + 17,)
+    _check_workload(w, step=1)
