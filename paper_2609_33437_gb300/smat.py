@@ -213,7 +213,8 @@ class SmatSession:
 
     # -- test hooks ----------------------------------------------------------
     def mask_bits(self, step: int, k: int, stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:
-        words = (self.numels[k] + 31) // 32
+        # an out-of-range k is passed through so the library reports it
+        words = (self.numels[k] + 31) // 32 if 0 <= k < self.n else 0
         out = torch.zeros(max(words, 1), dtype=torch.int32, device=self.device)
         check("smat_mask_bits", self._L.smat_mask_bits(self._ctx, int(step), int(k), ctypes.c_void_p(out.data_ptr()),
                                                        _stream_handle(stream)))

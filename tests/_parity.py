@@ -55,16 +55,28 @@ def _ordered_bf16(b: np.ndarray) -> np.ndarray:
     return np.where(b & 0x8000, -(b & 0x7FFF), b)
 
 
+def as_bits(a, dtype) -> np.ndarray:
+    """Storage bits of an output: bf16 as uint16, fp32 as uint32 (float arrays
+    are reinterpreted, never converted)."""
+    a = np.asarray(a)
+    if dtype == O.BF16:
+        if a.dtype == np.uint16:
+            return a
+        if a.dtype == np.uint32:
+            assert int(a.max(initial=0)) < 65536
+            return a.astype(np.uint16)
+    else:
+        if a.dtype == np.float32:
+            return a.view(np.uint32)
+        if a.dtype == np.uint32:
+            return a
+    raise TypeError(f"unexpected array dtype {a.dtype} for storage dtype {dtype}")
+
+
 def compare(got_bits, ref_bits, dtype, noise, th=None, t0=None, what=""):
     """Assert GPU bits match oracle bits within the stated tolerance."""
-    got_bits = np.asarray(got_bits)
-    ref_bits = np.asarray(ref_bits)
-    if dtype == O.BF16:
-        got_bits = got_bits.astype(np.uint16)
-        ref_bits = ref_bits.astype(np.uint16)
-    else:
-        got_bits = got_bits.astype(np.uint32)
-        ref_bits = ref_bits.astype(np.uint32)
+    got_bits = as_bits(got_bits, dtype)
+    ref_bits = as_bits(ref_bits, dtype)
     g = f32_of(got_bits) if dtype == O.BF16 else got_bits.view(np.float32)
     r = f32_of(ref_bits) if dtype == O.BF16 else ref_bits.view(np.float32)
     nan_g, nan_r = np.isnan(g), np.isnan(r)
