@@ -49,6 +49,7 @@ def lib():
         L.orc_philox.argtypes = [P, P, ctypes.c_int32, P]
         L.orc_stream_words.argtypes = [P, ctypes.c_uint32, ctypes.c_uint32, P, P, ctypes.c_int64, P]
         L.orc_f32_to_bf16.argtypes = [P, ctypes.c_int64, P]
+        L.orc_erfinv.argtypes = [P, ctypes.c_int64, P]
         L.orc_scalars.argtypes = [P, P, P, P, P]
         L.orc_delta_stats.argtypes = [P, P, P, P]
         L.orc_simulate.argtypes = [P, P, P, P, P]
@@ -59,7 +60,7 @@ def lib():
         L.orc_gauss_z.argtypes = [P, P, P, ctypes.c_int64, P]
         L.orc_simulate_f64.argtypes = [P, P, ctypes.c_float, P, P, P]
         L.orc_gradmap_f64.argtypes = [P, P, P, P]
-        for name in ("orc_philox", "orc_stream_words", "orc_f32_to_bf16", "orc_scalars",
+        for name in ("orc_philox", "orc_stream_words", "orc_f32_to_bf16", "orc_erfinv", "orc_scalars",
                      "orc_delta_stats", "orc_simulate", "orc_simulate_at", "orc_gradmap",
                      "orc_gradmap_at", "orc_mask_bits", "orc_gauss_z", "orc_simulate_f64",
                      "orc_gradmap_f64"):
@@ -109,6 +110,13 @@ def f32_to_bf16(x):
     x = _c(x, np.float32).ravel()
     out = np.zeros(x.shape[0], np.uint16)
     lib().orc_f32_to_bf16(_p(x), x.shape[0], _p(out))
+    return out
+
+
+def erfinv(v):
+    v = _c(v, np.float64).ravel()
+    out = np.zeros(v.shape[0], np.float64)
+    lib().orc_erfinv(_p(v), v.shape[0], _p(out))
     return out
 
 

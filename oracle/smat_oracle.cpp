@@ -26,13 +26,15 @@
 //   streams: MASK = 0, NOISE = 1, ALPHA_E = 2, ALPHA_T = 3, MASK_LO = 4.
 //   gidx    = elem_offset + i  (global element index of local element i)
 //   u01(u)      = (u >> 8) * 2^-24          in [0, 1)
-//   u01_open(u) = ((u >> 8) + 1) * 2^-24    in (0, 1]
 //   sym(u)      = (2 (u >> 8) + 1 - 2^24) * 2^-24   odd multiples of 2^-24 in (-1, 1)
 //   Mask uniform U(gidx) in [0, 2^32):
 //     hi = byte (gidx & 3) of W(MASK, tid, gidx >> 4)[(gidx >> 2) & 3]
 //     lo = W(MASK_LO, tid, gidx >> 2)[gidx & 3] >> 8
 //     U  = hi * 2^24 + lo ;  kept  <=>  U < T,  T = floor(p_keep * 2^32)
 //   Noise word  n = W(NOISE, tid, gidx >> 2)[gidx & 3]
+//     uniform   eps = fl(sqrt3 sigma) * sym(n)
+//     Gaussian  eps = fl(sqrt2 sigma) * fl(erfinv(sym(n)))  (inverse-CDF transform:
+//               sqrt2 erfinv(v) is N(0, 1) for v uniform on (-1, 1))
 //   Alpha:  per tensor  alpha = fma(amax - amin, u01(W(ALPHA_T, t_a, 0)[0]), amin)
 //           t_a = 0x0FFFFFFF (one alpha for all tensors) or the tensor id;
 //           per element alpha = fma(amax - amin, u01(W(ALPHA_E, tid, gidx >> 2)[gidx & 3]), amin)
@@ -128,8 +130,6 @@ uint32_t stream_word(const OrcConfig& cfg, uint32_t stream, uint32_t tid,
 const float kTwoPow24Inv = 5.9604644775390625e-08f;  // 2^-24, exact
 
 float u01(uint32_t u) { return (float)(u >> 8) * kTwoPow24Inv; }
-double u01_open_d(uint32_t u) { return (double)((u >> 8) + 1u) * 0x1p-24; }
-double u01_d(uint32_t u) { return (double)(u >> 8) * 0x1p-24; }
 float sym(uint32_t u) {
   const int32_t k = (int32_t)(u >> 8);
   return (float)(2 * k + 1 - (1 << 24)) * kTwoPow24Inv;
@@ -180,7 +180,7 @@ struct Scalars {
   float c;            // alpha * inv_keep
   uint64_t T;         // keep threshold on the 32-bit mask uniform
   float sigma;        // Perturb RMS for this call
-  float noise_scale;  // sqrt(3) sigma (uniform) or sigma (Gaussian)
+  float noise_scale;  // fl(sqrt3 sigma) (uniform) or fl(sqrt2 sigma) (Gaussian)
 };
 
 // Population mean and centred second moment of delta = theta - theta0 (each
@@ -228,8 +228,7 @@ Scalars make_scalars(const OrcConfig& cfg, const OrcTensor& t, float sigma) {
   s.c = s.alpha * s.inv_keep;
   s.T = (uint64_t)std::floor((double)t.keep_prob * 4294967296.0);
   s.sigma = sigma;
-  s.noise_scale = (cfg.noise == NOISE_UNIFORM) ? (float)(std::sqrt(3.0) * (double)sigma)
-                                               : sigma;
+  s.noise_scale = (float)(std::sqrt(cfg.noise == NOISE_UNIFORM ? 3.0 : 2.0) * (double)sigma);
   return s;
 }
 
@@ -250,24 +249,43 @@ float element_c(const OrcConfig& cfg, const OrcTensor& t, const Scalars& s, uint
   return alpha * s.inv_keep;
 }
 
-// Standard-normal variate of element gidx: Box-Muller on the word pair
-// (2q, 2q+1) of its noise block, evaluated in double and rounded once.
+// erfinv(v) for -1 < v < 1 in double: the root y of erf(y) = |v| (or, for
+// |v| > 1/2, of erfc(y) = 1 - |v|, which is exact in double for the 24-bit
+// values sym() produces), by safeguarded Newton steps from a bracket.
+double erfinv_d(double v) {
+  if (v == 0.0) return 0.0;
+  const double a = std::fabs(v);
+  const bool tail = a > 0.5;
+  const double r = 1.0 - a;  // exact for a = odd multiple of 2^-24
+  const double two_over_sqrt_pi = 1.1283791670955126;
+  double lo = 0.0, hi = 6.0;  // erf(6) = 1 - 2e-17 exceeds every input
+  double y = tail ? std::sqrt(-std::log(r * (2.0 - r))) : a * 0.886226925452758;
+  if (!(y > lo && y < hi)) y = 0.5 * (lo + hi);
+  for (int it = 0; it < 200; ++it) {
+    // f(y) increasing in y: erf(y) - a, or (1 - a) - erfc(y) in the tail
+    const double f = tail ? (r - std::erfc(y)) : (std::erf(y) - a);
+    if (f > 0.0) hi = y; else lo = y;
+    const double fp = two_over_sqrt_pi * std::exp(-y * y);
+    double yn = y - f / fp;
+    if (!(yn > lo && yn < hi)) yn = 0.5 * (lo + hi);
+    if (std::fabs(yn - y) <= 1e-17 * y || hi - lo <= 1e-17 * y) { y = yn; break; }
+    y = yn;
+  }
+  return v < 0.0 ? -y : y;
+}
+
+double sym_d(uint32_t u) { return (double)(2 * (int64_t)(u >> 8) + 1 - (1 << 24)) * 0x1p-24; }
+
+// Unit-variance normal variate of element gidx: sqrt2 erfinv(sym(n)).
 double gauss_z(const OrcConfig& cfg, const OrcTensor& t, uint64_t gidx) {
-  const unsigned w = (unsigned)(gidx & 3);
-  const unsigned q = w >> 1;
-  const uint32_t a = stream_word(cfg, S_NOISE, t.tensor_id, gidx >> 2, 2 * q);
-  const uint32_t b = stream_word(cfg, S_NOISE, t.tensor_id, gidx >> 2, 2 * q + 1);
-  const double rho = std::sqrt(-2.0 * std::log(u01_open_d(a)));
-  const double phi = 2.0 * M_PI * u01_d(b);
-  return (w & 1u) ? rho * std::sin(phi) : rho * std::cos(phi);
+  const uint32_t n = stream_word(cfg, S_NOISE, t.tensor_id, gidx >> 2, (unsigned)(gidx & 3));
+  return std::sqrt(2.0) * erfinv_d(sym_d(n));
 }
 
 float noise_eps(const OrcConfig& cfg, const OrcTensor& t, const Scalars& s, uint64_t gidx) {
-  if (cfg.noise == NOISE_UNIFORM) {
-    const uint32_t n = stream_word(cfg, S_NOISE, t.tensor_id, gidx >> 2, (unsigned)(gidx & 3));
-    return s.noise_scale * sym(n);
-  }
-  return s.noise_scale * (float)gauss_z(cfg, t, gidx);
+  const uint32_t n = stream_word(cfg, S_NOISE, t.tensor_id, gidx >> 2, (unsigned)(gidx & 3));
+  if (cfg.noise == NOISE_UNIFORM) return s.noise_scale * sym(n);
+  return s.noise_scale * (float)erfinv_d(sym_d(n));
 }
 
 // Eq. smat-state for one element, fp32 arithmetic, before the storage rounding.
@@ -312,6 +330,11 @@ void orc_stream_words(const OrcConfig* cfg, uint32_t stream, uint32_t tid, const
 // fp32 <-> bf16 bit conversions (storage rounding of the oracle).
 void orc_f32_to_bf16(const float* x, int64_t n, uint16_t* out) {
   for (int64_t i = 0; i < n; ++i) out[i] = f32_to_bf16_bits(x[i]);
+}
+
+// erfinv in double (the Gaussian transform's definition), for its pin.
+void orc_erfinv(const double* v, int64_t n, double* out) {
+  for (int64_t i = 0; i < n; ++i) out[i] = erfinv_d(v[i]);
 }
 
 // Per-call scalars: out = {alpha, inv_keep, c, T, sigma_t, noise_scale}.
@@ -394,7 +417,7 @@ void orc_mask_bits(const OrcConfig* cfg, const OrcTensor* t, uint32_t* bits) {
   }
 }
 
-// Standard-normal variates z (before the sigma scaling) of the Gaussian mode.
+// Unit-variance normal variates z = sqrt2 erfinv(sym(n)) of the Gaussian mode.
 void orc_gauss_z(const OrcConfig* cfg, const OrcTensor* t, const uint64_t* gidx, int64_t n,
                  double* z) {
   for (int64_t k = 0; k < n; ++k) z[k] = gauss_z(*cfg, *t, gidx[k]);
@@ -418,7 +441,8 @@ void orc_simulate_f64(const OrcConfig* cfg, const OrcTensor* t, float sigma_t, c
         const uint32_t nw = stream_word(*cfg, S_NOISE, t->tensor_id, gidx >> 2, (unsigned)(gidx & 3));
         x += (double)s.noise_scale * (double)sym(nw);
       } else {
-        x += (double)s.noise_scale * gauss_z(*cfg, *t, gidx);
+        const uint32_t nw = stream_word(*cfg, S_NOISE, t->tensor_id, gidx >> 2, (unsigned)(gidx & 3));
+        x += (double)s.noise_scale * erfinv_d(sym_d(nw));
       }
     }
     out[i] = x;

@@ -37,111 +37,151 @@ constexpr int NOISE_GAUSSIAN = 1;
 constexpr int DT_F32 = 0;
 constexpr int DT_BF16 = 1;
 
-// One Philox-4x32-R block with round keys precomputed from the seed.
+// One Philox-4x32-R block with round keys precomputed from the seed. Each
+// round takes the full 64-bit products of words 0 and 2 with the round
+// multipliers (one wide multiply each).
 template <int R>
 __device__ __forceinline__ uint4 philox(uint32_t c0, uint32_t c1, uint32_t c2, uint32_t c3,
                                         const RoundKeys& k) {
 #pragma unroll
   for (int r = 0; r < R; ++r) {
-    const uint32_t hiA = __umulhi(kMulA, c0);
-    const uint32_t loA = kMulA * c0;
-    const uint32_t hiB = __umulhi(kMulB, c2);
-    const uint32_t loB = kMulB * c2;
-    c0 = hiB ^ c1 ^ k.k0[r];
-    c1 = loB;
-    c2 = hiA ^ c3 ^ k.k1[r];
-    c3 = loA;
+    const uint64_t pA = (uint64_t)c0 * kMulA;
+    const uint64_t pB = (uint64_t)c2 * kMulB;
+    c0 = (uint32_t)(pB >> 32) ^ c1 ^ k.k0[r];
+    c1 = (uint32_t)pB;
+    c2 = (uint32_t)(pA >> 32) ^ c3 ^ k.k1[r];
+    c3 = (uint32_t)pA;
   }
   return make_uint4(c0, c1, c2, c3);
 }
 
-// Block j of sub-stream `stream` of tensor `tid` at this call's step.
-template <int R>
+// Block j of sub-stream `stream` of tensor `tid` at this call's step. J0: the
+// caller guarantees j < 2^32, so counter word 1 is the constant 0 and the
+// loop-invariant part of the first two rounds can be hoisted.
+template <int R, bool J0 = false>
 __device__ __forceinline__ uint4 stream_block(const KArgs& a, uint32_t stream, uint32_t tid,
                                               uint64_t j) {
-  return philox<R>((uint32_t)j, (uint32_t)(j >> 32), (stream << 28) | tid, a.step, a.key);
+  return philox<R>((uint32_t)j, J0 ? 0u : (uint32_t)(j >> 32), (stream << 28) | tid, a.step, a.key);
 }
 
 __device__ __forceinline__ uint32_t pick(const uint4& w, unsigned i) {
   return i == 0 ? w.x : (i == 1 ? w.y : (i == 2 ? w.z : w.w));
 }
 
-// u01(u) = (u >> 8) 2^-24, u01_open(u) = ((u >> 8) + 1) 2^-24,
-// sym(u) = (2 (u >> 8) + 1 - 2^24) 2^-24; all exact in fp32.
+// u01(u) = (u >> 8) 2^-24 and sym(u) = (2 (u >> 8) + 1 - 2^24) 2^-24, both
+// exact in fp32.
 __device__ __forceinline__ float u01(uint32_t u) {
   return __fmul_rn(__uint2float_rn(u >> 8), 5.9604644775390625e-08f);
-}
-__device__ __forceinline__ float u01_open(uint32_t u) {
-  return __fmul_rn(__uint2float_rn((u >> 8) + 1u), 5.9604644775390625e-08f);
 }
 __device__ __forceinline__ float sym(uint32_t u) {
   const int k = (int)(u >> 8);
   return __fmul_rn(__int2float_rn(2 * k + 1 - (1 << 24)), 5.9604644775390625e-08f);
 }
 
-// Standard-normal pair from two words (Box-Muller; CUDA's logf / sqrtf /
-// sincospif, 2 u01(b) is exact so the angle needs no reduction).
-__device__ __forceinline__ void box_muller(uint32_t a, uint32_t b, float& z0, float& z1) {
-  const float rho = sqrtf(__fmul_rn(-2.0f, logf(u01_open(a))));
-  float s, c;
-  sincospif(__fmul_rn(2.0f, u01(b)), &s, &c);
-  z0 = __fmul_rn(rho, c);
-  z1 = __fmul_rn(rho, s);
-}
-
+// Perturb of one element from its noise word: uniform scale * sym(n) with
+// scale = fl(sqrt3 sigma), or Gaussian scale * erfinv(sym(n)) with
+// scale = fl(sqrt2 sigma) (inverse-CDF transform; CUDA's erfinvf).
 template <int NOISE>
-__device__ __forceinline__ void noise4(const uint4& w, float scale, float (&eps)[4]) {
-  if (NOISE == NOISE_UNIFORM) {
-    eps[0] = __fmul_rn(scale, sym(w.x));
-    eps[1] = __fmul_rn(scale, sym(w.y));
-    eps[2] = __fmul_rn(scale, sym(w.z));
-    eps[3] = __fmul_rn(scale, sym(w.w));
-  } else {
-    float z0, z1, z2, z3;
-    box_muller(w.x, w.y, z0, z1);
-    box_muller(w.z, w.w, z2, z3);
-    eps[0] = __fmul_rn(scale, z0);
-    eps[1] = __fmul_rn(scale, z1);
-    eps[2] = __fmul_rn(scale, z2);
-    eps[3] = __fmul_rn(scale, z3);
-  }
+__device__ __forceinline__ float noise_of(uint32_t n, float scale) {
+  if (NOISE == NOISE_UNIFORM) return __fmul_rn(scale, sym(n));
+  return __fmul_rn(scale, erfinvf(sym(n)));
 }
 
-template <int NOISE>
-__device__ __forceinline__ float noise1(const uint4& w, unsigned word, float scale) {
-  if (NOISE == NOISE_UNIFORM) return __fmul_rn(scale, sym(pick(w, word)));
-  float z0, z1;
-  if (word < 2)
-    box_muller(w.x, w.y, z0, z1);
-  else
-    box_muller(w.z, w.w, z0, z1);
-  return __fmul_rn(scale, (word & 1u) ? z1 : z0);
+// Set element e's flag without indexing kw by a run-time value (which would
+// move the array to local memory).
+__device__ __forceinline__ void set_kept(uint32_t (&kw)[4], int e) {
+  const uint32_t bit = 0x80u << (8 * (e & 3));
+  const int q = e >> 2;
+  kw[0] |= (q == 0) ? bit : 0u;
+  kw[1] |= (q == 1) ? bit : 0u;
+  kw[2] |= (q == 2) ? bit : 0u;
+  kw[3] |= (q == 3) ? bit : 0u;
 }
 
-// Keep bits of the 16 elements gidx0 .. gidx0 + 15 (gidx0 % 16 == 0): the high
-// byte of each element's mask uniform comes from one MASK block; the low 24
-// bits are drawn only when the byte ties with the threshold's high byte.
-template <int R>
-__device__ __forceinline__ uint32_t group_keep16(const KArgs& a, uint32_t tid, uint32_t t_hi,
-                                                 uint32_t t_lo, uint64_t gidx0) {
-  const uint4 w = stream_block<R>(a, S_MASK, tid, gidx0 >> 4);
+__device__ __forceinline__ bool kept_of(const uint32_t (&kw)[4], int e) {
+  return (kw[e >> 2] & (0x80u << (8 * (e & 3)))) != 0u;
+}
+
+// Keep flags of the 16 elements gidx0 .. gidx0 + 15 (gidx0 % 16 == 0). The
+// high byte of each element's 32-bit mask uniform comes from one MASK block
+// (byte b of word q serves element 4q + b); it is compared with the
+// threshold's high byte four bytes at a time (SWAR, no carries between
+// bytes). Bit 8b + 7 of kw[q] is element 4q + b's flag. Bytes equal to the
+// threshold byte (probability 1/256 each) need the low 24 bits of their
+// uniform from the MASK_LO stream: they are returned in *ties (bit e for
+// element e, flag left clear) when ties != nullptr, else drawn here.
+template <int R, bool J0>
+__device__ __forceinline__ void group_keep16(const KArgs& a, uint32_t tid, uint32_t t_hi,
+                                             uint32_t t_lo, uint64_t gidx0, uint32_t (&kw)[4],
+                                             uint32_t* ties) {
+  const uint4 w = stream_block<R, J0>(a, S_MASK, tid, gidx0 >> 4);
   const uint32_t words[4] = {w.x, w.y, w.z, w.w};
-  uint32_t keep = 0u, tie = 0u;
+  const uint32_t tt = t_hi * 0x01010101u;
+  const uint32_t tl = tt & 0x7F7F7F7Fu;
+  uint32_t anytie = 0u;
 #pragma unroll
-  for (int k = 0; k < 16; ++k) {
-    const uint32_t hi = (words[k >> 2] >> (8 * (k & 3))) & 0xFFu;
-    keep |= (uint32_t)(hi < t_hi) << k;
-    tie |= (uint32_t)(hi == t_hi) << k;
+  for (int q = 0; q < 4; ++q) {
+    const uint32_t x = words[q];
+    // bit 7 of each byte of d: low 7 bits of x >= low 7 bits of t
+    const uint32_t d = (x | 0x80808080u) - tl;
+    kw[q] = ((~x & tt) | (~(x ^ tt) & ~d)) & 0x80808080u;  // x < t per byte
+    const uint32_t e = x ^ tt;
+    anytie |= (e - 0x01010101u) & ~e & 0x80808080u;  // nonzero iff some byte equals t
   }
-  if (t_lo == 0u) tie = 0u;  // U = T_hi 2^24 + lo >= T: dropped without a draw
-  while (tie) {
-    const int k = __ffs(tie) - 1;
-    tie &= tie - 1u;
-    const uint4 l = stream_block<R>(a, S_MASK_LO, tid, (gidx0 >> 2) + (uint64_t)(k >> 2));
-    keep |= (uint32_t)((pick(l, k & 3) >> 8) < t_lo) << k;
+  if (t_lo != 0u && anytie != 0u) {
+    uint32_t tbits = 0u;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint32_t e = words[q] ^ tt;
+      const uint32_t eq = ~(((e & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | e) & 0x80808080u;  // exact per byte
+      tbits |= ((eq >> 7) & 1u) << (4 * q) | ((eq >> 15) & 1u) << (4 * q + 1) |
+               ((eq >> 23) & 1u) << (4 * q + 2) | ((eq >> 31) & 1u) << (4 * q + 3);
+    }
+    if (ties != nullptr) {
+      *ties = tbits;
+    } else {
+      while (tbits) {
+        const int e = __ffs(tbits) - 1;
+        tbits &= tbits - 1u;
+        const uint4 l = stream_block<R, J0>(a, S_MASK_LO, tid, (gidx0 >> 2) + (uint64_t)(e >> 2));
+        if ((pick(l, (unsigned)(e & 3)) >> 8) < t_lo) set_kept(kw, e);
+      }
+    }
+  } else if (ties != nullptr) {
+    *ties = 0u;
   }
-  return keep;
 }
+
+// Tie elements whose low 24 mask bits are drawn at the end of the chunk, so
+// the rare Philox call runs once for the whole warp instead of once per
+// group. Up to four 16-bit in-chunk offsets per thread, two per register.
+struct TieList {
+  uint32_t w0 = 0u, w1 = 0u;
+  int n = 0;
+  __device__ __forceinline__ bool push(uint32_t off) {
+    switch (n) {
+      case 0: w0 = off; break;
+      case 1: w0 |= off << 16; break;
+      case 2: w1 = off; break;
+      case 3: w1 |= off << 16; break;
+      default: return false;
+    }
+    ++n;
+    return true;
+  }
+  __device__ __forceinline__ uint32_t at(int k) const {
+    const uint32_t w = (k < 2) ? w0 : w1;
+    return (k & 1) ? (w >> 16) : (w & 0xFFFFu);
+  }
+};
+
+// Low-24-bit test of one tie element.
+template <int R, bool J0>
+__device__ __forceinline__ bool tie_kept(const KArgs& a, uint32_t tid, uint32_t t_lo, uint64_t gidx) {
+  const uint4 l = stream_block<R, J0>(a, S_MASK_LO, tid, gidx >> 2);
+  return (pick(l, (unsigned)(gidx & 3)) >> 8) < t_lo;
+}
+
 
 // Keep decision of one element (any alignment).
 template <int R>
@@ -173,28 +213,25 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&v);
 }
 
-// 16 consecutive elements starting at element i (32-byte aligned for bf16,
-// 64-byte aligned for fp32 under TF_VEC), widened to fp32.
+// 16 consecutive elements starting at element i, kept as loaded (bf16: 8
+// words of two elements, fp32: 16 words); 32-byte aligned under TF_VEC.
 template <int DT>
-__device__ __forceinline__ void load16(const void* base, int64_t i, float (&v)[16]) {
+struct Raw16 {
+  uint32_t r[DT == DT_BF16 ? 8 : 16];
+  __device__ __forceinline__ float at(int e) const {
+    if (DT == DT_BF16) return __uint_as_float((e & 1) ? (r[e >> 1] & 0xFFFF0000u) : (r[e >> 1] << 16));
+    return __uint_as_float(r[e]);
+  }
+};
+
+template <int DT>
+__device__ __forceinline__ void load16(const void* base, int64_t i, Raw16<DT>& v) {
   if (DT == DT_BF16) {
-    uint32_t r[8];
-    ld32B(static_cast<const uint16_t*>(base) + i, r);
-#pragma unroll
-    for (int m = 0; m < 8; ++m) {
-      v[2 * m] = __uint_as_float(r[m] << 16);
-      v[2 * m + 1] = __uint_as_float(r[m] & 0xFFFF0000u);
-    }
+    ld32B(static_cast<const uint16_t*>(base) + i, *reinterpret_cast<uint32_t(*)[8]>(v.r));
   } else {
-    uint32_t r[8], s[8];
     const float* p = static_cast<const float*>(base) + i;
-    ld32B(p, r);
-    ld32B(p + 8, s);
-#pragma unroll
-    for (int m = 0; m < 8; ++m) {
-      v[m] = __uint_as_float(r[m]);
-      v[8 + m] = __uint_as_float(s[m]);
-    }
+    ld32B(p, *reinterpret_cast<uint32_t(*)[8]>(v.r));
+    ld32B(p + 8, *reinterpret_cast<uint32_t(*)[8]>(v.r + 8));
   }
 }
 
@@ -235,15 +272,6 @@ __device__ __forceinline__ void store1(void* base, int64_t i, float v) {
   }
 }
 
-// Eq. smat-state for one element given its keep decision, c and eps.
-__device__ __forceinline__ float combine(bool kept, float c, float th, float t0, bool has_noise,
-                                         float eps) {
-  float x = t0;
-  if (kept) x = (c == 1.0f) ? th : __fmaf_rn(c, __fsub_rn(th, t0), t0);
-  if (has_noise) x = __fadd_rn(x, eps);
-  return x;
-}
-
 __device__ __forceinline__ float alpha_elem(const KArgs& a, uint32_t u) {
   return __fmaf_rn(a.alpha_width, u01(u), a.alpha_min);
 }
@@ -271,116 +299,237 @@ __device__ __forceinline__ TView make_view(const DevTensor& T, const DevScalars&
 }
 
 // --------------------------------------------------------------- a3: forward ---
+// One 16-element group on the vector path. IDENT: c == 1 for the whole tensor
+// (kept elements are theta itself); only used without per-element alpha.
+// Tie elements are written as dropped and queued in tl (resolved at the end
+// of the chunk); if the queue is full they are resolved here.
+template <int R, int DT, int NOISE, bool PE, bool IDENT, bool J0>
+__device__ __forceinline__ void sim_group16(const KArgs& a, const TView& v, const void* th_p,
+                                            const void* t0_p, void* sim_p, int64_t i, uint32_t off,
+                                            TieList& tl) {
+  const uint64_t g0 = (uint64_t)(v.off + i);
+  Raw16<DT> th, t0;
+  load16<DT>(th_p, i, th);
+  load16<DT>(t0_p, i, t0);
+  uint32_t kw[4] = {0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u};
+  if (v.flags & TF_MASK) {
+    uint32_t ties = 0u;
+    group_keep16<R, J0>(a, v.tid, v.t_hi, v.t_lo, g0, kw, &ties);
+    while (ties) {
+      const int e = __ffs(ties) - 1;
+      ties &= ties - 1u;
+      if (!tl.push(off + (uint32_t)e) && tie_kept<R, J0>(a, v.tid, v.t_lo, g0 + (uint64_t)e))
+        set_kept(kw, e);
+    }
+  }
+  float out[16];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    uint4 nw = make_uint4(0u, 0u, 0u, 0u);
+    if (v.has_noise) nw = stream_block<R, J0>(a, S_NOISE, v.tid, (g0 >> 2) + q);
+    uint4 aw = make_uint4(0u, 0u, 0u, 0u);
+    if (PE) aw = stream_block<R, J0>(a, S_ALPHA_E, v.tid, (g0 >> 2) + q);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int e = 4 * q + k;
+      const float x_th = th.at(e), x_t0 = t0.at(e);
+      float kept_val;
+      if (PE) {
+        const float c = __fmul_rn(alpha_elem(a, pick(aw, k)), v.inv_keep);
+        kept_val = (c == 1.0f) ? x_th : __fmaf_rn(c, __fsub_rn(x_th, x_t0), x_t0);
+      } else if (IDENT) {
+        kept_val = x_th;
+      } else {
+        kept_val = __fmaf_rn(v.c, __fsub_rn(x_th, x_t0), x_t0);
+      }
+      float x = kept_of(kw, e) ? kept_val : x_t0;
+      if (v.has_noise) x = __fadd_rn(x, noise_of<NOISE>(pick(nw, k), v.noise_scale));
+      out[e] = x;
+    }
+  }
+  store16<DT>(sim_p, i, out);
+}
+
+// One element given its keep decision (any alignment).
 template <int R, int DT, int NOISE, bool PE>
-__global__ void __launch_bounds__(kBlock) simulate_kernel(const __grid_constant__ KArgs a) {
+__device__ __forceinline__ void sim_elem_as(const KArgs& a, const TView& v, const void* th_p,
+                                            const void* t0_p, void* sim_p, int64_t e, bool kept) {
+  const uint64_t g = (uint64_t)(v.off + e);
+  float c = v.c;
+  if (PE) {
+    const uint4 w = stream_block<R>(a, S_ALPHA_E, v.tid, g >> 2);
+    c = __fmul_rn(alpha_elem(a, pick(w, (unsigned)(g & 3))), v.inv_keep);
+  }
+  const float x_th = load1<DT>(th_p, e), x_t0 = load1<DT>(t0_p, e);
+  float x = x_t0;
+  if (kept) x = (c == 1.0f) ? x_th : __fmaf_rn(c, __fsub_rn(x_th, x_t0), x_t0);
+  if (v.has_noise)
+    x = __fadd_rn(x, noise_of<NOISE>(pick(stream_block<R>(a, S_NOISE, v.tid, g >> 2), (unsigned)(g & 3)),
+                                     v.noise_scale));
+  store1<DT>(sim_p, e, x);
+}
+
+template <int R, int DT, int NOISE, bool PE, bool IDENT, bool J0>
+__device__ __forceinline__ void sim_chunk(const KArgs& a, const TView& v, const DevTensor& T,
+                                          const Chunk& ch) {
+  const bool vec = (v.flags & TF_VEC) != 0u;
+  const bool masked = (v.flags & TF_MASK) != 0u;
+  TieList tl;
+  for (int64_t i = ch.begin + 16 * (int64_t)threadIdx.x; i < ch.end; i += 16 * (int64_t)kBlock) {
+    if (vec && i + 16 <= ch.end) {
+      sim_group16<R, DT, NOISE, PE, IDENT, J0>(a, v, T.theta, T.theta0, T.sim, i, (uint32_t)(i - ch.begin), tl);
+    } else {
+      const int64_t e_end = (i + 16 < ch.end) ? i + 16 : ch.end;
+      for (int64_t e = i; e < e_end; ++e) {
+        const bool kept = masked ? elem_kept<R>(a, v.tid, v.t_hi, v.t_lo, (uint64_t)(v.off + e)) : true;
+        sim_elem_as<R, DT, NOISE, PE>(a, v, T.theta, T.theta0, T.sim, e, kept);
+      }
+    }
+  }
+  // queued ties: rewrite the few that the low 24 bits keep
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    if (k < tl.n) {
+      const int64_t e = ch.begin + (int64_t)tl.at(k);
+      if (tie_kept<R, J0>(a, v.tid, v.t_lo, (uint64_t)(v.off + e)))
+        sim_elem_as<R, DT, NOISE, PE>(a, v, T.theta, T.theta0, T.sim, e, true);
+    }
+  }
+}
+
+template <int R, int DT, int NOISE, bool PE>
+__global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 4 : 2) simulate_kernel(const __grid_constant__ KArgs a) {
   for (int64_t ci = a.chunk_begin + blockIdx.x; ci < a.chunk_end; ci += gridDim.x) {
     const Chunk ch = a.chunks[ci];
     const DevTensor& T = a.tensors[ch.tensor];
     const TView v = make_view(T, a.scal[ch.tensor]);
-    const void* th_p = T.theta;
-    const void* t0_p = T.theta0;
-    void* sim_p = T.sim;
-    const bool vec = (v.flags & TF_VEC) != 0u;
-    const bool masked = (v.flags & TF_MASK) != 0u;
-    for (int64_t i = ch.begin + 16 * (int64_t)threadIdx.x; i < ch.end; i += 16 * (int64_t)kBlock) {
-      const uint64_t g0 = (uint64_t)(v.off + i);
-      if (vec && i + 16 <= ch.end) {
-        float th[16], t0[16], out[16];
-        load16<DT>(th_p, i, th);
-        load16<DT>(t0_p, i, t0);
-        const uint32_t keep = masked ? group_keep16<R>(a, v.tid, v.t_hi, v.t_lo, g0) : 0xFFFFu;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          float eps[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-          if (v.has_noise) noise4<NOISE>(stream_block<R>(a, S_NOISE, v.tid, (g0 >> 2) + q),
-                                         v.noise_scale, eps);
-          float c4[4] = {v.c, v.c, v.c, v.c};
-          if (PE) {
-            const uint4 w = stream_block<R>(a, S_ALPHA_E, v.tid, (g0 >> 2) + q);
-            c4[0] = __fmul_rn(alpha_elem(a, w.x), v.inv_keep);
-            c4[1] = __fmul_rn(alpha_elem(a, w.y), v.inv_keep);
-            c4[2] = __fmul_rn(alpha_elem(a, w.z), v.inv_keep);
-            c4[3] = __fmul_rn(alpha_elem(a, w.w), v.inv_keep);
-          }
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            const int e = 4 * q + k;
-            out[e] = combine((keep >> e) & 1u, c4[k], th[e], t0[e], v.has_noise, eps[k]);
-          }
-        }
-        store16<DT>(sim_p, i, out);
-      } else {
-        const int64_t e_end = (i + 16 < ch.end) ? i + 16 : ch.end;
-        for (int64_t e = i; e < e_end; ++e) {
-          const uint64_t g = (uint64_t)(v.off + e);
-          const bool kept = masked ? elem_kept<R>(a, v.tid, v.t_hi, v.t_lo, g) : true;
-          float c = v.c;
-          if (PE) {
-            const uint4 w = stream_block<R>(a, S_ALPHA_E, v.tid, g >> 2);
-            c = __fmul_rn(alpha_elem(a, pick(w, (unsigned)(g & 3))), v.inv_keep);
-          }
-          float eps = 0.0f;
-          if (v.has_noise)
-            eps = noise1<NOISE>(stream_block<R>(a, S_NOISE, v.tid, g >> 2), (unsigned)(g & 3),
-                                v.noise_scale);
-          store1<DT>(sim_p, e, combine(kept, c, load1<DT>(th_p, e), load1<DT>(t0_p, e), v.has_noise, eps));
-        }
-      }
+    const bool j0 = (uint64_t)(v.off + ch.end) <= (uint64_t(1) << 34);  // gidx >> 2 < 2^32
+    if (!PE && v.c == 1.0f) {
+      if (j0) sim_chunk<R, DT, NOISE, PE, true, true>(a, v, T, ch);
+      else sim_chunk<R, DT, NOISE, PE, true, false>(a, v, T, ch);
+    } else {
+      if (j0) sim_chunk<R, DT, NOISE, PE, false, true>(a, v, T, ch);
+      else sim_chunk<R, DT, NOISE, PE, false, false>(a, v, T, ch);
     }
   }
 }
 
 // ---------------------------------------------------------- a5: gradient map ---
+// When `defer` (no accumulation and g_out distinct from g_sim, so the
+// incoming gradient can be re-read), tie elements are written as dropped (+0)
+// and queued; otherwise they are resolved at once.
+template <int R, int GDT, bool PE, bool ACC, bool J0>
+__device__ __forceinline__ void grad_compute16(const KArgs& a, const TView& v, uint64_t g0, uint32_t off,
+                                               bool defer, TieList& tl, const Raw16<GDT>& gs,
+                                               const Raw16<GDT>& go, float (&out)[16]) {
+  uint32_t kw[4] = {0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u};
+  if (v.flags & TF_MASK) {
+    if (ACC || !defer) {
+      group_keep16<R, J0>(a, v.tid, v.t_hi, v.t_lo, g0, kw, nullptr);
+    } else {
+      uint32_t ties = 0u;
+      group_keep16<R, J0>(a, v.tid, v.t_hi, v.t_lo, g0, kw, &ties);
+      while (ties) {
+        const int e = __ffs(ties) - 1;
+        ties &= ties - 1u;
+        if (!tl.push(off + (uint32_t)e) && tie_kept<R, J0>(a, v.tid, v.t_lo, g0 + (uint64_t)e))
+          set_kept(kw, e);
+      }
+    }
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    uint4 aw = make_uint4(0u, 0u, 0u, 0u);
+    if (PE) aw = stream_block<R, J0>(a, S_ALPHA_E, v.tid, (g0 >> 2) + q);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int e = 4 * q + k;
+      const float c = PE ? __fmul_rn(alpha_elem(a, pick(aw, k)), v.inv_keep) : v.c;
+      float g = kept_of(kw, e) ? __fmul_rn(c, gs.at(e)) : 0.0f;
+      if (ACC) g = __fadd_rn(go.at(e), g);
+      out[e] = g;
+    }
+  }
+}
+
 template <int R, int GDT, bool PE, bool ACC>
-__global__ void __launch_bounds__(kBlock) gradmap_kernel(const __grid_constant__ KArgs a) {
+__device__ __forceinline__ void grad_elem_as(const KArgs& a, const TView& v, const GradPtr& G, int64_t e,
+                                             bool kept) {
+  const uint64_t g = (uint64_t)(v.off + e);
+  float c = v.c;
+  if (PE) {
+    const uint4 w = stream_block<R>(a, S_ALPHA_E, v.tid, g >> 2);
+    c = __fmul_rn(alpha_elem(a, pick(w, (unsigned)(g & 3))), v.inv_keep);
+  }
+  float r = kept ? __fmul_rn(c, load1<GDT>(G.g_sim, e)) : 0.0f;
+  if (ACC) r = __fadd_rn(load1<GDT>(G.g_out, e), r);
+  store1<GDT>(G.g_out, e, r);
+}
+
+// Two groups per iteration (strides apart) so each thread keeps two loads of
+// g~ in flight before the mask work.
+template <int R, int GDT, bool PE, bool ACC, bool J0>
+__device__ __forceinline__ void grad_chunk(const KArgs& a, const TView& v, const GradPtr& G, const Chunk& ch) {
+  constexpr int64_t kStride = 16 * (int64_t)kBlock;
+  const bool masked = (v.flags & TF_MASK) != 0u;
+  const bool defer = !ACC && G.g_sim != G.g_out;
+  TieList tl;
+  for (int64_t i = ch.begin + 16 * (int64_t)threadIdx.x; i < ch.end; i += 2 * kStride) {
+    const int64_t i2 = i + kStride;
+    if (G.vec && i2 + 16 <= ch.end) {
+      Raw16<GDT> gs1, gs2, go1, go2;
+      load16<GDT>(G.g_sim, i, gs1);
+      load16<GDT>(G.g_sim, i2, gs2);
+      if (ACC) {
+        load16<GDT>(G.g_out, i, go1);
+        load16<GDT>(G.g_out, i2, go2);
+      }
+      float out[16];
+      grad_compute16<R, GDT, PE, ACC, J0>(a, v, (uint64_t)(v.off + i), (uint32_t)(i - ch.begin), defer, tl, gs1, go1, out);
+      store16<GDT>(G.g_out, i, out);
+      grad_compute16<R, GDT, PE, ACC, J0>(a, v, (uint64_t)(v.off + i2), (uint32_t)(i2 - ch.begin), defer, tl, gs2, go2, out);
+      store16<GDT>(G.g_out, i2, out);
+    } else {
+      for (int half = 0; half < 2; ++half) {
+        const int64_t b = half ? i2 : i;
+        if (b >= ch.end) break;
+        if (G.vec && b + 16 <= ch.end) {
+          Raw16<GDT> gs1, go1;
+          load16<GDT>(G.g_sim, b, gs1);
+          if (ACC) load16<GDT>(G.g_out, b, go1);
+          float out[16];
+          grad_compute16<R, GDT, PE, ACC, J0>(a, v, (uint64_t)(v.off + b), (uint32_t)(b - ch.begin), defer, tl, gs1, go1, out);
+          store16<GDT>(G.g_out, b, out);
+        } else {
+          const int64_t e_end = (b + 16 < ch.end) ? b + 16 : ch.end;
+          for (int64_t e = b; e < e_end; ++e) {
+            const bool kept = masked ? elem_kept<R>(a, v.tid, v.t_hi, v.t_lo, (uint64_t)(v.off + e)) : true;
+            grad_elem_as<R, GDT, PE, ACC>(a, v, G, e, kept);
+          }
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    if (k < tl.n) {
+      const int64_t e = ch.begin + (int64_t)tl.at(k);
+      if (tie_kept<R, J0>(a, v.tid, v.t_lo, (uint64_t)(v.off + e))) grad_elem_as<R, GDT, PE, ACC>(a, v, G, e, true);
+    }
+  }
+}
+
+template <int R, int GDT, bool PE, bool ACC>
+__global__ void __launch_bounds__(kBlock, (GDT == DT_BF16 && !ACC) ? 3 : 2) gradmap_kernel(const __grid_constant__ KArgs a) {
   for (int64_t ci = a.chunk_begin + blockIdx.x; ci < a.chunk_end; ci += gridDim.x) {
     const Chunk ch = a.chunks[ci];
     const DevTensor& T = a.tensors[ch.tensor];
     const GradPtr G = a.grads[ch.tensor];
     const TView v = make_view(T, a.scal[ch.tensor]);
-    const bool masked = (v.flags & TF_MASK) != 0u;
-    for (int64_t i = ch.begin + 16 * (int64_t)threadIdx.x; i < ch.end; i += 16 * (int64_t)kBlock) {
-      const uint64_t g0 = (uint64_t)(v.off + i);
-      if (G.vec && i + 16 <= ch.end) {
-        float gs[16], go[16], out[16];
-        load16<GDT>(G.g_sim, i, gs);
-        if (ACC) load16<GDT>(G.g_out, i, go);
-        const uint32_t keep = masked ? group_keep16<R>(a, v.tid, v.t_hi, v.t_lo, g0) : 0xFFFFu;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          float c4[4] = {v.c, v.c, v.c, v.c};
-          if (PE) {
-            const uint4 w = stream_block<R>(a, S_ALPHA_E, v.tid, (g0 >> 2) + q);
-            c4[0] = __fmul_rn(alpha_elem(a, w.x), v.inv_keep);
-            c4[1] = __fmul_rn(alpha_elem(a, w.y), v.inv_keep);
-            c4[2] = __fmul_rn(alpha_elem(a, w.z), v.inv_keep);
-            c4[3] = __fmul_rn(alpha_elem(a, w.w), v.inv_keep);
-          }
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            const int e = 4 * q + k;
-            float g = ((keep >> e) & 1u) ? __fmul_rn(c4[k], gs[e]) : 0.0f;
-            if (ACC) g = __fadd_rn(go[e], g);
-            out[e] = g;
-          }
-        }
-        store16<GDT>(G.g_out, i, out);
-      } else {
-        const int64_t e_end = (i + 16 < ch.end) ? i + 16 : ch.end;
-        for (int64_t e = i; e < e_end; ++e) {
-          const uint64_t g = (uint64_t)(v.off + e);
-          const bool kept = masked ? elem_kept<R>(a, v.tid, v.t_hi, v.t_lo, g) : true;
-          float c = v.c;
-          if (PE) {
-            const uint4 w = stream_block<R>(a, S_ALPHA_E, v.tid, g >> 2);
-            c = __fmul_rn(alpha_elem(a, pick(w, (unsigned)(g & 3))), v.inv_keep);
-          }
-          float r = kept ? __fmul_rn(c, load1<GDT>(G.g_sim, e)) : 0.0f;
-          if (ACC) r = __fadd_rn(load1<GDT>(G.g_out, e), r);
-          store1<GDT>(G.g_out, e, r);
-        }
-      }
-    }
+    if ((uint64_t)(v.off + ch.end) <= (uint64_t(1) << 34))
+      grad_chunk<R, GDT, PE, ACC, true>(a, v, G, ch);
+    else
+      grad_chunk<R, GDT, PE, ACC, false>(a, v, G, ch);
   }
 }
 
@@ -404,12 +553,12 @@ __global__ void __launch_bounds__(kBlock) delta_stats_kernel(const __grid_consta
     float s = 0.0f, q = 0.0f;
     for (int64_t i = ch.begin + 16 * (int64_t)threadIdx.x; i < ch.end; i += 16 * (int64_t)kBlock) {
       if (vec && i + 16 <= ch.end) {
-        float th[16], t0[16];
+        Raw16<DT> th, t0;
         load16<DT>(T.theta, i, th);
         load16<DT>(T.theta0, i, t0);
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
-          const float d = __fsub_rn(th[k], t0[k]);
+          const float d = __fsub_rn(th.at(k), t0.at(k));
           s += d;
           q = __fmaf_rn(d, d, q);
         }
@@ -479,7 +628,7 @@ __global__ void scalars_kernel(const __grid_constant__ KArgs a) {
       S.c = __fmul_rn(S.alpha, T.inv_keep);
     }
     S.sigma = sigma;
-    S.noise_scale = (NOISE == NOISE_UNIFORM) ? (float)(sqrt(3.0) * (double)sigma) : sigma;
+    S.noise_scale = (float)(sqrt(NOISE == NOISE_UNIFORM ? 3.0 : 2.0) * (double)sigma);
     a.scal[t] = S;
   }
 }
@@ -500,8 +649,11 @@ __global__ void __launch_bounds__(kBlock) mask_bits_kernel(const __grid_constant
       bits = 0xFFFFFFFFu;
     } else if (aligned && i0 + 32 <= numel) {
       const uint64_t g0 = (uint64_t)(T.elem_offset + i0);
-      bits = group_keep16<R>(a, T.tid, T.t_hi, T.t_lo, g0) |
-             (group_keep16<R>(a, T.tid, T.t_hi, T.t_lo, g0 + 16) << 16);
+      uint32_t kw[4];
+      for (int h = 0; h < 2; ++h) {
+        group_keep16<R, false>(a, T.tid, T.t_hi, T.t_lo, g0 + 16 * h, kw, nullptr);
+        for (int e = 0; e < 16; ++e) bits |= (uint32_t)kept_of(kw, e) << (16 * h + e);
+      }
     } else {
       for (int k = 0; k < 32 && i0 + k < numel; ++k)
         bits |= (uint32_t)elem_kept<R>(a, T.tid, T.t_hi, T.t_lo, (uint64_t)(T.elem_offset + i0 + k)) << k;
