@@ -45,7 +45,8 @@ UNIT = "GB/s"
 FALLBACK_HBM_GBS = 6800.0
 NOMINAL_HBM_GBS = 8000.0
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2609_33437_gb300", "csrc", f)
-                  for f in ("smat_kernels.cu", "smat_internal.h")]
+                  for f in ("smat_device.cuh", "smat_simulate.cuh", "smat_sim_bf16.cu", "smat_gradmap.cu",
+                            "smat_internal.h")]
 
 
 def parse():

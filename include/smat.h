@@ -170,6 +170,13 @@ smat_status smat_destroy(smat_ctx* ctx);
 smat_status smat_debug_philox(const uint32_t* d_ctr, int64_t n, uint64_t seed, int32_t rounds,
                               uint32_t* d_out, uint32_t* d_out_ref, smat_stream_t stream);
 
+/* Test hook: the unit noise transform of n raw noise words d_words (device):
+ * d_out[i] = sym(w) = (2 (w >> 8) + 1 - 2^24) 2^-24 for SMAT_NOISE_UNIFORM,
+ * or erfinv(sym(w)) as the forward evaluates it for SMAT_NOISE_GAUSSIAN
+ * (the forward scales these by fl(sqrt3 sigma) and fl(sqrt2 sigma)). */
+smat_status smat_debug_noise_unit(const uint32_t* d_words, int64_t n, int32_t noise, float* d_out,
+                                  smat_stream_t stream);
+
 /* Per-kernel timing (for measurement): while enabled, every kernel this
  * context launches is bracketed by two CUDA events recorded on the launching
  * stream. Kinds: 0 delta statistics (a2), 1 per-call scalars (a1),

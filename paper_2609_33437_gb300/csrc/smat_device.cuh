@@ -1,0 +1,347 @@
+#pragma once
+// SMAT simulated-merge device code for GB300 (sm_103a): shared helpers.
+//
+// Rows of the hot path implemented here:
+//   a1 scalars_kernel      per-call scalars (Scale alpha_t, c_t = alpha_t / p_keep,
+//                          sigma_t, noise scale), Sec. 4.1
+//   a2 delta_stats_kernel  per-chunk sums of delta = theta - theta0 and delta^2
+//   a3 simulate_kernel     theta~ = theta0 + alpha m (.) (theta - theta0) + eps
+//                          (Eq. smat-state, Eq. smat-mask, Perturb of Sec. 4.1)
+//   a5 gradmap_kernel      g = alpha m (.) g~ (Eq. smat-gradient), mask regenerated
+//   a6 mask_bits_kernel    packed keep bits (test hook)
+//
+// All of them are multi-tensor launches over a chunk table: each CTA walks
+// chunks of 2^16 elements of one tensor in grid-stride order; each thread
+// owns 16 consecutive elements at a time (one 256-bit load per bf16 input,
+// two per fp32 input), which is exactly one Philox block of the mask stream
+// (16 high bytes) and four blocks of the noise stream. The random words stay
+// in registers; masks and noise are never written to memory.
+//
+// The path is elementwise and bound by HBM bandwidth or by the integer
+// pipeline (Philox): there is no contraction, so no tensor-core work.
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <curand_philox4x32_x.h>
+
+#include "smat_internal.h"
+
+namespace smat {
+namespace {
+
+// Philox-4x32 round multipliers (Salmon et al., SC'11).
+constexpr uint32_t kMulA = 0xD2511F53u;
+constexpr uint32_t kMulB = 0xCD9E8D57u;
+
+constexpr int NOISE_UNIFORM = 0;
+constexpr int NOISE_GAUSSIAN = 1;
+constexpr int NOISE_NONE = 2;  // sigma_t == 0: no add at all (chunk-level choice)
+constexpr int DT_F32 = 0;
+constexpr int DT_BF16 = 1;
+
+// One Philox-4x32-R block with round keys precomputed from the seed. Each
+// round takes the full 64-bit products of words 0 and 2 with the round
+// multipliers (one wide multiply each).
+template <int R>
+__device__ __forceinline__ uint4 philox(uint32_t c0, uint32_t c1, uint32_t c2, uint32_t c3,
+                                        const RoundKeys& k) {
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
+    const uint64_t pA = (uint64_t)c0 * kMulA;
+    const uint64_t pB = (uint64_t)c2 * kMulB;
+    c0 = (uint32_t)(pB >> 32) ^ c1 ^ k.k0[r];
+    c1 = (uint32_t)pB;
+    c2 = (uint32_t)(pA >> 32) ^ c3 ^ k.k1[r];
+    c3 = (uint32_t)pA;
+  }
+  return make_uint4(c0, c1, c2, c3);
+}
+
+// Block j of sub-stream `stream` of tensor `tid` at this call's step. J0: the
+// caller guarantees j < 2^32, so counter word 1 is the constant 0 and the
+// loop-invariant part of the first two rounds can be hoisted.
+template <int R, bool J0 = false>
+__device__ __forceinline__ uint4 stream_block(const KArgs& a, uint32_t stream, uint32_t tid,
+                                              uint64_t j) {
+  return philox<R>((uint32_t)j, J0 ? 0u : (uint32_t)(j >> 32), (stream << 28) | tid, a.step, a.key);
+}
+
+__device__ __forceinline__ uint32_t pick(const uint4& w, unsigned i) {
+  return i == 0 ? w.x : (i == 1 ? w.y : (i == 2 ? w.z : w.w));
+}
+
+// u01(u) = (u >> 8) 2^-24 and sym(u) = (2 (u >> 8) + 1 - 2^24) 2^-24, both
+// exact in fp32.
+__device__ __forceinline__ float u01(uint32_t u) {
+  return __fmul_rn(__uint2float_rn(u >> 8), 5.9604644775390625e-08f);
+}
+__device__ __forceinline__ float sym(uint32_t u) {
+  const int k = (int)(u >> 8);
+  return __fmul_rn(__int2float_rn(2 * k + 1 - (1 << 24)), 5.9604644775390625e-08f);
+}
+
+// erfinv(x) for |x| <= 1 - 2^-24 (every value sym() produces), after the
+// structure of M. Giles, "Approximating the erfinv function" (GPU Computing
+// Gems Jade Edition, 2011), with coefficients fitted for this form by
+// csrc/fit_erfinv.py: with L = log2(1 - x^2) (one fused multiply-add and the
+// hardware log2),
+//   L >= -8:  erfinv(x) = x * P(L)                 (degree 9, 99.8% of inputs)
+//   L <  -8:  erfinv(x) = x * Q(sqrt(-L) - 3.8125)  (degree 9)
+// Both ratios erfinv(x) / x are even in x, so the result is exactly odd.
+// Relative error about 2e-7 (a few fp32 ulps); the tests bound it.
+__device__ __forceinline__ float erfinv_poly(float x) {
+  const float t = __fmaf_rn(-x, x, 1.0f);
+  float L;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(L) : "f"(t));
+  float p;
+  if (L >= -8.0f) {
+    p = 2.676246447e-10f;
+    p = __fmaf_rn(p, L, 9.962457526e-09f);
+    p = __fmaf_rn(p, L, 1.280022701e-07f);
+    p = __fmaf_rn(p, L, 2.725655577e-07f);
+    p = __fmaf_rn(p, L, -7.822631233e-06f);
+    p = __fmaf_rn(p, L, -3.107573502e-05f);
+    p = __fmaf_rn(p, L, 7.751958910e-04f);
+    p = __fmaf_rn(p, L, 5.547157954e-03f);
+    p = __fmaf_rn(p, L, -1.608200818e-01f);
+    p = __fmaf_rn(p, L, 8.862268925e-01f);
+  } else {
+    const float v = __fsub_rn(sqrtf(-L), 3.8125f);
+    p = 2.205743658e-05f;
+    p = __fmaf_rn(p, v, -2.623226646e-05f);
+    p = __fmaf_rn(p, v, -9.935771232e-05f);
+    p = __fmaf_rn(p, v, 3.947049263e-04f);
+    p = __fmaf_rn(p, v, -8.652319084e-04f);
+    p = __fmaf_rn(p, v, 1.542331069e-03f);
+    p = __fmaf_rn(p, v, -2.662600018e-03f);
+    p = __fmaf_rn(p, v, 4.380439408e-03f);
+    p = __fmaf_rn(p, v, 8.361965418e-01f);
+    p = __fmaf_rn(p, v, 3.007633686e+00f);
+  }
+  return __fmul_rn(x, p);
+}
+
+// Perturb of one element from its noise word: uniform scale * sym(n) with
+// scale = fl(sqrt3 sigma), or Gaussian scale * erfinv(sym(n)) with
+// scale = fl(sqrt2 sigma) (inverse-CDF transform: sqrt2 erfinv(v) is
+// N(0, 1) for v uniform on (-1, 1)).
+template <int NOISE>
+__device__ __forceinline__ float noise_of(uint32_t n, float scale) {
+  if (NOISE == NOISE_UNIFORM) return __fmul_rn(scale, sym(n));
+  if (NOISE == NOISE_GAUSSIAN) return __fmul_rn(scale, erfinv_poly(sym(n)));
+  return 0.0f;
+}
+
+// Set element e's flag without indexing kw by a run-time value (which would
+// move the array to local memory).
+__device__ __forceinline__ void set_kept(uint32_t (&kw)[4], int e) {
+  const uint32_t bit = 0x80u << (8 * (e & 3));
+  const int q = e >> 2;
+  kw[0] |= (q == 0) ? bit : 0u;
+  kw[1] |= (q == 1) ? bit : 0u;
+  kw[2] |= (q == 2) ? bit : 0u;
+  kw[3] |= (q == 3) ? bit : 0u;
+}
+
+__device__ __forceinline__ bool kept_of(const uint32_t (&kw)[4], int e) {
+  return (kw[e >> 2] & (0x80u << (8 * (e & 3)))) != 0u;
+}
+
+// Keep flags of the 16 elements gidx0 .. gidx0 + 15 (gidx0 % 16 == 0). The
+// high byte of each element's 32-bit mask uniform comes from one MASK block
+// (byte b of word q serves element 4q + b); it is compared with the
+// threshold's high byte four bytes at a time (SWAR, no carries between
+// bytes). Bit 8b + 7 of kw[q] is element 4q + b's flag. Bytes equal to the
+// threshold byte (probability 1/256 each) need the low 24 bits of their
+// uniform from the MASK_LO stream: they are returned in *ties (bit e for
+// element e, flag left clear) when ties != nullptr, else drawn here.
+template <int R, bool J0>
+__device__ __forceinline__ void group_keep16(const KArgs& a, uint32_t tid, uint32_t t_hi,
+                                             uint32_t t_lo, uint64_t gidx0, uint32_t (&kw)[4],
+                                             uint32_t* ties) {
+  const uint4 w = stream_block<R, J0>(a, S_MASK, tid, gidx0 >> 4);
+  const uint32_t words[4] = {w.x, w.y, w.z, w.w};
+  const uint32_t tt = t_hi * 0x01010101u;
+  const uint32_t tl = tt & 0x7F7F7F7Fu;
+  uint32_t anytie = 0u;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const uint32_t x = words[q];
+    // bit 7 of each byte of d: low 7 bits of x >= low 7 bits of t
+    const uint32_t d = (x | 0x80808080u) - tl;
+    kw[q] = ((~x & tt) | (~(x ^ tt) & ~d)) & 0x80808080u;  // x < t per byte
+    const uint32_t e = x ^ tt;
+    anytie |= (e - 0x01010101u) & ~e & 0x80808080u;  // nonzero iff some byte equals t
+  }
+  if (t_lo != 0u && anytie != 0u) {
+    uint32_t tbits = 0u;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint32_t e = words[q] ^ tt;
+      const uint32_t eq = ~(((e & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | e) & 0x80808080u;  // exact per byte
+      tbits |= ((eq >> 7) & 1u) << (4 * q) | ((eq >> 15) & 1u) << (4 * q + 1) |
+               ((eq >> 23) & 1u) << (4 * q + 2) | ((eq >> 31) & 1u) << (4 * q + 3);
+    }
+    if (ties != nullptr) {
+      *ties = tbits;
+    } else {
+      while (tbits) {
+        const int e = __ffs(tbits) - 1;
+        tbits &= tbits - 1u;
+        const uint4 l = stream_block<R, J0>(a, S_MASK_LO, tid, (gidx0 >> 2) + (uint64_t)(e >> 2));
+        if ((pick(l, (unsigned)(e & 3)) >> 8) < t_lo) set_kept(kw, e);
+      }
+    }
+  } else if (ties != nullptr) {
+    *ties = 0u;
+  }
+}
+
+// Tie elements whose low 24 mask bits are drawn at the end of the chunk, so
+// the rare Philox call runs once for the whole warp instead of once per
+// group. Up to four 16-bit in-chunk offsets per thread, two per register.
+struct TieList {
+  uint32_t w0 = 0u, w1 = 0u;
+  int n = 0;
+  __device__ __forceinline__ bool push(uint32_t off) {
+    switch (n) {
+      case 0: w0 = off; break;
+      case 1: w0 |= off << 16; break;
+      case 2: w1 = off; break;
+      case 3: w1 |= off << 16; break;
+      default: return false;
+    }
+    ++n;
+    return true;
+  }
+  __device__ __forceinline__ uint32_t at(int k) const {
+    const uint32_t w = (k < 2) ? w0 : w1;
+    return (k & 1) ? (w >> 16) : (w & 0xFFFFu);
+  }
+};
+
+// Low-24-bit test of one tie element.
+template <int R, bool J0>
+__device__ __forceinline__ bool tie_kept(const KArgs& a, uint32_t tid, uint32_t t_lo, uint64_t gidx) {
+  const uint4 l = stream_block<R, J0>(a, S_MASK_LO, tid, gidx >> 2);
+  return (pick(l, (unsigned)(gidx & 3)) >> 8) < t_lo;
+}
+
+
+// Keep decision of one element (any alignment).
+template <int R>
+__device__ __forceinline__ bool elem_kept(const KArgs& a, uint32_t tid, uint32_t t_hi,
+                                          uint32_t t_lo, uint64_t gidx) {
+  const uint4 w = stream_block<R>(a, S_MASK, tid, gidx >> 4);
+  const uint32_t hi = (pick(w, (unsigned)((gidx >> 2) & 3)) >> (8u * (unsigned)(gidx & 3))) & 0xFFu;
+  if (hi != t_hi) return hi < t_hi;
+  if (t_lo == 0u) return false;
+  const uint4 l = stream_block<R>(a, S_MASK_LO, tid, gidx >> 2);
+  return (pick(l, (unsigned)(gidx & 3)) >> 8) < t_lo;
+}
+
+// ------------------------------------------------------------ memory I/O ---
+__device__ __forceinline__ void ld32B(const void* p, uint32_t (&r)[8]) {
+  asm("ld.global.L1::no_allocate.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7])
+      : "l"(p));
+}
+__device__ __forceinline__ void st32B(void* p, const uint32_t (&r)[8]) {
+  asm volatile("st.global.v8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "r"(r[0]), "r"(r[1]),
+               "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+               : "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+// 16 consecutive elements starting at element i, kept as loaded (bf16: 8
+// words of two elements, fp32: 16 words); 32-byte aligned under TF_VEC.
+template <int DT>
+struct Raw16 {
+  uint32_t r[DT == DT_BF16 ? 8 : 16];
+  __device__ __forceinline__ float at(int e) const {
+    if (DT == DT_BF16) return __uint_as_float((e & 1) ? (r[e >> 1] & 0xFFFF0000u) : (r[e >> 1] << 16));
+    return __uint_as_float(r[e]);
+  }
+};
+
+template <int DT>
+__device__ __forceinline__ void load16(const void* base, int64_t i, Raw16<DT>& v) {
+  if (DT == DT_BF16) {
+    ld32B(static_cast<const uint16_t*>(base) + i, *reinterpret_cast<uint32_t(*)[8]>(v.r));
+  } else {
+    const float* p = static_cast<const float*>(base) + i;
+    ld32B(p, *reinterpret_cast<uint32_t(*)[8]>(v.r));
+    ld32B(p + 8, *reinterpret_cast<uint32_t(*)[8]>(v.r + 8));
+  }
+}
+
+template <int DT>
+__device__ __forceinline__ void store16(void* base, int64_t i, const float (&v)[16]) {
+  if (DT == DT_BF16) {
+    uint32_t r[8];
+#pragma unroll
+    for (int m = 0; m < 8; ++m) r[m] = pack_bf16x2(v[2 * m], v[2 * m + 1]);
+    st32B(static_cast<uint16_t*>(base) + i, r);
+  } else {
+    uint32_t r[8], s[8];
+#pragma unroll
+    for (int m = 0; m < 8; ++m) {
+      r[m] = __float_as_uint(v[m]);
+      s[m] = __float_as_uint(v[8 + m]);
+    }
+    float* p = static_cast<float*>(base) + i;
+    st32B(p, r);
+    st32B(p + 8, s);
+  }
+}
+
+template <int DT>
+__device__ __forceinline__ float load1(const void* base, int64_t i) {
+  if (DT == DT_BF16)
+    return __uint_as_float((uint32_t)(static_cast<const uint16_t*>(base)[i]) << 16);
+  return static_cast<const float*>(base)[i];
+}
+
+template <int DT>
+__device__ __forceinline__ void store1(void* base, int64_t i, float v) {
+  if (DT == DT_BF16) {
+    const __nv_bfloat16 h = __float2bfloat16_rn(v);
+    static_cast<__nv_bfloat16*>(base)[i] = h;
+  } else {
+    static_cast<float*>(base)[i] = v;
+  }
+}
+
+__device__ __forceinline__ float alpha_elem(const KArgs& a, uint32_t u) {
+  return __fmaf_rn(a.alpha_width, u01(u), a.alpha_min);
+}
+
+// Per-chunk view of one tensor's constants.
+struct TView {
+  int64_t off;
+  uint32_t tid, flags, t_hi, t_lo;
+  float inv_keep, c, noise_scale;
+  bool has_noise;
+};
+
+__device__ __forceinline__ TView make_view(const DevTensor& T, const DevScalars& S) {
+  TView v;
+  v.off = T.elem_offset;
+  v.tid = T.tid;
+  v.flags = T.flags;
+  v.t_hi = T.t_hi;
+  v.t_lo = T.t_lo;
+  v.inv_keep = T.inv_keep;
+  v.c = S.c;
+  v.noise_scale = S.noise_scale;
+  v.has_noise = S.sigma > 0.0f;
+  return v;
+}
+
+}  // namespace
+}  // namespace smat

@@ -1,0 +1,172 @@
+// Row a5 (gradient map) kernels and launchers.
+#include "smat_device.cuh"
+
+namespace smat {
+namespace {
+
+// ---------------------------------------------------------- a5: gradient map ---
+// When `defer` (no accumulation and g_out distinct from g_sim, so the
+// incoming gradient can be re-read), tie elements are written as dropped (+0)
+// and queued; otherwise they are resolved at once.
+template <int R, int GDT, bool PE, bool ACC, bool J0>
+__device__ __forceinline__ void grad_compute16(const KArgs& a, const TView& v, uint64_t g0, uint32_t off,
+                                               bool defer, TieList& tl, const Raw16<GDT>& gs,
+                                               const Raw16<GDT>& go, float (&out)[16]) {
+  uint32_t kw[4] = {0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u};
+  if (v.flags & TF_MASK) {
+    if (ACC || !defer) {
+      group_keep16<R, J0>(a, v.tid, v.t_hi, v.t_lo, g0, kw, nullptr);
+    } else {
+      uint32_t ties = 0u;
+      group_keep16<R, J0>(a, v.tid, v.t_hi, v.t_lo, g0, kw, &ties);
+      while (ties) {
+        const int e = __ffs(ties) - 1;
+        ties &= ties - 1u;
+        if (!tl.push(off + (uint32_t)e) && tie_kept<R, J0>(a, v.tid, v.t_lo, g0 + (uint64_t)e))
+          set_kept(kw, e);
+      }
+    }
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    uint4 aw = make_uint4(0u, 0u, 0u, 0u);
+    if (PE) aw = stream_block<R, J0>(a, S_ALPHA_E, v.tid, (g0 >> 2) + q);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int e = 4 * q + k;
+      const float c = PE ? __fmul_rn(alpha_elem(a, pick(aw, k)), v.inv_keep) : v.c;
+      float g = kept_of(kw, e) ? __fmul_rn(c, gs.at(e)) : 0.0f;
+      if (ACC) g = __fadd_rn(go.at(e), g);
+      out[e] = g;
+    }
+  }
+}
+
+template <int R, int GDT, bool PE, bool ACC>
+__device__ __forceinline__ void grad_elem_as(const KArgs& a, const TView& v, const GradPtr& G, int64_t e,
+                                             bool kept) {
+  const uint64_t g = (uint64_t)(v.off + e);
+  float c = v.c;
+  if (PE) {
+    const uint4 w = stream_block<R>(a, S_ALPHA_E, v.tid, g >> 2);
+    c = __fmul_rn(alpha_elem(a, pick(w, (unsigned)(g & 3))), v.inv_keep);
+  }
+  float r = kept ? __fmul_rn(c, load1<GDT>(G.g_sim, e)) : 0.0f;
+  if (ACC) r = __fadd_rn(load1<GDT>(G.g_out, e), r);
+  store1<GDT>(G.g_out, e, r);
+}
+
+// Two groups per iteration (strides apart) so each thread keeps two loads of
+// g~ in flight before the mask work.
+template <int R, int GDT, bool PE, bool ACC, bool J0>
+__device__ __forceinline__ void grad_chunk(const KArgs& a, const TView& v, const GradPtr& G, const Chunk& ch) {
+  constexpr int64_t kStride = 16 * (int64_t)kBlock;
+  const bool masked = (v.flags & TF_MASK) != 0u;
+  const bool defer = !ACC && G.g_sim != G.g_out;
+  TieList tl;
+  for (int64_t i = ch.begin + 16 * (int64_t)threadIdx.x; i < ch.end; i += 2 * kStride) {
+    const int64_t i2 = i + kStride;
+    if (G.vec && i2 + 16 <= ch.end) {
+      Raw16<GDT> gs1, gs2, go1, go2;
+      load16<GDT>(G.g_sim, i, gs1);
+      load16<GDT>(G.g_sim, i2, gs2);
+      if (ACC) {
+        load16<GDT>(G.g_out, i, go1);
+        load16<GDT>(G.g_out, i2, go2);
+      }
+      float out[16];
+      grad_compute16<R, GDT, PE, ACC, J0>(a, v, (uint64_t)(v.off + i), (uint32_t)(i - ch.begin), defer, tl, gs1, go1, out);
+      store16<GDT>(G.g_out, i, out);
+      grad_compute16<R, GDT, PE, ACC, J0>(a, v, (uint64_t)(v.off + i2), (uint32_t)(i2 - ch.begin), defer, tl, gs2, go2, out);
+      store16<GDT>(G.g_out, i2, out);
+    } else {
+      for (int half = 0; half < 2; ++half) {
+        const int64_t b = half ? i2 : i;
+        if (b >= ch.end) break;
+        if (G.vec && b + 16 <= ch.end) {
+          Raw16<GDT> gs1, go1;
+          load16<GDT>(G.g_sim, b, gs1);
+          if (ACC) load16<GDT>(G.g_out, b, go1);
+          float out[16];
+          grad_compute16<R, GDT, PE, ACC, J0>(a, v, (uint64_t)(v.off + b), (uint32_t)(b - ch.begin), defer, tl, gs1, go1, out);
+          store16<GDT>(G.g_out, b, out);
+        } else {
+          const int64_t e_end = (b + 16 < ch.end) ? b + 16 : ch.end;
+          for (int64_t e = b; e < e_end; ++e) {
+            const bool kept = masked ? elem_kept<R>(a, v.tid, v.t_hi, v.t_lo, (uint64_t)(v.off + e)) : true;
+            grad_elem_as<R, GDT, PE, ACC>(a, v, G, e, kept);
+          }
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    if (k < tl.n) {
+      const int64_t e = ch.begin + (int64_t)tl.at(k);
+      if (tie_kept<R, J0>(a, v.tid, v.t_lo, (uint64_t)(v.off + e))) grad_elem_as<R, GDT, PE, ACC>(a, v, G, e, true);
+    }
+  }
+}
+
+template <int R, int GDT, bool PE, bool ACC>
+__global__ void __launch_bounds__(kBlock, (GDT == DT_BF16 && !ACC) ? 3 : 2) gradmap_kernel(const __grid_constant__ KArgs a) {
+  for (int64_t ci = a.chunk_begin + blockIdx.x; ci < a.chunk_end; ci += gridDim.x) {
+    const Chunk ch = a.chunks[ci];
+    const DevTensor& T = a.tensors[ch.tensor];
+    const GradPtr G = a.grads[ch.tensor];
+    const TView v = make_view(T, a.scal[ch.tensor]);
+    if ((uint64_t)(v.off + ch.end) <= (uint64_t(1) << 34))
+      grad_chunk<R, GDT, PE, ACC, true>(a, v, G, ch);
+    else
+      grad_chunk<R, GDT, PE, ACC, false>(a, v, G, ch);
+  }
+}
+
+
+template <typename Kernel>
+int occupancy_of(Kernel k) {
+  int v = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, k, kBlock, 0) != cudaSuccess || v < 1) v = 1;
+  return v;
+}
+
+template <int R, int GDT, bool PE, bool ACC>
+int grad_occ() {
+  static int v = occupancy_of(gradmap_kernel<R, GDT, PE, ACC>);
+  return v;
+}
+template <int R, int GDT, bool PE, bool ACC>
+cudaError_t grad_run(const KArgs& a, int grid, cudaStream_t s) {
+  gradmap_kernel<R, GDT, PE, ACC><<<grid, kBlock, 0, s>>>(a);
+  return cudaGetLastError();
+}
+template <int R, int GDT>
+cudaError_t grad_flags(const KArgs& a, int grid, bool pe, bool acc, cudaStream_t s) {
+  if (pe) return acc ? grad_run<R, GDT, true, true>(a, grid, s) : grad_run<R, GDT, true, false>(a, grid, s);
+  return acc ? grad_run<R, GDT, false, true>(a, grid, s) : grad_run<R, GDT, false, false>(a, grid, s);
+}
+template <int R>
+cudaError_t grad_dt(const KArgs& a, int grid, int gdt, bool pe, bool acc, cudaStream_t s) {
+  return gdt == DT_BF16 ? grad_flags<R, DT_BF16>(a, grid, pe, acc, s)
+                        : grad_flags<R, DT_F32>(a, grid, pe, acc, s);
+}
+
+}  // namespace
+
+cudaError_t launch_gradmap(const KArgs& a, int grid, int gdtype, bool per_elem_alpha, bool accumulate,
+                           int rounds, cudaStream_t s) {
+  if (a.chunk_end <= a.chunk_begin) return cudaSuccess;
+  return rounds == 7 ? grad_dt<7>(a, grid, gdtype, per_elem_alpha, accumulate, s)
+                     : grad_dt<10>(a, grid, gdtype, per_elem_alpha, accumulate, s);
+}
+
+int gradmap_ctas_per_sm(int gdtype, bool pe, bool acc, int rounds) {
+#define SMAT_GOCC(R, G) (pe ? (acc ? grad_occ<R, G, true, true>() : grad_occ<R, G, true, false>()) \
+                           : (acc ? grad_occ<R, G, false, true>() : grad_occ<R, G, false, false>()))
+  if (rounds == 7) return gdtype == DT_BF16 ? SMAT_GOCC(7, DT_BF16) : SMAT_GOCC(7, DT_F32);
+  return gdtype == DT_BF16 ? SMAT_GOCC(10, DT_BF16) : SMAT_GOCC(10, DT_F32);
+#undef SMAT_GOCC
+}
+
+}  // namespace smat

@@ -530,6 +530,18 @@ smat_status smat_debug_philox(const uint32_t* d_ctr, int64_t n, uint64_t seed, i
   return SMAT_OK;
 }
 
+smat_status smat_debug_noise_unit(const uint32_t* d_words, int64_t n, int32_t noise, float* d_out,
+                                  smat_stream_t stream) {
+  if (n < 0) return fail(SMAT_ERR_INVALID_ARG, "n < 0");
+  if (n == 0) return SMAT_OK;
+  if (!d_words || !d_out) return fail(SMAT_ERR_INVALID_ARG, "NULL pointer");
+  if (noise != SMAT_NOISE_UNIFORM && noise != SMAT_NOISE_GAUSSIAN)
+    return fail(SMAT_ERR_UNSUPPORTED, "noise %d not supported", noise);
+  const cudaError_t e = launch_debug_noise_unit(d_words, n, noise, d_out, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "noise transform launch");
+  return SMAT_OK;
+}
+
 const char* smat_status_string(smat_status s) {
   switch (s) {
     case SMAT_OK: return "SMAT_OK";

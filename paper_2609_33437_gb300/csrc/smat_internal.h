@@ -93,16 +93,24 @@ struct KArgs {
   int32_t with_sigma;    // scalars: 1 = derive sigma_t from the delta-statistics partials
 };
 
-// Kernel launchers (smat_kernels.cu). Each returns the launch's error code.
+// Kernel launchers (smat_aux.cu, smat_gradmap.cu, smat_sim_*.cu). Each
+// returns the launch's error code.
 cudaError_t launch_delta_stats(const KArgs& a, int grid, int dtype, cudaStream_t s);
 cudaError_t launch_scalars(const KArgs& a, int noise, int rounds, cudaStream_t s);
 cudaError_t launch_simulate(const KArgs& a, int grid, int dtype, int noise, bool per_elem_alpha,
                             int rounds, cudaStream_t s);
 cudaError_t launch_gradmap(const KArgs& a, int grid, int gdtype, bool per_elem_alpha, bool accumulate,
                            int rounds, cudaStream_t s);
+cudaError_t launch_simulate_f32(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
+                                cudaStream_t s);
+cudaError_t launch_simulate_bf16(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
+                                 cudaStream_t s);
+int simulate_ctas_per_sm_f32(int noise, bool per_elem_alpha, int rounds);
+int simulate_ctas_per_sm_bf16(int noise, bool per_elem_alpha, int rounds);
 cudaError_t launch_mask_bits(const KArgs& a, int64_t numel, int rounds, cudaStream_t s);
 cudaError_t launch_debug_philox(const uint32_t* ctr, int64_t n, const RoundKeys& key, int rounds,
                                 uint32_t* out, uint32_t* out_ref, cudaStream_t s);
+cudaError_t launch_debug_noise_unit(const uint32_t* words, int64_t n, int noise, float* out, cudaStream_t s);
 // Resident CTAs per SM of the streaming kernels (for grid sizing).
 int streaming_ctas_per_sm(int dtype, int noise, bool per_elem_alpha, int rounds);
 int gradmap_ctas_per_sm(int gdtype, bool per_elem_alpha, bool accumulate, int rounds);

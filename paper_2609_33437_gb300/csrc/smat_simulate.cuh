@@ -1,0 +1,169 @@
+// Row a3 (forward) kernels, instantiated per parameter dtype by
+// smat_sim_f32.cu and smat_sim_bf16.cu so the two compile in parallel.
+#pragma once
+#include "smat_device.cuh"
+
+namespace smat {
+namespace {
+
+// --------------------------------------------------------------- a3: forward ---
+// One 16-element group on the vector path. IDENT: c == 1 for the whole tensor
+// (kept elements are theta itself); only used without per-element alpha.
+// Tie elements are written as dropped and queued in tl (resolved at the end
+// of the chunk); if the queue is full they are resolved here.
+template <int R, int DT, int NOISE, bool PE, bool IDENT, bool J0>
+__device__ __forceinline__ void sim_group16(const KArgs& a, const TView& v, const void* th_p,
+                                            const void* t0_p, void* sim_p, int64_t i, uint32_t off,
+                                            TieList& tl) {
+  const uint64_t g0 = (uint64_t)(v.off + i);
+  Raw16<DT> th, t0;
+  load16<DT>(th_p, i, th);
+  load16<DT>(t0_p, i, t0);
+  uint32_t kw[4] = {0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u};
+  if (v.flags & TF_MASK) {
+    uint32_t ties = 0u;
+    group_keep16<R, J0>(a, v.tid, v.t_hi, v.t_lo, g0, kw, &ties);
+    while (ties) {
+      const int e = __ffs(ties) - 1;
+      ties &= ties - 1u;
+      if (!tl.push(off + (uint32_t)e) && tie_kept<R, J0>(a, v.tid, v.t_lo, g0 + (uint64_t)e))
+        set_kept(kw, e);
+    }
+  }
+  float out[16];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    uint4 nw = make_uint4(0u, 0u, 0u, 0u);
+    if (NOISE != NOISE_NONE) nw = stream_block<R, J0>(a, S_NOISE, v.tid, (g0 >> 2) + q);
+    uint4 aw = make_uint4(0u, 0u, 0u, 0u);
+    if (PE) aw = stream_block<R, J0>(a, S_ALPHA_E, v.tid, (g0 >> 2) + q);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int e = 4 * q + k;
+      const float x_th = th.at(e), x_t0 = t0.at(e);
+      float kept_val;
+      if (PE) {
+        const float c = __fmul_rn(alpha_elem(a, pick(aw, k)), v.inv_keep);
+        kept_val = (c == 1.0f) ? x_th : __fmaf_rn(c, __fsub_rn(x_th, x_t0), x_t0);
+      } else if (IDENT) {
+        kept_val = x_th;
+      } else {
+        kept_val = __fmaf_rn(v.c, __fsub_rn(x_th, x_t0), x_t0);
+      }
+      float x = kept_of(kw, e) ? kept_val : x_t0;
+      if (NOISE != NOISE_NONE) x = __fadd_rn(x, noise_of<NOISE>(pick(nw, k), v.noise_scale));
+      out[e] = x;
+    }
+  }
+  store16<DT>(sim_p, i, out);
+}
+
+// One element given its keep decision (any alignment).
+template <int R, int DT, int NOISE, bool PE>
+__device__ __forceinline__ void sim_elem_as(const KArgs& a, const TView& v, const void* th_p,
+                                            const void* t0_p, void* sim_p, int64_t e, bool kept) {
+  const uint64_t g = (uint64_t)(v.off + e);
+  float c = v.c;
+  if (PE) {
+    const uint4 w = stream_block<R>(a, S_ALPHA_E, v.tid, g >> 2);
+    c = __fmul_rn(alpha_elem(a, pick(w, (unsigned)(g & 3))), v.inv_keep);
+  }
+  const float x_th = load1<DT>(th_p, e), x_t0 = load1<DT>(t0_p, e);
+  float x = x_t0;
+  if (kept) x = (c == 1.0f) ? x_th : __fmaf_rn(c, __fsub_rn(x_th, x_t0), x_t0);
+  if (NOISE != NOISE_NONE)
+    x = __fadd_rn(x, noise_of<NOISE>(pick(stream_block<R>(a, S_NOISE, v.tid, g >> 2), (unsigned)(g & 3)),
+                                     v.noise_scale));
+  store1<DT>(sim_p, e, x);
+}
+
+template <int R, int DT, int NOISE, bool PE, bool IDENT, bool J0>
+__device__ __forceinline__ void sim_chunk(const KArgs& a, const TView& v, const DevTensor& T,
+                                          const Chunk& ch) {
+  const bool vec = (v.flags & TF_VEC) != 0u;
+  const bool masked = (v.flags & TF_MASK) != 0u;
+  TieList tl;
+  for (int64_t i = ch.begin + 16 * (int64_t)threadIdx.x; i < ch.end; i += 16 * (int64_t)kBlock) {
+    if (vec && i + 16 <= ch.end) {
+      sim_group16<R, DT, NOISE, PE, IDENT, J0>(a, v, T.theta, T.theta0, T.sim, i, (uint32_t)(i - ch.begin), tl);
+    } else {
+      const int64_t e_end = (i + 16 < ch.end) ? i + 16 : ch.end;
+      for (int64_t e = i; e < e_end; ++e) {
+        const bool kept = masked ? elem_kept<R>(a, v.tid, v.t_hi, v.t_lo, (uint64_t)(v.off + e)) : true;
+        sim_elem_as<R, DT, NOISE, PE>(a, v, T.theta, T.theta0, T.sim, e, kept);
+      }
+    }
+  }
+  // queued ties: rewrite the few that the low 24 bits keep
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    if (k < tl.n) {
+      const int64_t e = ch.begin + (int64_t)tl.at(k);
+      if (tie_kept<R, J0>(a, v.tid, v.t_lo, (uint64_t)(v.off + e)))
+        sim_elem_as<R, DT, NOISE, PE>(a, v, T.theta, T.theta0, T.sim, e, true);
+    }
+  }
+}
+
+template <int R, int DT, int NOISE, bool PE, bool IDENT, bool J0>
+__device__ __forceinline__ void sim_chunk_noise(const KArgs& a, const TView& v, const DevTensor& T,
+                                                const Chunk& ch) {
+  if (v.has_noise)
+    sim_chunk<R, DT, NOISE, PE, IDENT, J0>(a, v, T, ch);
+  else
+    sim_chunk<R, DT, NOISE_NONE, PE, IDENT, J0>(a, v, T, ch);
+}
+
+template <int R, int DT, int NOISE, bool PE>
+__global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 4 : 2) simulate_kernel(const __grid_constant__ KArgs a) {
+  for (int64_t ci = a.chunk_begin + blockIdx.x; ci < a.chunk_end; ci += gridDim.x) {
+    const Chunk ch = a.chunks[ci];
+    const DevTensor& T = a.tensors[ch.tensor];
+    const TView v = make_view(T, a.scal[ch.tensor]);
+    const bool j0 = (uint64_t)(v.off + ch.end) <= (uint64_t(1) << 34);  // gidx >> 2 < 2^32
+    if (!PE && v.c == 1.0f) {
+      if (j0) sim_chunk_noise<R, DT, NOISE, PE, true, true>(a, v, T, ch);
+      else sim_chunk_noise<R, DT, NOISE, PE, true, false>(a, v, T, ch);
+    } else {
+      if (j0) sim_chunk_noise<R, DT, NOISE, PE, false, true>(a, v, T, ch);
+      else sim_chunk_noise<R, DT, NOISE, PE, false, false>(a, v, T, ch);
+    }
+  }
+}
+
+
+template <typename Kernel>
+int occupancy_of(Kernel k) {
+  int v = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, k, kBlock, 0) != cudaSuccess || v < 1) v = 1;
+  return v;
+}
+
+template <int R, int DT, int NOISE, bool PE>
+struct SimVariant {
+  static int occ() {
+    static int v = occupancy_of(simulate_kernel<R, DT, NOISE, PE>);
+    return v;
+  }
+  static cudaError_t run(const KArgs& a, int grid, cudaStream_t s) {
+    simulate_kernel<R, DT, NOISE, PE><<<grid, kBlock, 0, s>>>(a);
+    return cudaGetLastError();
+  }
+};
+
+template <int R, int DT>
+cudaError_t sim_run(const KArgs& a, int grid, int noise, bool pe, cudaStream_t s) {
+  if (noise == NOISE_GAUSSIAN)
+    return pe ? SimVariant<R, DT, NOISE_GAUSSIAN, true>::run(a, grid, s) : SimVariant<R, DT, NOISE_GAUSSIAN, false>::run(a, grid, s);
+  return pe ? SimVariant<R, DT, NOISE_UNIFORM, true>::run(a, grid, s) : SimVariant<R, DT, NOISE_UNIFORM, false>::run(a, grid, s);
+}
+
+template <int R, int DT>
+int sim_occ(int noise, bool pe) {
+  if (noise == NOISE_GAUSSIAN)
+    return pe ? SimVariant<R, DT, NOISE_GAUSSIAN, true>::occ() : SimVariant<R, DT, NOISE_GAUSSIAN, false>::occ();
+  return pe ? SimVariant<R, DT, NOISE_UNIFORM, true>::occ() : SimVariant<R, DT, NOISE_UNIFORM, false>::occ();
+}
+
+}  // namespace
+}  // namespace smat

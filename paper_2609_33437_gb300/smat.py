@@ -24,7 +24,7 @@ SMAT_ALPHA_GLOBAL, SMAT_ALPHA_PER_TENSOR, SMAT_ALPHA_PER_ELEMENT = 0, 1, 2
 
 EXPORTED = ("smat_workspace_bytes", "smat_init", "smat_simulate_multi", "smat_grad_map_multi",
             "smat_swap", "smat_active", "smat_mask_bits", "smat_tensor_scalars", "smat_destroy",
-            "smat_debug_philox", "smat_timing_enable", "smat_timing_read", "smat_status_string",
+            "smat_debug_philox", "smat_debug_noise_unit", "smat_timing_enable", "smat_timing_read", "smat_status_string",
             "smat_last_error", "smat_abi_version")
 
 
@@ -76,6 +76,7 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
     L.smat_tensor_scalars.argtypes = [P, U32, P, P]
     L.smat_destroy.argtypes = [P]
     L.smat_debug_philox.argtypes = [P, I64, U64, I32, P, P, P]
+    L.smat_debug_noise_unit.argtypes = [P, I64, I32, P, P]
     L.smat_timing_enable.argtypes = [P, I32]
     L.smat_timing_read.argtypes = [P, P, P]
     L.smat_status_string.argtypes = [I32]
@@ -84,7 +85,7 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
     L.smat_last_error.restype = ctypes.c_char_p
     L.smat_abi_version.restype = I32
     for name in ("smat_init", "smat_simulate_multi", "smat_grad_map_multi", "smat_swap", "smat_active",
-                 "smat_mask_bits", "smat_tensor_scalars", "smat_destroy", "smat_debug_philox",
+                 "smat_mask_bits", "smat_tensor_scalars", "smat_destroy", "smat_debug_philox", "smat_debug_noise_unit",
                  "smat_timing_enable", "smat_timing_read"):
         getattr(L, name).restype = I32
     _lib = L
@@ -264,6 +265,17 @@ def debug_philox(ctr: torch.Tensor, seed: int, rounds: int = 10, with_curand: bo
                                                    ctypes.c_void_p(ref.data_ptr() if ref is not None else 0),
                                                    _stream_handle(stream)))
     return out, ref
+
+
+def debug_noise_unit(words: torch.Tensor, noise: int, stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:
+    """Unit noise transform of raw words (int32 CUDA tensor): sym(w) or
+    erfinv(sym(w)) exactly as the forward evaluates it."""
+    L = load_library()
+    words = words.contiguous()
+    out = torch.empty(words.shape, dtype=torch.float32, device=words.device)
+    check("smat_debug_noise_unit", L.smat_debug_noise_unit(ctypes.c_void_p(words.data_ptr()), words.numel(), int(noise),
+                                                           ctypes.c_void_p(out.data_ptr()), _stream_handle(stream)))
+    return out
 
 
 class SmatParameters:
