@@ -17,7 +17,7 @@ LIB = os.path.join(PKG, "libsmat.so")
 
 SOURCES = ["smat_sim_bf16.cu", "smat_sim_f32.cu", "smat_gradmap.cu", "smat_aux.cu", "smat_host.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
+FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-fmad=false", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "--expt-relaxed-constexpr", "-I", INCLUDE, "-I", CSRC]
 
 

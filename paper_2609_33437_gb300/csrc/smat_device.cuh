@@ -121,10 +121,88 @@ __device__ __forceinline__ float erfinv_poly(float x) {
   return __fmul_rn(x, p);
 }
 
+// Packed fp32 pairs (sm_100 and later): two independent IEEE operations with
+// round-to-nearest in one instruction. Written as PTX with an explicit .rn
+// modifier: an operation with an explicit rounding mode is never contracted
+// with a neighbour into a fused multiply-add, so each one rounds exactly as
+// the specification's scalar operation does.
+__device__ __forceinline__ float2 splat(float v) { return make_float2(v, v); }
+
+__device__ __forceinline__ float2 mul2_rn(float2 a, float2 b) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+      "mul.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+
+__device__ __forceinline__ float2 add2_rn(float2 a, float2 b) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+      "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+
+__device__ __forceinline__ float2 fma2_rn(float2 a, float2 b, float2 c) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+      "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  return d;
+}
+
+__device__ __forceinline__ float2 sym2(uint32_t u0, uint32_t u1) {
+  const int k0 = (int)(u0 >> 8), k1 = (int)(u1 >> 8);
+  const float2 m = make_float2(__int2float_rn(2 * k0 + 1 - (1 << 24)), __int2float_rn(2 * k1 + 1 - (1 << 24)));
+  return mul2_rn(m, splat(5.9604644775390625e-08f));
+}
+
+__device__ __forceinline__ float lg2_approx(float t) {
+  float L;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(L) : "f"(t));
+  return L;
+}
+
+// erfinv_poly on a pair: the central polynomial with packed multiply-adds
+// when both lanes are central (99.6% of pairs), else lane by lane.
+__device__ __forceinline__ float2 erfinv_poly2(float2 x) {
+  const float2 t = fma2_rn(make_float2(-x.x, -x.y), x, splat(1.0f));
+  const float2 L = make_float2(lg2_approx(t.x), lg2_approx(t.y));
+  float2 p;
+  if (fminf(L.x, L.y) >= -8.0f) {
+    p = splat(2.676246447e-10f);
+    p = fma2_rn(p, L, splat(9.962457526e-09f));
+    p = fma2_rn(p, L, splat(1.280022701e-07f));
+    p = fma2_rn(p, L, splat(2.725655577e-07f));
+    p = fma2_rn(p, L, splat(-7.822631233e-06f));
+    p = fma2_rn(p, L, splat(-3.107573502e-05f));
+    p = fma2_rn(p, L, splat(7.751958910e-04f));
+    p = fma2_rn(p, L, splat(5.547157954e-03f));
+    p = fma2_rn(p, L, splat(-1.608200818e-01f));
+    p = fma2_rn(p, L, splat(8.862268925e-01f));
+    return mul2_rn(x, p);
+  }
+  return make_float2(erfinv_poly(x.x), erfinv_poly(x.y));
+}
+
 // Perturb of one element from its noise word: uniform scale * sym(n) with
 // scale = fl(sqrt3 sigma), or Gaussian scale * erfinv(sym(n)) with
 // scale = fl(sqrt2 sigma) (inverse-CDF transform: sqrt2 erfinv(v) is
 // N(0, 1) for v uniform on (-1, 1)).
+template <int NOISE>
+__device__ __forceinline__ float2 noise_of2(uint32_t n0, uint32_t n1, float2 scale) {
+  if (NOISE == NOISE_UNIFORM) return mul2_rn(scale, sym2(n0, n1));
+  if (NOISE == NOISE_GAUSSIAN) return mul2_rn(scale, erfinv_poly2(sym2(n0, n1)));
+  return splat(0.0f);
+}
+
 template <int NOISE>
 __device__ __forceinline__ float noise_of(uint32_t n, float scale) {
   if (NOISE == NOISE_UNIFORM) return __fmul_rn(scale, sym(n));
@@ -266,6 +344,11 @@ struct Raw16 {
   __device__ __forceinline__ float at(int e) const {
     if (DT == DT_BF16) return __uint_as_float((e & 1) ? (r[e >> 1] & 0xFFFF0000u) : (r[e >> 1] << 16));
     return __uint_as_float(r[e]);
+  }
+  // elements 2m and 2m + 1
+  __device__ __forceinline__ float2 pair(int m) const {
+    if (DT == DT_BF16) return make_float2(__uint_as_float(r[m] << 16), __uint_as_float(r[m] & 0xFFFF0000u));
+    return make_float2(__uint_as_float(r[2 * m]), __uint_as_float(r[2 * m + 1]));
   }
 };
 

@@ -31,6 +31,8 @@ __device__ __forceinline__ void sim_group16(const KArgs& a, const TView& v, cons
     }
   }
   float out[16];
+  const float2 c2 = splat(v.c);
+  const float2 scale2 = splat(v.noise_scale);
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     uint4 nw = make_uint4(0u, 0u, 0u, 0u);
@@ -38,21 +40,29 @@ __device__ __forceinline__ void sim_group16(const KArgs& a, const TView& v, cons
     uint4 aw = make_uint4(0u, 0u, 0u, 0u);
     if (PE) aw = stream_block<R, J0>(a, S_ALPHA_E, v.tid, (g0 >> 2) + q);
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const int e = 4 * q + k;
-      const float x_th = th.at(e), x_t0 = t0.at(e);
-      float kept_val;
+    for (int h = 0; h < 2; ++h) {
+      const int e0 = 4 * q + 2 * h;  // elements e0, e0 + 1
+      const float2 th2 = th.pair(e0 >> 1), t02 = t0.pair(e0 >> 1);
+      float2 kv;
       if (PE) {
-        const float c = __fmul_rn(alpha_elem(a, pick(aw, k)), v.inv_keep);
-        kept_val = (c == 1.0f) ? x_th : __fmaf_rn(c, __fsub_rn(x_th, x_t0), x_t0);
+        const float2 cc = make_float2(__fmul_rn(alpha_elem(a, pick(aw, 2 * h)), v.inv_keep),
+                                      __fmul_rn(alpha_elem(a, pick(aw, 2 * h + 1)), v.inv_keep));
+        const float2 f = fma2_rn(cc, add2_rn(th2, make_float2(-t02.x, -t02.y)), t02);
+        kv = make_float2(cc.x == 1.0f ? th2.x : f.x, cc.y == 1.0f ? th2.y : f.y);
       } else if (IDENT) {
-        kept_val = x_th;
+        kv = th2;
       } else {
-        kept_val = __fmaf_rn(v.c, __fsub_rn(x_th, x_t0), x_t0);
+        kv = fma2_rn(c2, add2_rn(th2, make_float2(-t02.x, -t02.y)), t02);
       }
-      float x = kept_of(kw, e) ? kept_val : x_t0;
-      if (NOISE != NOISE_NONE) x = __fadd_rn(x, noise_of<NOISE>(pick(nw, k), v.noise_scale));
-      out[e] = x;
+      float x0 = kept_of(kw, e0) ? kv.x : t02.x;
+      float x1 = kept_of(kw, e0 + 1) ? kv.y : t02.y;
+      if (NOISE != NOISE_NONE) {
+        const float2 eps = noise_of2<NOISE>(pick(nw, 2 * h), pick(nw, 2 * h + 1), scale2);
+        x0 = __fadd_rn(x0, eps.x);
+        x1 = __fadd_rn(x1, eps.y);
+      }
+      out[e0] = x0;
+      out[e0 + 1] = x1;
     }
   }
   store16<DT>(sim_p, i, out);
@@ -115,7 +125,7 @@ __device__ __forceinline__ void sim_chunk_noise(const KArgs& a, const TView& v, 
 }
 
 template <int R, int DT, int NOISE, bool PE>
-__global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 4 : 2) simulate_kernel(const __grid_constant__ KArgs a) {
+__global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 3 : 2) simulate_kernel(const __grid_constant__ KArgs a) {
   for (int64_t ci = a.chunk_begin + blockIdx.x; ci < a.chunk_end; ci += gridDim.x) {
     const Chunk ch = a.chunks[ci];
     const DevTensor& T = a.tensors[ch.tensor];
