@@ -94,6 +94,9 @@ typedef struct {
   float sigma_rel;     /* >= 0; if > 0, sigma_t = sigma_rel * std(theta - theta0) at each call */
 } smat_tensor_desc;
 
+/* smat_config.flags */
+#define SMAT_FLAG_UNFUSED_STATS 1 /* run delta statistics as a separate pass before the forward */
+
 typedef struct {
   uint64_t seed;         /* Philox key */
   float alpha_min;       /* Scale: alpha ~ U[alpha_min, alpha_max); paper: alpha_max = 1 */
@@ -101,6 +104,7 @@ typedef struct {
   int32_t alpha_mode;    /* smat_alpha_mode */
   int32_t noise;         /* smat_noise */
   int32_t philox_rounds; /* 10 (default) or 7 */
+  int32_t flags;         /* SMAT_FLAG_*; 0 = defaults */
 } smat_config;
 
 /* Bytes of device workspace smat_init needs for this tensor list (0 on
@@ -119,10 +123,13 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
                       smat_stream_t stream);
 
 /* Forward (Eq. smat-state) for every tensor at SMAT step `step`: computes the
- * per-call scalars (and, for sigma_rel tensors, the delta statistics first)
- * and writes theta~ into each tensor's `sim`. Requires the original storage to
- * be active (SMAT_ERR_STATE otherwise): the simulated state is rebuilt only
- * while the model reads theta. */
+ * per-call scalars (and, for sigma_rel tensors, the delta statistics) and
+ * writes theta~ into each tensor's `sim`. Requires the original storage to be
+ * active (SMAT_ERR_STATE otherwise): the simulated state is rebuilt only
+ * while the model reads theta. With sigma_rel tensors the statistics and the
+ * forward run in one persistent launch by default (statistics of later
+ * tensors beside the forward of earlier ones); SMAT_FLAG_UNFUSED_STATS runs
+ * them as two passes. Results are identical either way. */
 smat_status smat_simulate_multi(smat_ctx* ctx, uint32_t step, smat_stream_t stream);
 
 /* Gradient map (Eq. smat-gradient) at step `step`: for tensor k,
@@ -177,10 +184,27 @@ smat_status smat_debug_philox(const uint32_t* d_ctr, int64_t n, uint64_t seed, i
 smat_status smat_debug_noise_unit(const uint32_t* d_words, int64_t n, int32_t noise, float* d_out,
                                   smat_stream_t stream);
 
+/* Read and clear the context's device error flags (bit 0: a forward item of
+ * the fused launch gave up waiting for its tensor's statistics after about a
+ * second and was skipped, so that call's output is incomplete). Synchronises
+ * `stream`. *errors_out receives the flags (0 = none). */
+smat_status smat_poll_errors(smat_ctx* ctx, smat_stream_t stream, int32_t* errors_out);
+
+/* Test hook: run the fused statistics + forward launch of the bf16 range
+ * over a caller-given device list of n_items work items (chunk index, high
+ * bit set for a forward item) with the ready flags expected at an epoch that
+ * is `epoch_skew` calls ahead. With epoch_skew != 0 no flag ever matches, so
+ * every forward item of a sigma_rel tensor waits until its bounded wait runs
+ * out (about a second), sets error bit 0 and is skipped; the host then reads
+ * the bit with smat_poll_errors. Requires a context with sigma_rel tensors. */
+smat_status smat_debug_fused(smat_ctx* ctx, uint32_t step, const int32_t* d_items, int32_t n_items,
+                             uint32_t epoch_skew, smat_stream_t stream);
+
 /* Per-kernel timing (for measurement): while enabled, every kernel this
  * context launches is bracketed by two CUDA events recorded on the launching
- * stream. Kinds: 0 delta statistics (a2), 1 per-call scalars (a1),
- * 2 forward (a3), 3 gradient map (a5). Enabling clears the totals. Host-side
+ * stream. Kinds: 0 delta statistics (a2, unfused), 1 per-call scalars (a1),
+ * 2 forward (a3; with fused statistics when they are fused), 3 gradient map
+ * (a5). Enabling clears the totals. Host-side
  * events only; no device memory is allocated. */
 smat_status smat_timing_enable(smat_ctx* ctx, int32_t enable);
 

@@ -6,59 +6,21 @@ namespace smat {
 namespace {
 
 // -------------------------------------------------------- a2: delta sums ---
-__device__ __forceinline__ double warp_sum(double x) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
-  return x;
-}
 
 template <int DT>
 __global__ void __launch_bounds__(kBlock) delta_stats_kernel(const __grid_constant__ KArgs a) {
   __shared__ double sh_s[kBlock / 32];
   __shared__ double sh_q[kBlock / 32];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int64_t ci = a.chunk_begin + blockIdx.x; ci < a.chunk_end; ci += gridDim.x) {
     const Chunk ch = a.chunks[ci];
     const DevTensor& T = a.tensors[ch.tensor];
     if (!(T.flags & TF_SIGMA_REL)) continue;  // uniform across the CTA
-    const bool vec = (T.flags & TF_VEC) != 0u;
-    float s = 0.0f, q = 0.0f;
-    for (int64_t i = ch.begin + 16 * (int64_t)threadIdx.x; i < ch.end; i += 16 * (int64_t)kBlock) {
-      if (vec && i + 16 <= ch.end) {
-        Raw16<DT> th, t0;
-        load16<DT>(T.theta, i, th);
-        load16<DT>(T.theta0, i, t0);
-#pragma unroll
-        for (int k = 0; k < 16; ++k) {
-          const float d = __fsub_rn(th.at(k), t0.at(k));
-          s += d;
-          q = __fmaf_rn(d, d, q);
-        }
-      } else {
-        const int64_t e_end = (i + 16 < ch.end) ? i + 16 : ch.end;
-        for (int64_t e = i; e < e_end; ++e) {
-          const float d = __fsub_rn(load1<DT>(T.theta, e), load1<DT>(T.theta0, e));
-          s += d;
-          q = __fmaf_rn(d, d, q);
-        }
-      }
-    }
-    double ds = warp_sum((double)s), dq = warp_sum((double)q);
-    if (lane == 0) {
-      sh_s[warp] = ds;
-      sh_q[warp] = dq;
-    }
-    __syncthreads();
+    double ds, dq;
+    chunk_delta_sums<DT>(T, ch, sh_s, sh_q, ds, dq);
     if (threadIdx.x == 0) {
-      double ts = 0.0, tq = 0.0;
-      for (int w = 0; w < kBlock / 32; ++w) {
-        ts += sh_s[w];
-        tq += sh_q[w];
-      }
-      a.partials[ci].sum = ts;
-      a.partials[ci].sumsq = tq;
+      a.partials[ci].sum = ds;
+      a.partials[ci].sumsq = dq;
     }
-    __syncthreads();
   }
 }
 
@@ -68,6 +30,12 @@ __global__ void scalars_kernel(const __grid_constant__ KArgs a) {
   const int t = blockIdx.x;
   const int lane = threadIdx.x;
   const DevTensor& T = a.tensors[t];
+  // reset the fused kernel's counters for the launch that follows on this stream
+  if (a.tensor_done != nullptr && lane == 0) {
+    a.tensor_done[t] = 0;
+    if (t == 0)
+      for (int r = 0; r < kMaxRanges; ++r) a.work_counter[r] = 0;
+  }
   float sigma = (T.flags & TF_SIGMA_REL) ? 0.0f : T.sigma;
   if ((T.flags & TF_SIGMA_REL) && a.with_sigma) {
     double s = 0.0, q = 0.0;
@@ -78,15 +46,7 @@ __global__ void scalars_kernel(const __grid_constant__ KArgs a) {
     }
     s = warp_sum(s);
     q = warp_sum(q);
-    if (T.numel > 0) {
-      const double n = (double)T.numel;
-      const double mean = s / n;
-      double var = q / n - mean * mean;
-      if (var < 0.0) var = 0.0;
-      sigma = (float)((double)T.sigma_rel * sqrt(var));
-    } else {
-      sigma = 0.0f;
-    }
+    sigma = sigma_from_sums(s, q, T.numel, T.sigma_rel);
   }
   if (lane == 0) {
     DevScalars S;

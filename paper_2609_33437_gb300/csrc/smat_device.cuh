@@ -412,6 +412,68 @@ struct TView {
   bool has_noise;
 };
 
+__device__ __forceinline__ double warp_sum(double x) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
+  return x;
+}
+
+// Row a2 for one chunk: sums of delta = theta - theta0 (each one fp32
+// subtraction) and delta^2 over the chunk, fp32 per thread, then double in a
+// fixed order; the result is valid on thread 0. All threads must call it.
+template <int DT>
+__device__ __forceinline__ void chunk_delta_sums(const DevTensor& T, const Chunk& ch, double* sh_s,
+                                                 double* sh_q, double& sum, double& sumsq) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const bool vec = (T.flags & TF_VEC) != 0u;
+  float s = 0.0f, q = 0.0f;
+  for (int64_t i = ch.begin + 16 * (int64_t)threadIdx.x; i < ch.end; i += 16 * (int64_t)kBlock) {
+    if (vec && i + 16 <= ch.end) {
+      Raw16<DT> th, t0;
+      load16<DT>(T.theta, i, th);
+      load16<DT>(T.theta0, i, t0);
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const float d = __fsub_rn(th.at(k), t0.at(k));
+        s = __fadd_rn(s, d);
+        q = __fmaf_rn(d, d, q);
+      }
+    } else {
+      const int64_t e_end = (i + 16 < ch.end) ? i + 16 : ch.end;
+      for (int64_t e = i; e < e_end; ++e) {
+        const float d = __fsub_rn(load1<DT>(T.theta, e), load1<DT>(T.theta0, e));
+        s = __fadd_rn(s, d);
+        q = __fmaf_rn(d, d, q);
+      }
+    }
+  }
+  const double ds = warp_sum((double)s), dq = warp_sum((double)q);
+  if (lane == 0) {
+    sh_s[warp] = ds;
+    sh_q[warp] = dq;
+  }
+  __syncthreads();
+  sum = 0.0;
+  sumsq = 0.0;
+  if (threadIdx.x == 0) {
+    for (int w = 0; w < kBlock / 32; ++w) {
+      sum += sh_s[w];
+      sumsq += sh_q[w];
+    }
+  }
+  __syncthreads();
+}
+
+// sigma_t from the summed chunk sums of a tensor (population std of delta).
+__device__ __forceinline__ float sigma_from_sums(double s, double q, int64_t n, float sigma_rel) {
+  if (n <= 0) return 0.0f;
+  const double dn = (double)n;
+  const double mean = s / dn;
+  double var = q / dn - mean * mean;
+  if (var < 0.0) var = 0.0;
+  return (float)((double)sigma_rel * sqrt(var));
+}
+
 __device__ __forceinline__ TView make_view(const DevTensor& T, const DevScalars& S) {
   TView v;
   v.off = T.elem_offset;

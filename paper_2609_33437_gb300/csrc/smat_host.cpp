@@ -1,6 +1,7 @@
 // Host side of libsmat: argument validation, device tables, launches.
 // The C ABI is declared in include/smat.h.
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -40,8 +41,12 @@ size_t elem_size(int32_t dt) { return dt == SMAT_BF16 ? 2 : 4; }
 constexpr int64_t kMaxNumel = int64_t(1) << 40;
 
 struct Layout {
-  size_t tensors, chunks, scal, partials, grads, total;
+  size_t tensors, chunks, scal, partials, grads, items, sync, total;
 };
+
+// sync region: work counters (kMaxRanges), error flag, pad, then per tensor
+// tensor_done and ready.
+size_t sync_words(int32_t n) { return 4 + 2 * (size_t)n; }
 
 int64_t chunks_of(int64_t numel) { return (numel + kChunkElems - 1) / kChunkElems; }
 
@@ -53,6 +58,8 @@ Layout layout_for(int32_t n, int64_t n_chunks, bool any_sigma_rel) {
   L.scal = off;    off = align_up(off + sizeof(DevScalars) * (size_t)n);
   L.partials = off; off = align_up(off + (any_sigma_rel ? sizeof(StatPartial) * (size_t)n_chunks : 0));
   L.grads = off;   off = align_up(off + sizeof(GradPtr) * (size_t)n);
+  L.items = off;   off = align_up(off + (any_sigma_rel ? sizeof(int32_t) * 2 * (size_t)n_chunks : 0));
+  L.sync = off;    off = align_up(off + sizeof(int32_t) * sync_words(n));
   L.total = off;
   return L;
 }
@@ -67,6 +74,8 @@ smat_status check_config(const smat_config* cfg) {
     return fail(SMAT_ERR_UNSUPPORTED, "noise %d not supported", cfg->noise);
   if (cfg->philox_rounds != 0 && cfg->philox_rounds != 7 && cfg->philox_rounds != 10)
     return fail(SMAT_ERR_UNSUPPORTED, "philox_rounds %d not supported (7 or 10)", cfg->philox_rounds);
+  if (cfg->flags & ~SMAT_FLAG_UNFUSED_STATS)
+    return fail(SMAT_ERR_UNSUPPORTED, "unknown flags 0x%x", cfg->flags);
   if (!finite(cfg->alpha_min) || !finite(cfg->alpha_max) || cfg->alpha_min > cfg->alpha_max)
     return fail(SMAT_ERR_INVALID_ARG, "alpha range [%g, %g) invalid", cfg->alpha_min, cfg->alpha_max);
   return SMAT_OK;
@@ -155,6 +164,14 @@ struct smat_ctx {
   bool scalars_sigma = false; // the table's sigma_t are current
   std::vector<GradPtr> h_grads;
   bool grads_uploaded = false;
+  // fused statistics + forward
+  bool fused = false;
+  std::vector<int32_t> h_items;
+  int32_t item_begin[kMaxRanges] = {0, 0};
+  int32_t item_count[kMaxRanges] = {0, 0};
+  int32_t* d_items = nullptr;
+  int32_t* d_sync = nullptr;  // see sync_words()
+  uint32_t epoch = 0;
   // optional per-kernel timing
   bool timing = false;
   struct Mark { int kind; cudaEvent_t start, stop; };
@@ -213,7 +230,37 @@ KArgs base_args(const smat_ctx* c, uint32_t step) {
   a.alpha_min = c->cfg.alpha_min;
   a.alpha_width = c->cfg.alpha_max - c->cfg.alpha_min;
   a.alpha_mode = c->cfg.alpha_mode;
+  if (c->d_sync) {
+    a.work_counter = c->d_sync;
+    a.error = c->d_sync + 2;
+    a.tensor_done = c->d_sync + 4;
+    a.ready = reinterpret_cast<uint32_t*>(c->d_sync + 4 + c->desc.size());
+  }
   return a;
+}
+
+// Work list of the fused launch for one dtype range: statistics items (chunk
+// c at key 2c) and forward items; a forward item of a sigma_rel tensor gets
+// key 2 (last + lead + its position in the tensor) + 1, so all statistics
+// items of its tensor come first and the forward trails by `lead` chunks.
+void build_items(smat_ctx* c, int dt, int64_t lead) {
+  std::vector<std::pair<int64_t, int32_t>> keyed;
+  for (int64_t ci = c->range_begin[dt]; ci < c->range_end[dt]; ++ci) {
+    const Chunk& ch = c->h_chunks[(size_t)ci];
+    const DevTensor& T = c->h_tensors[ch.tensor];
+    const int64_t first = T.chunk_first, last = T.chunk_first + T.n_chunks - 1;
+    if (T.flags & TF_SIGMA_REL) {
+      keyed.push_back({2 * ci, (int32_t)ci});
+      keyed.push_back({2 * (last + lead + (ci - first)) + 1, (int32_t)(ci | (int64_t)kItemForward)});
+    } else {
+      keyed.push_back({2 * ci + 1, (int32_t)(ci | (int64_t)kItemForward)});
+    }
+  }
+  std::stable_sort(keyed.begin(), keyed.end(),
+                   [](const std::pair<int64_t, int32_t>& x, const std::pair<int64_t, int32_t>& y) { return x.first < y.first; });
+  c->item_begin[dt] = (int32_t)c->h_items.size();
+  for (auto& kv : keyed) c->h_items.push_back(kv.second);
+  c->item_count[dt] = (int32_t)keyed.size();
 }
 
 int grid_for(const smat_ctx* c, int64_t chunks, int dtype) {
@@ -292,6 +339,9 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
   c->d_scal = reinterpret_cast<DevScalars*>(ws + L.scal);
   c->d_partials = rel ? reinterpret_cast<StatPartial*>(ws + L.partials) : nullptr;
   c->d_grads = reinterpret_cast<GradPtr*>(ws + L.grads);
+  c->d_items = rel ? reinterpret_cast<int32_t*>(ws + L.items) : nullptr;
+  c->d_sync = reinterpret_cast<int32_t*>(ws + L.sync);
+  c->fused = rel && !(cfg->flags & SMAT_FLAG_UNFUSED_STATS);
 
   c->h_tensors.resize(n_tensors);
   c->h_chunks.reserve((size_t)nc);
@@ -351,6 +401,17 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
   if (e == cudaSuccess && nc > 0)
     e = cudaMemcpyAsync(c->d_chunks, c->h_chunks.data(), sizeof(Chunk) * (size_t)nc,
                         cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(c->d_sync, 0, sizeof(int32_t) * sync_words(n_tensors), stream);
+  if (e == cudaSuccess && c->fused) {
+    // lead of about two grid widths of the bf16 forward
+    const int64_t lead = 2 * (int64_t)c->sm_count *
+                         streaming_ctas_per_sm(SMAT_BF16, cfg->noise, cfg->alpha_mode == SMAT_ALPHA_PER_ELEMENT,
+                                               c->rounds);
+    for (int dt = 0; dt < 2; ++dt) build_items(c, dt, lead);
+    if (!c->h_items.empty())
+      e = cudaMemcpyAsync(c->d_items, c->h_items.data(), sizeof(int32_t) * c->h_items.size(),
+                          cudaMemcpyHostToDevice, stream);
+  }
   // The host vectors are pageable: the copies above have been staged when
   // they return, but keep the data in the context anyway for its lifetime.
   if (e != cudaSuccess) {
@@ -365,6 +426,30 @@ smat_status smat_simulate_multi(smat_ctx* c, uint32_t step, smat_stream_t stream
   if (!c) return fail(SMAT_ERR_INVALID_ARG, "ctx is NULL");
   if (c->active != 0)
     return fail(SMAT_ERR_STATE, "simulate called while the simulated storage is active; swap back first");
+  if (c->fused) {
+    // a1 (alpha, c; sigma of fixed-sigma tensors; counter reset), then a2 + a3 in one launch
+    smat_status st = run_scalars(c, step, false, stream);
+    if (st != SMAT_OK) return st;
+    c->scalars_sigma = true;
+    c->epoch += 1;
+    if (c->epoch == 0) c->epoch = 1;
+    KArgs a = base_args(c, step);
+    a.epoch = c->epoch;
+    for (int dt = 0; dt < 2; ++dt) {
+      if (c->item_count[dt] == 0) continue;
+      a.items = c->d_items + c->item_begin[dt];
+      a.n_items = c->item_count[dt];
+      a.work_counter = c->d_sync + dt;
+      const int grid = grid_for(c, c->range_end[dt] - c->range_begin[dt], dt);
+      Timed t(c, 2, stream);
+      const cudaError_t e = dt == SMAT_BF16
+          ? launch_stats_simulate_bf16(a, grid, c->cfg.noise, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT, c->rounds, stream)
+          : launch_stats_simulate_f32(a, grid, c->cfg.noise, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT, c->rounds, stream);
+      t.done();
+      if (e != cudaSuccess) return cuda_fail(e, "fused statistics + forward launch");
+    }
+    return SMAT_OK;
+  }
   smat_status st = run_scalars(c, step, true, stream);
   if (st != SMAT_OK) return st;
   KArgs a = base_args(c, step);
@@ -475,6 +560,50 @@ smat_status smat_tensor_scalars(smat_ctx* c, uint32_t step, float* d_out, smat_s
   if (st != SMAT_OK) return st;
   const cudaError_t e = cudaMemcpyAsync(d_out, c->d_scal, sizeof(DevScalars) * n, cudaMemcpyDeviceToDevice, stream);
   if (e != cudaSuccess) return cuda_fail(e, "scalars copy");
+  return SMAT_OK;
+}
+
+smat_status smat_debug_fused(smat_ctx* c, uint32_t step, const int32_t* d_items, int32_t n_items,
+                             uint32_t epoch_skew, smat_stream_t stream) {
+  if (!c) return fail(SMAT_ERR_INVALID_ARG, "ctx is NULL");
+  if (!c->any_sigma_rel) return fail(SMAT_ERR_STATE, "context has no sigma_rel tensor");
+  if (n_items < 0 || (n_items > 0 && !d_items)) return fail(SMAT_ERR_INVALID_ARG, "bad item list");
+  if (c->range_end[SMAT_BF16] <= c->range_begin[SMAT_BF16]) return fail(SMAT_ERR_STATE, "no bf16 tensors");
+  // items must name chunks of the bf16 range; checked on the host copy the caller passes through
+  std::vector<int32_t> h((size_t)n_items);
+  cudaError_t e = n_items ? cudaMemcpyAsync(h.data(), d_items, sizeof(int32_t) * (size_t)n_items,
+                                            cudaMemcpyDeviceToHost, stream) : cudaSuccess;
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_fail(e, "item list read");
+  for (int32_t v : h) {
+    const int64_t ci = (int64_t)((uint32_t)v & ~kItemForward);
+    if (ci < c->range_begin[SMAT_BF16] || ci >= c->range_end[SMAT_BF16])
+      return fail(SMAT_ERR_INVALID_ARG, "item names chunk %lld outside the bf16 range", (long long)ci);
+  }
+  smat_status st = run_scalars(c, step, false, stream);
+  if (st != SMAT_OK) return st;
+  c->epoch += 1;
+  if (c->epoch == 0) c->epoch = 1;
+  KArgs a = base_args(c, step);
+  a.epoch = c->epoch + epoch_skew;
+  a.items = d_items;
+  a.n_items = n_items;
+  a.work_counter = c->d_sync + SMAT_BF16;
+  e = launch_stats_simulate_bf16(a, grid_for(c, c->range_end[SMAT_BF16] - c->range_begin[SMAT_BF16], SMAT_BF16),
+                                 c->cfg.noise, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT, c->rounds, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "fused launch");
+  c->scalars_step = -1;  // sigma_t of this call may be incomplete
+  return SMAT_OK;
+}
+
+smat_status smat_poll_errors(smat_ctx* c, smat_stream_t stream, int32_t* errors_out) {
+  if (!c || !errors_out) return fail(SMAT_ERR_INVALID_ARG, "NULL argument");
+  int32_t v = 0;
+  cudaError_t e = cudaMemcpyAsync(&v, c->d_sync + 2, sizeof(int32_t), cudaMemcpyDeviceToHost, stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e == cudaSuccess && v != 0) e = cudaMemsetAsync(c->d_sync + 2, 0, sizeof(int32_t), stream);
+  if (e != cudaSuccess) return cuda_fail(e, "error flag read");
+  *errors_out = v;
   return SMAT_OK;
 }
 

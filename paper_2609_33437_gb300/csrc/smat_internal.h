@@ -91,7 +91,18 @@ struct KArgs {
   int32_t alpha_mode;
   int32_t tensor_index;  // mask_bits: the tensor
   int32_t with_sigma;    // scalars: 1 = derive sigma_t from the delta-statistics partials
+  // fused statistics + forward (stats_simulate_kernel)
+  const int32_t* items;  // work items: chunk index, high bit set for a forward item
+  int32_t n_items;
+  int32_t* work_counter; // next item to take (zeroed by the scalars kernel)
+  int32_t* tensor_done;  // statistics chunks finished per tensor (zeroed by the scalars kernel)
+  uint32_t* ready;       // per tensor: epoch of the call whose sigma_t is published
+  int32_t* error;        // device error flags (bit 0: a wait ran out)
+  uint32_t epoch;        // this call's epoch (>= 1)
 };
+
+constexpr uint32_t kItemForward = 0x80000000u;
+constexpr int kMaxRanges = 2;  // one item list per parameter dtype
 
 // Kernel launchers (smat_aux.cu, smat_gradmap.cu, smat_sim_*.cu). Each
 // returns the launch's error code.
@@ -107,6 +118,10 @@ cudaError_t launch_simulate_bf16(const KArgs& a, int grid, int noise, bool per_e
                                  cudaStream_t s);
 int simulate_ctas_per_sm_f32(int noise, bool per_elem_alpha, int rounds);
 int simulate_ctas_per_sm_bf16(int noise, bool per_elem_alpha, int rounds);
+cudaError_t launch_stats_simulate_f32(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
+                                      cudaStream_t s);
+cudaError_t launch_stats_simulate_bf16(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
+                                       cudaStream_t s);
 cudaError_t launch_mask_bits(const KArgs& a, int64_t numel, int rounds, cudaStream_t s);
 cudaError_t launch_debug_philox(const uint32_t* ctr, int64_t n, const RoundKeys& key, int rounds,
                                 uint32_t* out, uint32_t* out_ref, cudaStream_t s);

@@ -10,6 +10,13 @@ cudaError_t launch_simulate_f32(const KArgs& a, int grid, int noise, bool per_el
                      : sim_run<10, DT_F32>(a, grid, noise, per_elem_alpha, s);
 }
 
+cudaError_t launch_stats_simulate_f32(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
+                                      cudaStream_t s) {
+  if (a.n_items <= 0) return cudaSuccess;
+  return rounds == 7 ? fused_run<7, DT_F32>(a, grid, noise, per_elem_alpha, s)
+                     : fused_run<10, DT_F32>(a, grid, noise, per_elem_alpha, s);
+}
+
 int simulate_ctas_per_sm_f32(int noise, bool per_elem_alpha, int rounds) {
   return rounds == 7 ? sim_occ<7, DT_F32>(noise, per_elem_alpha) : sim_occ<10, DT_F32>(noise, per_elem_alpha);
 }

@@ -124,23 +124,158 @@ __device__ __forceinline__ void sim_chunk_noise(const KArgs& a, const TView& v, 
     sim_chunk<R, DT, NOISE_NONE, PE, IDENT, J0>(a, v, T, ch);
 }
 
+// ------------------------------------------- a2 + a3 fused (sigma_rel lists) ---
+// A persistent kernel that takes work items in list order from a counter:
+// statistics items (a2, one chunk each) and forward items (a3). Every
+// statistics item of a tensor precedes its forward items in the list (with a
+// lead of about two grid widths), so the bandwidth-bound statistics of later
+// tensors run beside the compute-bound forward of earlier ones. The CTA that
+// finishes a tensor's last statistics chunk sums the chunk partials in chunk
+// order, publishes sigma_t and releases the tensor's ready flag; forward items
+// of that tensor wait for the flag.
+//
+// Progress: items are taken in list order and a statistics item never waits,
+// so every item a waiting forward item depends on is already held by a
+// running CTA. The wait is bounded all the same: after kWaitLimit polls
+// (about one second) it sets bit 0 of *a.error, skips the item and returns to
+// the queue.
+constexpr uint32_t kWaitLimit = 1u << 22;
+
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_release(uint32_t* p, uint32_t v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ bool wait_ready(const KArgs& a, int t) {
+  for (uint32_t n = 0;; ++n) {
+    if (ld_acquire(a.ready + t) == a.epoch) return true;
+    if (n >= kWaitLimit) {
+      atomicOr(a.error, 1);
+      return false;
+    }
+    __nanosleep(256);
+  }
+}
+
+template <int R, int DT, int NOISE, bool PE>
+__device__ __forceinline__ void forward_chunk(const KArgs& a, const TView& v, const DevTensor& T,
+                                              const Chunk& ch) {
+  const bool j0 = (uint64_t)(v.off + ch.end) <= (uint64_t(1) << 34);
+  if (!PE && v.c == 1.0f) {
+    if (j0) sim_chunk_noise<R, DT, NOISE, PE, true, true>(a, v, T, ch);
+    else sim_chunk_noise<R, DT, NOISE, PE, true, false>(a, v, T, ch);
+  } else {
+    if (j0) sim_chunk_noise<R, DT, NOISE, PE, false, true>(a, v, T, ch);
+    else sim_chunk_noise<R, DT, NOISE, PE, false, false>(a, v, T, ch);
+  }
+}
+
+template <int R, int DT, int NOISE, bool PE>
+__global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 3 : 2)
+    stats_simulate_kernel(const __grid_constant__ KArgs a) {
+  __shared__ double sh_s[kBlock / 32];
+  __shared__ double sh_q[kBlock / 32];
+  __shared__ int s_item;
+  __shared__ int s_flag;
+  for (;;) {
+    if (threadIdx.x == 0) s_item = atomicAdd(a.work_counter, 1);
+    __syncthreads();
+    const int it = s_item;
+    if (it >= a.n_items) break;  // same value in every thread
+    const uint32_t code = (uint32_t)a.items[it];
+    const int64_t ci = (int64_t)(code & ~kItemForward);
+    const Chunk ch = a.chunks[ci];
+    const DevTensor& T = a.tensors[ch.tensor];
+    if (!(code & kItemForward)) {
+      double ds, dq;
+      chunk_delta_sums<DT>(T, ch, sh_s, sh_q, ds, dq);
+      if (threadIdx.x == 0) {
+        a.partials[ci].sum = ds;
+        a.partials[ci].sumsq = dq;
+        __threadfence();
+        s_flag = (atomicAdd(a.tensor_done + ch.tensor, 1) == T.n_chunks - 1) ? 1 : 0;
+      }
+      __syncthreads();
+      if (s_flag) {
+        // last statistics chunk of this tensor: sum the partials in chunk order
+        __threadfence();
+        double s = 0.0, q = 0.0;
+        for (int k = threadIdx.x; k < T.n_chunks; k += kBlock) {
+          s += __ldcg(&a.partials[T.chunk_first + k].sum);
+          q += __ldcg(&a.partials[T.chunk_first + k].sumsq);
+        }
+        s = warp_sum(s);
+        q = warp_sum(q);
+        if ((threadIdx.x & 31) == 0) {
+          sh_s[threadIdx.x >> 5] = s;
+          sh_q[threadIdx.x >> 5] = q;
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+          double ts = 0.0, tq = 0.0;
+          for (int w = 0; w < kBlock / 32; ++w) {
+            ts += sh_s[w];
+            tq += sh_q[w];
+          }
+          const float sigma = sigma_from_sums(ts, tq, T.numel, T.sigma_rel);
+          a.scal[ch.tensor].sigma = sigma;
+          a.scal[ch.tensor].noise_scale =
+              (float)(sqrt(NOISE == NOISE_UNIFORM ? 3.0 : 2.0) * (double)sigma);
+          __threadfence();
+          st_release(a.ready + ch.tensor, a.epoch);
+        }
+      }
+    } else {
+      if (T.flags & TF_SIGMA_REL) {
+        if (threadIdx.x == 0) s_flag = wait_ready(a, ch.tensor) ? 1 : 0;
+        __syncthreads();
+      } else if (threadIdx.x == 0) {
+        s_flag = 1;
+      }
+      __syncthreads();
+      if (s_flag) {
+        DevScalars S;
+        S.alpha = __ldcg(&a.scal[ch.tensor].alpha);
+        S.c = __ldcg(&a.scal[ch.tensor].c);
+        S.sigma = __ldcg(&a.scal[ch.tensor].sigma);
+        S.noise_scale = __ldcg(&a.scal[ch.tensor].noise_scale);
+        forward_chunk<R, DT, NOISE, PE>(a, make_view(T, S), T, ch);
+      }
+    }
+    __syncthreads();  // s_item, s_flag and the shared sums are reused by the next item
+  }
+}
+
 template <int R, int DT, int NOISE, bool PE>
 __global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 3 : 2) simulate_kernel(const __grid_constant__ KArgs a) {
   for (int64_t ci = a.chunk_begin + blockIdx.x; ci < a.chunk_end; ci += gridDim.x) {
     const Chunk ch = a.chunks[ci];
     const DevTensor& T = a.tensors[ch.tensor];
     const TView v = make_view(T, a.scal[ch.tensor]);
-    const bool j0 = (uint64_t)(v.off + ch.end) <= (uint64_t(1) << 34);  // gidx >> 2 < 2^32
-    if (!PE && v.c == 1.0f) {
-      if (j0) sim_chunk_noise<R, DT, NOISE, PE, true, true>(a, v, T, ch);
-      else sim_chunk_noise<R, DT, NOISE, PE, true, false>(a, v, T, ch);
-    } else {
-      if (j0) sim_chunk_noise<R, DT, NOISE, PE, false, true>(a, v, T, ch);
-      else sim_chunk_noise<R, DT, NOISE, PE, false, false>(a, v, T, ch);
-    }
+    forward_chunk<R, DT, NOISE, PE>(a, v, T, ch);
   }
 }
 
+
+template <int R, int DT, int NOISE, bool PE>
+struct FusedVariant {
+  static cudaError_t run(const KArgs& a, int grid, cudaStream_t s) {
+    stats_simulate_kernel<R, DT, NOISE, PE><<<grid, kBlock, 0, s>>>(a);
+    return cudaGetLastError();
+  }
+};
+
+template <int R, int DT>
+cudaError_t fused_run(const KArgs& a, int grid, int noise, bool pe, cudaStream_t s) {
+  if (noise == NOISE_GAUSSIAN)
+    return pe ? FusedVariant<R, DT, NOISE_GAUSSIAN, true>::run(a, grid, s) : FusedVariant<R, DT, NOISE_GAUSSIAN, false>::run(a, grid, s);
+  return pe ? FusedVariant<R, DT, NOISE_UNIFORM, true>::run(a, grid, s) : FusedVariant<R, DT, NOISE_UNIFORM, false>::run(a, grid, s);
+}
 
 template <typename Kernel>
 int occupancy_of(Kernel k) {

@@ -24,7 +24,7 @@ SMAT_ALPHA_GLOBAL, SMAT_ALPHA_PER_TENSOR, SMAT_ALPHA_PER_ELEMENT = 0, 1, 2
 
 EXPORTED = ("smat_workspace_bytes", "smat_init", "smat_simulate_multi", "smat_grad_map_multi",
             "smat_swap", "smat_active", "smat_mask_bits", "smat_tensor_scalars", "smat_destroy",
-            "smat_debug_philox", "smat_debug_noise_unit", "smat_timing_enable", "smat_timing_read", "smat_status_string",
+            "smat_debug_philox", "smat_debug_noise_unit", "smat_debug_fused", "smat_poll_errors", "smat_timing_enable", "smat_timing_read", "smat_status_string",
             "smat_last_error", "smat_abi_version")
 
 
@@ -44,7 +44,11 @@ class TensorDesc(ctypes.Structure):
 
 class Config(ctypes.Structure):
     _fields_ = [("seed", ctypes.c_uint64), ("alpha_min", ctypes.c_float), ("alpha_max", ctypes.c_float),
-                ("alpha_mode", ctypes.c_int32), ("noise", ctypes.c_int32), ("philox_rounds", ctypes.c_int32)]
+                ("alpha_mode", ctypes.c_int32), ("noise", ctypes.c_int32), ("philox_rounds", ctypes.c_int32),
+                ("flags", ctypes.c_int32)]
+
+
+SMAT_FLAG_UNFUSED_STATS = 1
 
 
 _lib = None
@@ -77,6 +81,8 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
     L.smat_destroy.argtypes = [P]
     L.smat_debug_philox.argtypes = [P, I64, U64, I32, P, P, P]
     L.smat_debug_noise_unit.argtypes = [P, I64, I32, P, P]
+    L.smat_poll_errors.argtypes = [P, P, ctypes.POINTER(I32)]
+    L.smat_debug_fused.argtypes = [P, U32, P, I32, U32, P]
     L.smat_timing_enable.argtypes = [P, I32]
     L.smat_timing_read.argtypes = [P, P, P]
     L.smat_status_string.argtypes = [I32]
@@ -86,7 +92,7 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
     L.smat_abi_version.restype = I32
     for name in ("smat_init", "smat_simulate_multi", "smat_grad_map_multi", "smat_swap", "smat_active",
                  "smat_mask_bits", "smat_tensor_scalars", "smat_destroy", "smat_debug_philox", "smat_debug_noise_unit",
-                 "smat_timing_enable", "smat_timing_read"):
+                 "smat_poll_errors", "smat_debug_fused", "smat_timing_enable", "smat_timing_read"):
         getattr(L, name).restype = I32
     _lib = L
     return L
@@ -126,7 +132,7 @@ class SmatSession:
                  sigma_rels: Optional[Sequence[float]] = None, tensor_ids: Optional[Sequence[int]] = None,
                  elem_offsets: Optional[Sequence[int]] = None, seed: int = 0, alpha_min: float = 0.0,
                  alpha_max: float = 1.0, alpha_mode: int = SMAT_ALPHA_GLOBAL,
-                 noise: int = SMAT_NOISE_UNIFORM, philox_rounds: int = 10,
+                 noise: int = SMAT_NOISE_UNIFORM, philox_rounds: int = 10, flags: int = 0,
                  stream: Optional[torch.cuda.Stream] = None):
         self._L = load_library()
         n = len(thetas)
@@ -157,7 +163,7 @@ class SmatSession:
             self.numels.append(th.numel())
         self._descs = descs
         self.config = Config(int(seed) & (2**64 - 1), float(alpha_min), float(alpha_max), int(alpha_mode),
-                             int(noise), int(philox_rounds))
+                             int(noise), int(philox_rounds), int(flags))
         self.device = thetas[0].device if n else torch.device("cuda", torch.cuda.current_device())
         nbytes = self._L.smat_workspace_bytes(ctypes.byref(descs), n, ctypes.byref(self.config))
         if nbytes == 0 and n > 0:
@@ -226,6 +232,19 @@ class SmatSession:
         check("smat_tensor_scalars", self._L.smat_tensor_scalars(self._ctx, int(step), ctypes.c_void_p(out.data_ptr()),
                                                                  _stream_handle(stream)))
         return out[:self.n]
+
+    def poll_errors(self, stream: Optional[torch.cuda.Stream] = None) -> int:
+        """Read and clear the device error flags (0 = none); synchronises the stream."""
+        v = ctypes.c_int32()
+        check("smat_poll_errors", self._L.smat_poll_errors(self._ctx, _stream_handle(stream), ctypes.byref(v)))
+        return v.value
+
+    def debug_fused(self, step: int, items: torch.Tensor, epoch_skew: int,
+                    stream: Optional[torch.cuda.Stream] = None):
+        """Test hook smat_debug_fused (items: int32 CUDA tensor of work items)."""
+        items = items.contiguous()
+        check("smat_debug_fused", self._L.smat_debug_fused(self._ctx, int(step), ctypes.c_void_p(items.data_ptr()),
+                                                           items.numel(), int(epoch_skew), _stream_handle(stream)))
 
     def timing_enable(self, enable: bool = True):
         check("smat_timing_enable", self._L.smat_timing_enable(self._ctx, int(bool(enable))))

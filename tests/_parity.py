@@ -145,4 +145,5 @@ def run_and_check_full(w: W.Workload, steps=(0, 1, 2), rounds=10, accumulate=Fal
                 assert np.float32(scal[k, 0]) == np.float32(s["alpha"]), "alpha"
                 assert np.float32(scal[k, 1]) == np.float32(s["c"]), "c"
             assert abs(float(scal[k, 2]) - s["sigma"]) <= 1e-5 * abs(s["sigma"]) + 1e-30, "sigma"
+    assert sess.poll_errors() == 0
     sess.close()
