@@ -419,35 +419,61 @@ __device__ __forceinline__ double warp_sum(double x) {
 }
 
 // Row a2 for one chunk: sums of delta = theta - theta0 (each one fp32
-// subtraction) and delta^2 over the chunk, fp32 per thread, then double in a
-// fixed order; the result is valid on thread 0. All threads must call it.
+// subtraction) and delta^2 over the chunk. Each thread keeps two 16-element
+// groups of loads in flight and accumulates on fp32 pairs; the partial sums
+// are combined in double in a fixed order (result valid on thread 0). All
+// threads must call it.
+template <int DT>
+__device__ __forceinline__ void delta_group(const Raw16<DT>& th, const Raw16<DT>& t0, float2& s2, float2& q2) {
+#pragma unroll
+  for (int m = 0; m < 8; ++m) {
+    const float2 a = th.pair(m), b = t0.pair(m);
+    const float2 d = add2_rn(a, make_float2(-b.x, -b.y));
+    s2 = add2_rn(s2, d);
+    q2 = fma2_rn(d, d, q2);
+  }
+}
+
 template <int DT>
 __device__ __forceinline__ void chunk_delta_sums(const DevTensor& T, const Chunk& ch, double* sh_s,
                                                  double* sh_q, double& sum, double& sumsq) {
+  constexpr int64_t kStride = 16 * (int64_t)kBlock;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const bool vec = (T.flags & TF_VEC) != 0u;
+  float2 s2 = splat(0.0f), q2 = splat(0.0f);
   float s = 0.0f, q = 0.0f;
-  for (int64_t i = ch.begin + 16 * (int64_t)threadIdx.x; i < ch.end; i += 16 * (int64_t)kBlock) {
-    if (vec && i + 16 <= ch.end) {
-      Raw16<DT> th, t0;
-      load16<DT>(T.theta, i, th);
-      load16<DT>(T.theta0, i, t0);
-#pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        const float d = __fsub_rn(th.at(k), t0.at(k));
-        s = __fadd_rn(s, d);
-        q = __fmaf_rn(d, d, q);
-      }
+  for (int64_t i = ch.begin + 16 * (int64_t)threadIdx.x; i < ch.end; i += 2 * kStride) {
+    const int64_t i2 = i + kStride;
+    if (vec && i2 + 16 <= ch.end) {
+      Raw16<DT> th1, t01, th2, t02;
+      load16<DT>(T.theta, i, th1);
+      load16<DT>(T.theta0, i, t01);
+      load16<DT>(T.theta, i2, th2);
+      load16<DT>(T.theta0, i2, t02);
+      delta_group<DT>(th1, t01, s2, q2);
+      delta_group<DT>(th2, t02, s2, q2);
     } else {
-      const int64_t e_end = (i + 16 < ch.end) ? i + 16 : ch.end;
-      for (int64_t e = i; e < e_end; ++e) {
-        const float d = __fsub_rn(load1<DT>(T.theta, e), load1<DT>(T.theta0, e));
-        s = __fadd_rn(s, d);
-        q = __fmaf_rn(d, d, q);
+      for (int half = 0; half < 2; ++half) {
+        const int64_t b = half ? i2 : i;
+        if (b >= ch.end) break;
+        if (vec && b + 16 <= ch.end) {
+          Raw16<DT> th1, t01;
+          load16<DT>(T.theta, b, th1);
+          load16<DT>(T.theta0, b, t01);
+          delta_group<DT>(th1, t01, s2, q2);
+        } else {
+          const int64_t e_end = (b + 16 < ch.end) ? b + 16 : ch.end;
+          for (int64_t e = b; e < e_end; ++e) {
+            const float d = __fsub_rn(load1<DT>(T.theta, e), load1<DT>(T.theta0, e));
+            s = __fadd_rn(s, d);
+            q = __fmaf_rn(d, d, q);
+          }
+        }
       }
     }
   }
-  const double ds = warp_sum((double)s), dq = warp_sum((double)q);
+  const double ds = warp_sum((double)s2.x + (double)s2.y + (double)s);
+  const double dq = warp_sum((double)q2.x + (double)q2.y + (double)q);
   if (lane == 0) {
     sh_s[warp] = ds;
     sh_q[warp] = dq;
