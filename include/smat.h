@@ -213,6 +213,28 @@ smat_status smat_timing_enable(smat_ctx* ctx, int32_t enable);
  * since timing was enabled. Either output may be NULL. */
 smat_status smat_timing_read(smat_ctx* ctx, double* ms_out, int64_t* launches_out);
 
+/* Allocation-free delta statistics of one tensor, for callers that cannot
+ * allocate device memory (for example a plugin inside a host framework that
+ * owns all of the GPU's memory, or code that must not grow a memory pool once
+ * a job runs). The paper has no counterpart; it is the sigma_rel computation
+ * of smat_simulate_multi, offered without a context or workspace.
+ *
+ * Writes *d_sigma (a device float) = sigma_rel * population std of
+ * theta - theta0 over numel elements of dtype (theta, theta0 device
+ * pointers). It calls no device allocation routine: its per-chunk partial
+ * sums go to one fixed 256 KiB array compiled into the library (every GPU that
+ * loads the library holds it until the process exits), so numel is limited
+ * to 16384 * 65536 = 2^30 elements (SMAT_ERR_INVALID_ARG beyond, with a
+ * message in smat_last_error()). The first call on each device looks up the
+ * array's device address and caches it; make that first call before any
+ * stream capture. Every call on a device shares the array: calls that overlap
+ * on the GPU (different streams, no ordering) race and give wrong results.
+ * Nothing in the array needs to start at zero: each call writes the partials
+ * it then reads. Asynchronous on `stream`. */
+smat_status smat_delta_sigma_noalloc(const void* d_theta, const void* d_theta0, int64_t numel,
+                                     int32_t dtype, float sigma_rel, float* d_sigma,
+                                     smat_stream_t stream);
+
 /* Static description of a status code. */
 const char* smat_status_string(smat_status s);
 

@@ -143,6 +143,11 @@ RoundKeys make_keys(uint64_t seed) {
 
 }  // namespace
 
+int smat::record_error_code(int status, const char* msg) {
+  g_last_error = msg;
+  return status;
+}
+
 struct smat_ctx {
   std::vector<smat_tensor_desc> desc;
   smat_config cfg;

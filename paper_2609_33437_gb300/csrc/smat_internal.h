@@ -132,4 +132,7 @@ int gradmap_ctas_per_sm(int gdtype, bool per_elem_alpha, bool accumulate, int ro
 
 constexpr int kBlock = 256;
 
+// Record `msg` as this thread's smat_last_error() text; returns `status`.
+int record_error_code(int status, const char* msg);
+
 }  // namespace smat

@@ -24,7 +24,8 @@ SMAT_ALPHA_GLOBAL, SMAT_ALPHA_PER_TENSOR, SMAT_ALPHA_PER_ELEMENT = 0, 1, 2
 
 EXPORTED = ("smat_workspace_bytes", "smat_init", "smat_simulate_multi", "smat_grad_map_multi",
             "smat_swap", "smat_active", "smat_mask_bits", "smat_tensor_scalars", "smat_destroy",
-            "smat_debug_philox", "smat_debug_noise_unit", "smat_debug_fused", "smat_poll_errors", "smat_timing_enable", "smat_timing_read", "smat_status_string",
+            "smat_debug_philox", "smat_debug_noise_unit", "smat_debug_fused", "smat_poll_errors",
+            "smat_delta_sigma_noalloc", "smat_timing_enable", "smat_timing_read", "smat_status_string",
             "smat_last_error", "smat_abi_version")
 
 
@@ -83,6 +84,8 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
     L.smat_debug_noise_unit.argtypes = [P, I64, I32, P, P]
     L.smat_poll_errors.argtypes = [P, P, ctypes.POINTER(I32)]
     L.smat_debug_fused.argtypes = [P, U32, P, I32, U32, P]
+    L.smat_delta_sigma_noalloc.argtypes = [P, P, I64, I32, ctypes.c_float, P, P]
+    L.smat_delta_sigma_noalloc.restype = I32
     L.smat_timing_enable.argtypes = [P, I32]
     L.smat_timing_read.argtypes = [P, P, P]
     L.smat_status_string.argtypes = [I32]
@@ -294,6 +297,23 @@ def debug_noise_unit(words: torch.Tensor, noise: int, stream: Optional[torch.cud
     out = torch.empty(words.shape, dtype=torch.float32, device=words.device)
     check("smat_debug_noise_unit", L.smat_debug_noise_unit(ctypes.c_void_p(words.data_ptr()), words.numel(), int(noise),
                                                            ctypes.c_void_p(out.data_ptr()), _stream_handle(stream)))
+    return out
+
+
+def delta_sigma_noalloc(theta: torch.Tensor, theta0: torch.Tensor, sigma_rel: float,
+                        out: Optional[torch.Tensor] = None, stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:
+    """smat_delta_sigma_noalloc: sigma_rel * std(theta - theta0) computed with
+    the library's fixed scratch array instead of any device allocation (the
+    result buffer `out`, one float on the device, is the caller's)."""
+    L = load_library()
+    if theta.dtype != theta0.dtype or theta.numel() != theta0.numel():
+        raise ValueError("theta and theta0 differ in dtype or numel")
+    if out is None:
+        out = torch.empty(1, dtype=torch.float32, device=theta.device)
+    check("smat_delta_sigma_noalloc",
+          L.smat_delta_sigma_noalloc(ctypes.c_void_p(theta.data_ptr()), ctypes.c_void_p(theta0.data_ptr()),
+                                     theta.numel(), dtype_code(theta.dtype), float(sigma_rel),
+                                     ctypes.c_void_p(out.data_ptr()), _stream_handle(stream)))
     return out
 
 
