@@ -195,12 +195,21 @@ def barrier(world):
 
 
 def max_over_ranks(x: float, world: int) -> float:
+    """Slowest rank's value (NCCL on the GPU, gloo on the host)."""
     if world == 1:
         return x
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def rank_workload(w: W.Workload, rank: int) -> W.Workload:
+    """Rank r trains its own expert: its own SMAT seed and its own data."""
+    w.seed = rank
+    w.data_seed = w.data_seed + 1000 * rank
+    return w
 
 
 # ------------------------------------------------------------ CPU oracle ---
@@ -339,9 +348,7 @@ def run_smat(args):
     from paper_2609_33437_gb300 import smat as S
     S.load_library()
     dev = torch.device("cuda", local)
-    w = workload(args)
-    w.seed = rank  # each rank: an independent expert
-    w.data_seed = w.data_seed + 1000 * rank
+    w = rank_workload(workload(args), rank)
 
     def make_session(th, t0, sim):
         return S.SmatSession(th, t0, sim, [t.keep_prob for t in w.tensors], [t.sigma for t in w.tensors],
@@ -438,7 +445,7 @@ def run_smat(args):
         if out is not None:
             out["e2e"] = e2e
     if out is not None and not args.no_cpu_baseline and world == 1:
-        secs, b, n, sample = oracle_run(w, 48_000_000)
+        secs, b, n, sample = oracle_run(w, 20_000_000)
         out["cpu_baseline"] = {"value": b / secs / 1e9, "unit": UNIT, "cores": 1, "kind": "oracle",
                                "sample": f"{sample} (single-threaded C++ oracle, forward + gradient map, "
                                          f"{secs:.1f} s)", "params_per_s": n / secs}
