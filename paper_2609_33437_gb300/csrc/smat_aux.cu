@@ -83,7 +83,8 @@ __global__ void __launch_bounds__(kBlock) mask_bits_kernel(const __grid_constant
       const uint64_t g0 = (uint64_t)(T.elem_offset + i0);
       uint32_t kw[4];
       for (int h = 0; h < 2; ++h) {
-        group_keep16<R, false>(a, T.tid, T.t_hi, T.t_lo, g0 + 16 * h, kw, nullptr);
+        if (group_keep16<R, false>(a, T.tid, T.t_hi, g0 + 16 * h, kw) && T.t_lo != 0u)
+          resolve_group_ties<R, false>(a, T.tid, T.t_hi, T.t_lo, g0 + 16 * h, kw);
         for (int e = 0; e < 16; ++e) bits |= (uint32_t)kept_of(kw, e) << (16 * h + e);
       }
     } else {

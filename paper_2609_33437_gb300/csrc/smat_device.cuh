@@ -229,14 +229,14 @@ __device__ __forceinline__ bool kept_of(const uint32_t (&kw)[4], int e) {
 // high byte of each element's 32-bit mask uniform comes from one MASK block
 // (byte b of word q serves element 4q + b); it is compared with the
 // threshold's high byte four bytes at a time (SWAR, no carries between
-// bytes). Bit 8b + 7 of kw[q] is element 4q + b's flag. Bytes equal to the
-// threshold byte (probability 1/256 each) need the low 24 bits of their
-// uniform from the MASK_LO stream: they are returned in *ties (bit e for
-// element e, flag left clear) when ties != nullptr, else drawn here.
+// bytes). Bit 8b + 7 of kw[q] is element 4q + b's flag. Returns whether some
+// byte equals the threshold's high byte (probability 1/256 per element): such
+// a tie is decided by the low 24 bits of the uniform (MASK_LO stream), which
+// the caller resolves (group_ties16 / resolve_group_ties); its flag is left
+// clear here.
 template <int R, bool J0>
-__device__ __forceinline__ void group_keep16(const KArgs& a, uint32_t tid, uint32_t t_hi,
-                                             uint32_t t_lo, uint64_t gidx0, uint32_t (&kw)[4],
-                                             uint32_t* ties) {
+__device__ __forceinline__ bool group_keep16(const KArgs& a, uint32_t tid, uint32_t t_hi, uint64_t gidx0,
+                                             uint32_t (&kw)[4]) {
   const uint4 w = stream_block<R, J0>(a, S_MASK, tid, gidx0 >> 4);
   const uint32_t words[4] = {w.x, w.y, w.z, w.w};
   const uint32_t tt = t_hi * 0x01010101u;
@@ -251,42 +251,59 @@ __device__ __forceinline__ void group_keep16(const KArgs& a, uint32_t tid, uint3
     const uint32_t e = x ^ tt;
     anytie |= (e - 0x01010101u) & ~e & 0x80808080u;  // nonzero iff some byte equals t
   }
-  if (t_lo != 0u && anytie != 0u) {
-    uint32_t tbits = 0u;
+  return anytie != 0u;
+}
+
+// Tie elements of the 16-element group at gidx0: bit e set iff element e's
+// mask byte equals the threshold's high byte.
+template <int R, bool J0>
+__device__ __forceinline__ uint32_t group_ties16(const KArgs& a, uint32_t tid, uint32_t t_hi, uint64_t gidx0) {
+  const uint4 w = stream_block<R, J0>(a, S_MASK, tid, gidx0 >> 4);
+  const uint32_t words[4] = {w.x, w.y, w.z, w.w};
+  const uint32_t tt = t_hi * 0x01010101u;
+  uint32_t tbits = 0u;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const uint32_t e = words[q] ^ tt;
-      const uint32_t eq = ~(((e & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | e) & 0x80808080u;  // exact per byte
-      tbits |= ((eq >> 7) & 1u) << (4 * q) | ((eq >> 15) & 1u) << (4 * q + 1) |
-               ((eq >> 23) & 1u) << (4 * q + 2) | ((eq >> 31) & 1u) << (4 * q + 3);
-    }
-    if (ties != nullptr) {
-      *ties = tbits;
-    } else {
-      while (tbits) {
-        const int e = __ffs(tbits) - 1;
-        tbits &= tbits - 1u;
-        const uint4 l = stream_block<R, J0>(a, S_MASK_LO, tid, (gidx0 >> 2) + (uint64_t)(e >> 2));
-        if ((pick(l, (unsigned)(e & 3)) >> 8) < t_lo) set_kept(kw, e);
-      }
-    }
-  } else if (ties != nullptr) {
-    *ties = 0u;
+  for (int q = 0; q < 4; ++q) {
+    const uint32_t e = words[q] ^ tt;
+    const uint32_t eq = ~(((e & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | e) & 0x80808080u;  // exact per byte
+    // bits 7, 15, 23, 31 -> bits 4q .. 4q + 3
+    tbits |= ((((eq >> 7) * 0x00204081u) >> 21) & 0xFu) << (4 * q);
+  }
+  return tbits;
+}
+
+// Low-24-bit test of one tie element.
+template <int R, bool J0>
+__device__ __forceinline__ bool tie_kept(const KArgs& a, uint32_t tid, uint32_t t_lo, uint64_t gidx) {
+  const uint4 l = stream_block<R, J0>(a, S_MASK_LO, tid, gidx >> 2);
+  return (pick(l, (unsigned)(gidx & 3)) >> 8) < t_lo;
+}
+
+// Decide the group's ties now (set their flags in kw).
+template <int R, bool J0>
+__device__ __forceinline__ void resolve_group_ties(const KArgs& a, uint32_t tid, uint32_t t_hi, uint32_t t_lo,
+                                                   uint64_t gidx0, uint32_t (&kw)[4]) {
+  uint32_t tb = group_ties16<R, J0>(a, tid, t_hi, gidx0);
+  while (tb) {
+    const int e = __ffs(tb) - 1;
+    tb &= tb - 1u;
+    if (tie_kept<R, J0>(a, tid, t_lo, gidx0 + (uint64_t)e)) set_kept(kw, e);
   }
 }
 
-// Tie elements whose low 24 mask bits are drawn at the end of the chunk, so
-// the rare Philox call runs once for the whole warp instead of once per
-// group. Up to four 16-bit in-chunk offsets per thread, two per register.
+// Groups with tie elements whose low 24 mask bits are drawn at the end of the
+// chunk, so the rare Philox calls run for the whole warp at once instead of
+// once per group. Up to four 16-bit group indices per thread (a chunk has
+// 4096 groups), two per register.
 struct TieList {
   uint32_t w0 = 0u, w1 = 0u;
   int n = 0;
-  __device__ __forceinline__ bool push(uint32_t off) {
+  __device__ __forceinline__ bool push(uint32_t g) {
     switch (n) {
-      case 0: w0 = off; break;
-      case 1: w0 |= off << 16; break;
-      case 2: w1 = off; break;
-      case 3: w1 |= off << 16; break;
+      case 0: w0 = g; break;
+      case 1: w0 |= g << 16; break;
+      case 2: w1 = g; break;
+      case 3: w1 |= g << 16; break;
       default: return false;
     }
     ++n;
@@ -297,14 +314,6 @@ struct TieList {
     return (k & 1) ? (w >> 16) : (w & 0xFFFFu);
   }
 };
-
-// Low-24-bit test of one tie element.
-template <int R, bool J0>
-__device__ __forceinline__ bool tie_kept(const KArgs& a, uint32_t tid, uint32_t t_lo, uint64_t gidx) {
-  const uint4 l = stream_block<R, J0>(a, S_MASK_LO, tid, gidx >> 2);
-  return (pick(l, (unsigned)(gidx & 3)) >> 8) < t_lo;
-}
-
 
 // Keep decision of one element (any alignment).
 template <int R>

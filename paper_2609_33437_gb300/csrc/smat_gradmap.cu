@@ -14,18 +14,9 @@ __device__ __forceinline__ void grad_compute16(const KArgs& a, const TView& v, u
                                                const Raw16<GDT>& go, float (&out)[16]) {
   uint32_t kw[4] = {0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u};
   if (v.flags & TF_MASK) {
-    if (ACC || !defer) {
-      group_keep16<R, J0>(a, v.tid, v.t_hi, v.t_lo, g0, kw, nullptr);
-    } else {
-      uint32_t ties = 0u;
-      group_keep16<R, J0>(a, v.tid, v.t_hi, v.t_lo, g0, kw, &ties);
-      while (ties) {
-        const int e = __ffs(ties) - 1;
-        ties &= ties - 1u;
-        if (!tl.push(off + (uint32_t)e) && tie_kept<R, J0>(a, v.tid, v.t_lo, g0 + (uint64_t)e))
-          set_kept(kw, e);
-      }
-    }
+    const bool tie = group_keep16<R, J0>(a, v.tid, v.t_hi, g0, kw);
+    if (v.t_lo != 0u && tie && (ACC || !defer || !tl.push(off >> 4)))
+      resolve_group_ties<R, J0>(a, v.tid, v.t_hi, v.t_lo, g0, kw);
   }
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
@@ -103,8 +94,14 @@ __device__ __forceinline__ void grad_chunk(const KArgs& a, const TView& v, const
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
     if (k < tl.n) {
-      const int64_t e = ch.begin + (int64_t)tl.at(k);
-      if (tie_kept<R, J0>(a, v.tid, v.t_lo, (uint64_t)(v.off + e))) grad_elem_as<R, GDT, PE, ACC>(a, v, G, e, true);
+      const int64_t gb = ch.begin + 16 * (int64_t)tl.at(k);
+      uint32_t tb = group_ties16<R, J0>(a, v.tid, v.t_hi, (uint64_t)(v.off + gb));
+      while (tb) {
+        const int e = __ffs(tb) - 1;
+        tb &= tb - 1u;
+        if (tie_kept<R, J0>(a, v.tid, v.t_lo, (uint64_t)(v.off + gb + e)))
+          grad_elem_as<R, GDT, PE, ACC>(a, v, G, gb + e, true);
+      }
     }
   }
 }

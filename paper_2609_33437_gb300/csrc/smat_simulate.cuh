@@ -21,14 +21,8 @@ __device__ __forceinline__ void sim_group16(const KArgs& a, const TView& v, cons
   load16<DT>(t0_p, i, t0);
   uint32_t kw[4] = {0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u};
   if (v.flags & TF_MASK) {
-    uint32_t ties = 0u;
-    group_keep16<R, J0>(a, v.tid, v.t_hi, v.t_lo, g0, kw, &ties);
-    while (ties) {
-      const int e = __ffs(ties) - 1;
-      ties &= ties - 1u;
-      if (!tl.push(off + (uint32_t)e) && tie_kept<R, J0>(a, v.tid, v.t_lo, g0 + (uint64_t)e))
-        set_kept(kw, e);
-    }
+    const bool tie = group_keep16<R, J0>(a, v.tid, v.t_hi, g0, kw);
+    if (v.t_lo != 0u && tie && !tl.push(off >> 4)) resolve_group_ties<R, J0>(a, v.tid, v.t_hi, v.t_lo, g0, kw);
   }
   float out[16];
   const float2 c2 = splat(v.c);
@@ -104,13 +98,18 @@ __device__ __forceinline__ void sim_chunk(const KArgs& a, const TView& v, const 
       }
     }
   }
-  // queued ties: rewrite the few that the low 24 bits keep
+  // queued tie groups: rewrite the few elements that the low 24 bits keep
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
     if (k < tl.n) {
-      const int64_t e = ch.begin + (int64_t)tl.at(k);
-      if (tie_kept<R, J0>(a, v.tid, v.t_lo, (uint64_t)(v.off + e)))
-        sim_elem_as<R, DT, NOISE, PE>(a, v, T.theta, T.theta0, T.sim, e, true);
+      const int64_t gb = ch.begin + 16 * (int64_t)tl.at(k);
+      uint32_t tb = group_ties16<R, J0>(a, v.tid, v.t_hi, (uint64_t)(v.off + gb));
+      while (tb) {
+        const int e = __ffs(tb) - 1;
+        tb &= tb - 1u;
+        if (tie_kept<R, J0>(a, v.tid, v.t_lo, (uint64_t)(v.off + gb + e)))
+          sim_elem_as<R, DT, NOISE, PE>(a, v, T.theta, T.theta0, T.sim, gb + e, true);
+      }
     }
   }
 }
