@@ -26,14 +26,18 @@
 //   streams: MASK = 0, NOISE = 1, ALPHA_E = 2, ALPHA_T = 3, MASK_LO = 4.
 //   gidx    = elem_offset + i  (global element index of local element i)
 //   u01(u)      = (u >> 8) * 2^-24          in [0, 1)
-//   sym(u)      = (2 (u >> 8) + 1 - 2^24) * 2^-24   odd multiples of 2^-24 in (-1, 1)
 //   Mask uniform U(gidx) in [0, 2^32):
 //     hi = byte (gidx & 3) of W(MASK, tid, gidx >> 4)[(gidx >> 2) & 3]
 //     lo = W(MASK_LO, tid, gidx >> 2)[gidx & 3] >> 8
 //     U  = hi * 2^24 + lo ;  kept  <=>  U < T,  T = floor(p_keep * 2^32)
-//   Noise word  n = W(NOISE, tid, gidx >> 2)[gidx & 3]
-//     uniform   eps = fl(sqrt3 sigma) * sym(n)
-//     Gaussian  eps = fl(sqrt2 sigma) * fl(erfinv(sym(n)))  (inverse-CDF transform:
+//   Noise field u (24 bits) of element gidx, k = gidx & 15, q = k >> 2, r = k & 3:
+//     S[0..11] = the 12 words of W(NOISE, tid, 3 (gidx >> 4) + b), b = 0, 1, 2
+//     (S[4b + w] = word w of block b); the quad q uses A = S[3q], B = S[3q+1],
+//     C = S[3q+2]: u = A >> 8, B >> 8, C >> 8 for r = 0, 1, 2, and for r = 3
+//     u = (A & 255) | (B & 255) << 8 | (C & 255) << 16.
+//     sym24(u) = (2u + 1 - 2^24) 2^-24
+//     uniform   eps = fl(sqrt3 sigma) * sym24(u)
+//     Gaussian  eps = fl(sqrt2 sigma) * fl(erfinv(sym24(u)))  (inverse-CDF transform:
 //               sqrt2 erfinv(v) is N(0, 1) for v uniform on (-1, 1))
 //   Alpha:  per tensor  alpha = fma(amax - amin, u01(W(ALPHA_T, t_a, 0)[0]), amin)
 //           t_a = 0x0FFFFFFF (one alpha for all tensors) or the tensor id;
@@ -130,10 +134,6 @@ uint32_t stream_word(const OrcConfig& cfg, uint32_t stream, uint32_t tid,
 const float kTwoPow24Inv = 5.9604644775390625e-08f;  // 2^-24, exact
 
 float u01(uint32_t u) { return (float)(u >> 8) * kTwoPow24Inv; }
-float sym(uint32_t u) {
-  const int32_t k = (int32_t)(u >> 8);
-  return (float)(2 * k + 1 - (1 << 24)) * kTwoPow24Inv;
-}
 
 // ------------------------------------------------------------- bf16 I/O ---
 float bf16_bits_to_f32(uint16_t h) {
@@ -274,18 +274,30 @@ double erfinv_d(double v) {
   return v < 0.0 ? -y : y;
 }
 
-double sym_d(uint32_t u) { return (double)(2 * (int64_t)(u >> 8) + 1 - (1 << 24)) * 0x1p-24; }
+// 24-bit noise field of element gidx (three noise words serve four elements).
+uint32_t noise_field(const OrcConfig& cfg, const OrcTensor& t, uint64_t gidx) {
+  const unsigned k = (unsigned)(gidx & 15), q = k >> 2, r = k & 3;
+  uint32_t quad[3];
+  for (unsigned m = 0; m < 3; ++m) {
+    const unsigned s_idx = 3 * q + m;  // index into the 12 words of the 3 blocks
+    quad[m] = stream_word(cfg, S_NOISE, t.tensor_id, 3 * (gidx >> 4) + s_idx / 4, s_idx % 4);
+  }
+  if (r < 3) return quad[r] >> 8;
+  return (quad[0] & 0xFFu) | ((quad[1] & 0xFFu) << 8) | ((quad[2] & 0xFFu) << 16);
+}
 
-// Unit-variance normal variate of element gidx: sqrt2 erfinv(sym(n)).
+float sym24(uint32_t u24) { return (float)(2 * (int32_t)u24 + 1 - (1 << 24)) * kTwoPow24Inv; }
+double sym24_d(uint32_t u24) { return (double)(2 * (int64_t)u24 + 1 - (1 << 24)) * 0x1p-24; }
+
+// Unit-variance normal variate of element gidx: sqrt2 erfinv(sym24(u)).
 double gauss_z(const OrcConfig& cfg, const OrcTensor& t, uint64_t gidx) {
-  const uint32_t n = stream_word(cfg, S_NOISE, t.tensor_id, gidx >> 2, (unsigned)(gidx & 3));
-  return std::sqrt(2.0) * erfinv_d(sym_d(n));
+  return std::sqrt(2.0) * erfinv_d(sym24_d(noise_field(cfg, t, gidx)));
 }
 
 float noise_eps(const OrcConfig& cfg, const OrcTensor& t, const Scalars& s, uint64_t gidx) {
-  const uint32_t n = stream_word(cfg, S_NOISE, t.tensor_id, gidx >> 2, (unsigned)(gidx & 3));
-  if (cfg.noise == NOISE_UNIFORM) return s.noise_scale * sym(n);
-  return s.noise_scale * (float)erfinv_d(sym_d(n));
+  const uint32_t u = noise_field(cfg, t, gidx);
+  if (cfg.noise == NOISE_UNIFORM) return s.noise_scale * sym24(u);
+  return s.noise_scale * (float)erfinv_d(sym24_d(u));
 }
 
 // Eq. smat-state for one element, fp32 arithmetic, before the storage rounding.
@@ -437,13 +449,11 @@ void orc_simulate_f64(const OrcConfig* cfg, const OrcTensor* t, float sigma_t, c
       x = t0[i] + c * (th[i] - t0[i]);
     }
     if (s.sigma > 0.0f) {
-      if (cfg->noise == NOISE_UNIFORM) {
-        const uint32_t nw = stream_word(*cfg, S_NOISE, t->tensor_id, gidx >> 2, (unsigned)(gidx & 3));
-        x += (double)s.noise_scale * (double)sym(nw);
-      } else {
-        const uint32_t nw = stream_word(*cfg, S_NOISE, t->tensor_id, gidx >> 2, (unsigned)(gidx & 3));
-        x += (double)s.noise_scale * erfinv_d(sym_d(nw));
-      }
+      const uint32_t u = noise_field(*cfg, *t, gidx);
+      if (cfg->noise == NOISE_UNIFORM)
+        x += (double)s.noise_scale * (double)sym24(u);
+      else
+        x += (double)s.noise_scale * erfinv_d(sym24_d(u));
     }
     out[i] = x;
   }

@@ -118,11 +118,11 @@ __global__ void debug_philox_kernel(const uint32_t* ctr, int64_t n, RoundKeys ke
   }
 }
 
-// Unit noise transforms of raw words (test hook): sym(n) or erfinv(sym(n)).
+// Unit noise transforms of raw words w (test hook): sym24(w >> 8) or erfinv of it.
 __global__ void debug_noise_unit_kernel(const uint32_t* words, int64_t n, int noise, float* out) {
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * blockDim.x) {
-    const float x = sym(words[i]);
+    const float x = sym24(words[i] >> 8);
     out[i] = (noise == NOISE_GAUSSIAN) ? erfinv_poly(x) : x;
   }
 }

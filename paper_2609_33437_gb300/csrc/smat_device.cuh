@@ -70,17 +70,16 @@ __device__ __forceinline__ uint32_t pick(const uint4& w, unsigned i) {
   return i == 0 ? w.x : (i == 1 ? w.y : (i == 2 ? w.z : w.w));
 }
 
-// u01(u) = (u >> 8) 2^-24 and sym(u) = (2 (u >> 8) + 1 - 2^24) 2^-24, both
-// exact in fp32.
+// u01(u) = (u >> 8) 2^-24 and sym24(u) = (2u + 1 - 2^24) 2^-24 (u a 24-bit
+// field), both exact in fp32.
 __device__ __forceinline__ float u01(uint32_t u) {
   return __fmul_rn(__uint2float_rn(u >> 8), 5.9604644775390625e-08f);
 }
-__device__ __forceinline__ float sym(uint32_t u) {
-  const int k = (int)(u >> 8);
-  return __fmul_rn(__int2float_rn(2 * k + 1 - (1 << 24)), 5.9604644775390625e-08f);
+__device__ __forceinline__ float sym24(uint32_t u) {
+  return __fmul_rn(__int2float_rn(2 * (int)u + 1 - (1 << 24)), 5.9604644775390625e-08f);
 }
 
-// erfinv(x) for |x| <= 1 - 2^-24 (every value sym() produces), after the
+// erfinv(x) for |x| <= 1 - 2^-24 (every value sym24() produces), after the
 // structure of M. Giles, "Approximating the erfinv function" (GPU Computing
 // Gems Jade Edition, 2011), with coefficients fitted for this form by
 // csrc/fit_erfinv.py: with L = log2(1 - x^2) (one fused multiply-add and the
@@ -158,10 +157,20 @@ __device__ __forceinline__ float2 fma2_rn(float2 a, float2 b, float2 c) {
   return d;
 }
 
+// sym24 of two 24-bit noise fields: (2u + 1 - 2^24) 2^-24, exact.
 __device__ __forceinline__ float2 sym2(uint32_t u0, uint32_t u1) {
-  const int k0 = (int)(u0 >> 8), k1 = (int)(u1 >> 8);
-  const float2 m = make_float2(__int2float_rn(2 * k0 + 1 - (1 << 24)), __int2float_rn(2 * k1 + 1 - (1 << 24)));
+  const float2 m = make_float2(__int2float_rn(2 * (int)u0 + 1 - (1 << 24)), __int2float_rn(2 * (int)u1 + 1 - (1 << 24)));
   return mul2_rn(m, splat(5.9604644775390625e-08f));
+}
+
+// The four 24-bit noise fields of a quad from its three noise words A, B, C:
+// the top 24 bits of each word, and the three low bytes combined.
+__device__ __forceinline__ void quad_fields(uint32_t A, uint32_t B, uint32_t C, uint32_t (&u)[4]) {
+  u[0] = A >> 8;
+  u[1] = B >> 8;
+  u[2] = C >> 8;
+  // bytes [x, A0, B0, C0] then drop x
+  u[3] = __byte_perm(__byte_perm(A, B, 0x0400u), C, 0x4210u) >> 8;
 }
 
 __device__ __forceinline__ float lg2_approx(float t) {
@@ -192,8 +201,9 @@ __device__ __forceinline__ float2 erfinv_poly2(float2 x) {
   return make_float2(erfinv_poly(x.x), erfinv_poly(x.y));
 }
 
-// Perturb of one element from its noise word: uniform scale * sym(n) with
-// scale = fl(sqrt3 sigma), or Gaussian scale * erfinv(sym(n)) with
+// Perturb of one element from its 24-bit noise field u: uniform
+// scale * sym24(u) with scale = fl(sqrt3 sigma), or Gaussian
+// scale * erfinv(sym24(u)) with
 // scale = fl(sqrt2 sigma) (inverse-CDF transform: sqrt2 erfinv(v) is
 // N(0, 1) for v uniform on (-1, 1)).
 template <int NOISE>
@@ -204,10 +214,33 @@ __device__ __forceinline__ float2 noise_of2(uint32_t n0, uint32_t n1, float2 sca
 }
 
 template <int NOISE>
-__device__ __forceinline__ float noise_of(uint32_t n, float scale) {
-  if (NOISE == NOISE_UNIFORM) return __fmul_rn(scale, sym(n));
-  if (NOISE == NOISE_GAUSSIAN) return __fmul_rn(scale, erfinv_poly(sym(n)));
+__device__ __forceinline__ float noise_of(uint32_t u24, float scale) {
+  if (NOISE == NOISE_UNIFORM) return __fmul_rn(scale, sym24(u24));
+  if (NOISE == NOISE_GAUSSIAN) return __fmul_rn(scale, erfinv_poly(sym24(u24)));
   return 0.0f;
+}
+
+// The 24-bit noise field of one element (any alignment): its quad's three
+// words come from one or two of the group's three noise blocks.
+template <int R>
+__device__ __forceinline__ uint32_t noise_field1(const KArgs& a, uint32_t tid, uint64_t gidx) {
+  const unsigned k = (unsigned)(gidx & 15), q = k >> 2, r = k & 3;
+  const uint64_t j0 = 3 * (gidx >> 4);
+  const unsigned s0 = 3 * q;  // first of the quad's words among the group's 12
+  const uint4 lo = stream_block<R>(a, S_NOISE, tid, j0 + s0 / 4);
+  const uint4 hi = (s0 / 4 == (s0 + 2) / 4) ? lo : stream_block<R>(a, S_NOISE, tid, j0 + (s0 + 2) / 4);
+  const uint32_t w8[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
+  // words s0, s0 + 1, s0 + 2 relative to block s0 / 4
+  const unsigned b = s0 % 4;
+  uint32_t ABC[3];
+#pragma unroll
+  for (int m = 0; m < 3; ++m) {
+    const unsigned idx = b + m;  // 0..5; indices >= 4 fall in `hi`
+    ABC[m] = idx == 0 ? w8[0] : idx == 1 ? w8[1] : idx == 2 ? w8[2] : idx == 3 ? w8[3] : idx == 4 ? w8[4] : w8[5];
+  }
+  uint32_t u[4];
+  quad_fields(ABC[0], ABC[1], ABC[2], u);
+  return r == 0 ? u[0] : r == 1 ? u[1] : r == 2 ? u[2] : u[3];
 }
 
 // Set element e's flag without indexing kw by a run-time value (which would

@@ -27,10 +27,21 @@ __device__ __forceinline__ void sim_group16(const KArgs& a, const TView& v, cons
   float out[16];
   const float2 c2 = splat(v.c);
   const float2 scale2 = splat(v.noise_scale);
+  // noise: three blocks per group, three words per quad (see quad_fields)
+  uint4 nb0 = make_uint4(0u, 0u, 0u, 0u), nb1 = nb0, nb2 = nb0;
+  const uint64_t jn = 3 * (g0 >> 4);
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
-    uint4 nw = make_uint4(0u, 0u, 0u, 0u);
-    if (NOISE != NOISE_NONE) nw = stream_block<R, J0>(a, S_NOISE, v.tid, (g0 >> 2) + q);
+    uint32_t u[4] = {0u, 0u, 0u, 0u};
+    if (NOISE != NOISE_NONE) {
+      if (q == 0) nb0 = stream_block<R, J0>(a, S_NOISE, v.tid, jn);
+      if (q == 1) nb1 = stream_block<R, J0>(a, S_NOISE, v.tid, jn + 1);
+      if (q == 2) nb2 = stream_block<R, J0>(a, S_NOISE, v.tid, jn + 2);
+      if (q == 0) quad_fields(nb0.x, nb0.y, nb0.z, u);
+      if (q == 1) quad_fields(nb0.w, nb1.x, nb1.y, u);
+      if (q == 2) quad_fields(nb1.z, nb1.w, nb2.x, u);
+      if (q == 3) quad_fields(nb2.y, nb2.z, nb2.w, u);
+    }
     uint4 aw = make_uint4(0u, 0u, 0u, 0u);
     if (PE) aw = stream_block<R, J0>(a, S_ALPHA_E, v.tid, (g0 >> 2) + q);
 #pragma unroll
@@ -51,7 +62,7 @@ __device__ __forceinline__ void sim_group16(const KArgs& a, const TView& v, cons
       float x0 = kept_of(kw, e0) ? kv.x : t02.x;
       float x1 = kept_of(kw, e0 + 1) ? kv.y : t02.y;
       if (NOISE != NOISE_NONE) {
-        const float2 eps = noise_of2<NOISE>(pick(nw, 2 * h), pick(nw, 2 * h + 1), scale2);
+        const float2 eps = noise_of2<NOISE>(u[2 * h], u[2 * h + 1], scale2);
         x0 = __fadd_rn(x0, eps.x);
         x1 = __fadd_rn(x1, eps.y);
       }
@@ -75,9 +86,7 @@ __device__ __forceinline__ void sim_elem_as(const KArgs& a, const TView& v, cons
   const float x_th = load1<DT>(th_p, e), x_t0 = load1<DT>(t0_p, e);
   float x = x_t0;
   if (kept) x = (c == 1.0f) ? x_th : __fmaf_rn(c, __fsub_rn(x_th, x_t0), x_t0);
-  if (NOISE != NOISE_NONE)
-    x = __fadd_rn(x, noise_of<NOISE>(pick(stream_block<R>(a, S_NOISE, v.tid, g >> 2), (unsigned)(g & 3)),
-                                     v.noise_scale));
+  if (NOISE != NOISE_NONE) x = __fadd_rn(x, noise_of<NOISE>(noise_field1<R>(a, v.tid, g), v.noise_scale));
   store1<DT>(sim_p, e, x);
 }
 
