@@ -201,6 +201,36 @@ __device__ __forceinline__ float2 erfinv_poly2(float2 x) {
   return make_float2(erfinv_poly(x.x), erfinv_poly(x.y));
 }
 
+// The group path's erfinv of a pair: the central polynomial only (packed,
+// branch free). minL collects the smallest L = log2(1 - x^2) seen, computed
+// exactly as erfinv_poly computes it; an element with L < -8 belongs to the
+// tail and its value here is wrong: the caller queues its group and rewrites
+// it through the element path (erfinv_poly).
+__device__ __forceinline__ float2 erfinv_central2(float2 x, float& minL) {
+  const float2 t = fma2_rn(make_float2(-x.x, -x.y), x, splat(1.0f));
+  const float2 L = make_float2(lg2_approx(t.x), lg2_approx(t.y));
+  minL = fminf(minL, fminf(L.x, L.y));
+  float2 p = splat(2.676246447e-10f);
+  p = fma2_rn(p, L, splat(9.962457526e-09f));
+  p = fma2_rn(p, L, splat(1.280022701e-07f));
+  p = fma2_rn(p, L, splat(2.725655577e-07f));
+  p = fma2_rn(p, L, splat(-7.822631233e-06f));
+  p = fma2_rn(p, L, splat(-3.107573502e-05f));
+  p = fma2_rn(p, L, splat(7.751958910e-04f));
+  p = fma2_rn(p, L, splat(5.547157954e-03f));
+  p = fma2_rn(p, L, splat(-1.608200818e-01f));
+  p = fma2_rn(p, L, splat(8.862268925e-01f));
+  return mul2_rn(x, p);
+}
+
+// Group-path noise of a pair (see erfinv_central2 for minL).
+template <int NOISE>
+__device__ __forceinline__ float2 noise_group2(uint32_t n0, uint32_t n1, float2 scale, float& minL) {
+  if (NOISE == NOISE_UNIFORM) return mul2_rn(scale, sym2(n0, n1));
+  if (NOISE == NOISE_GAUSSIAN) return mul2_rn(scale, erfinv_central2(sym2(n0, n1), minL));
+  return splat(0.0f);
+}
+
 // Perturb of one element from its 24-bit noise field u: uniform
 // scale * sym24(u) with scale = fl(sqrt3 sigma), or Gaussian
 // scale * erfinv(sym24(u)) with

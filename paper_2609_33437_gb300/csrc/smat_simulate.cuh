@@ -7,36 +7,40 @@ namespace smat {
 namespace {
 
 // --------------------------------------------------------------- a3: forward ---
+constexpr uint32_t kQueueTie = 1u;   // the group has a mask tie (low 24 bits decide)
+constexpr uint32_t kQueueTail = 2u;  // the group has a Gaussian tail element
+
 // One 16-element group on the vector path. IDENT: c == 1 for the whole tensor
 // (kept elements are theta itself); only used without per-element alpha.
-// Tie elements are written as dropped and queued in tl (resolved at the end
-// of the chunk); if the queue is full they are resolved here.
+// Tie elements are written as dropped and Gaussian noise takes the central
+// polynomial for every element; the returned flags (kQueueTie, kQueueTail)
+// say whether some element needs the element path afterwards.
 template <int R, int DT, int NOISE, bool PE, bool IDENT, bool J0>
-__device__ __forceinline__ void sim_group16(const KArgs& a, const TView& v, const void* th_p,
-                                            const void* t0_p, void* sim_p, int64_t i, uint32_t off,
-                                            TieList& tl) {
+__device__ __forceinline__ uint32_t sim_group16(const KArgs& a, const TView& v, const Raw16<DT>& th,
+                                                const Raw16<DT>& t0, void* sim_p, int64_t i) {
   const uint64_t g0 = (uint64_t)(v.off + i);
-  Raw16<DT> th, t0;
-  load16<DT>(th_p, i, th);
-  load16<DT>(t0_p, i, t0);
   uint32_t kw[4] = {0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u};
+  uint32_t flags = 0u;
   if (v.flags & TF_MASK) {
     const bool tie = group_keep16<R, J0>(a, v.tid, v.t_hi, g0, kw);
-    if (v.t_lo != 0u && tie && !tl.push(off >> 4)) resolve_group_ties<R, J0>(a, v.tid, v.t_hi, v.t_lo, g0, kw);
+    flags = (v.t_lo != 0u && tie) ? kQueueTie : 0u;
   }
   float out[16];
+  float minL = 0.0f;
   const float2 c2 = splat(v.c);
   const float2 scale2 = splat(v.noise_scale);
   // noise: three blocks per group, three words per quad (see quad_fields)
   uint4 nb0 = make_uint4(0u, 0u, 0u, 0u), nb1 = nb0, nb2 = nb0;
   const uint64_t jn = 3 * (g0 >> 4);
+  if (NOISE != NOISE_NONE) {
+    nb0 = stream_block<R, J0>(a, S_NOISE, v.tid, jn);
+    nb1 = stream_block<R, J0>(a, S_NOISE, v.tid, jn + 1);
+    nb2 = stream_block<R, J0>(a, S_NOISE, v.tid, jn + 2);
+  }
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     uint32_t u[4] = {0u, 0u, 0u, 0u};
     if (NOISE != NOISE_NONE) {
-      if (q == 0) nb0 = stream_block<R, J0>(a, S_NOISE, v.tid, jn);
-      if (q == 1) nb1 = stream_block<R, J0>(a, S_NOISE, v.tid, jn + 1);
-      if (q == 2) nb2 = stream_block<R, J0>(a, S_NOISE, v.tid, jn + 2);
       if (q == 0) quad_fields(nb0.x, nb0.y, nb0.z, u);
       if (q == 1) quad_fields(nb0.w, nb1.x, nb1.y, u);
       if (q == 2) quad_fields(nb1.z, nb1.w, nb2.x, u);
@@ -62,7 +66,7 @@ __device__ __forceinline__ void sim_group16(const KArgs& a, const TView& v, cons
       float x0 = kept_of(kw, e0) ? kv.x : t02.x;
       float x1 = kept_of(kw, e0 + 1) ? kv.y : t02.y;
       if (NOISE != NOISE_NONE) {
-        const float2 eps = noise_of2<NOISE>(u[2 * h], u[2 * h + 1], scale2);
+        const float2 eps = noise_group2<NOISE>(u[2 * h], u[2 * h + 1], scale2, minL);
         x0 = __fadd_rn(x0, eps.x);
         x1 = __fadd_rn(x1, eps.y);
       }
@@ -71,6 +75,33 @@ __device__ __forceinline__ void sim_group16(const KArgs& a, const TView& v, cons
     }
   }
   store16<DT>(sim_p, i, out);
+  if (NOISE == NOISE_GAUSSIAN && minL < -8.0f) flags |= kQueueTail;
+  return flags;
+}
+
+// Tail elements of the 16-element group at gidx0 (bit e set iff element e's
+// L = log2(1 - x^2) < -8), computed exactly as erfinv_central2 computes L.
+template <int R, bool J0>
+__device__ __forceinline__ uint32_t group_tails16(const KArgs& a, uint32_t tid, uint64_t gidx0) {
+  const uint64_t jn = 3 * (gidx0 >> 4);
+  const uint4 b0 = stream_block<R, J0>(a, S_NOISE, tid, jn);
+  const uint4 b1 = stream_block<R, J0>(a, S_NOISE, tid, jn + 1);
+  const uint4 b2 = stream_block<R, J0>(a, S_NOISE, tid, jn + 2);
+  uint32_t bits = 0u;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    uint32_t u[4];
+    if (q == 0) quad_fields(b0.x, b0.y, b0.z, u);
+    if (q == 1) quad_fields(b0.w, b1.x, b1.y, u);
+    if (q == 2) quad_fields(b1.z, b1.w, b2.x, u);
+    if (q == 3) quad_fields(b2.y, b2.z, b2.w, u);
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      const float x = sym24(u[r]);
+      if (lg2_approx(__fmaf_rn(-x, x, 1.0f)) < -8.0f) bits |= 1u << (4 * q + r);
+    }
+  }
+  return bits;
 }
 
 // One element given its keep decision (any alignment).
@@ -90,15 +121,58 @@ __device__ __forceinline__ void sim_elem_as(const KArgs& a, const TView& v, cons
   store1<DT>(sim_p, e, x);
 }
 
+// Rewrite the elements of a queued group that the group path got wrong: tie
+// elements the low 24 bits keep, and every Gaussian tail element.
+template <int R, int DT, int NOISE, bool PE, bool J0>
+__device__ __forceinline__ void sim_resolve(const KArgs& a, const TView& v, const DevTensor& T, int64_t gb,
+                                         uint32_t flags) {
+  const uint64_t g0 = (uint64_t)(v.off + gb);
+  const uint32_t tb = (flags & kQueueTie) ? group_ties16<R, J0>(a, v.tid, v.t_hi, g0) : 0u;
+  const uint32_t nb = (NOISE == NOISE_GAUSSIAN && (flags & kQueueTail)) ? group_tails16<R, J0>(a, v.tid, g0) : 0u;
+  const bool masked = (v.flags & TF_MASK) != 0u;
+  uint32_t todo = tb | nb;
+  while (todo) {
+    const int e = __ffs(todo) - 1;
+    todo &= todo - 1u;
+    bool kept;
+    if ((tb >> e) & 1u) kept = tie_kept<R, J0>(a, v.tid, v.t_lo, g0 + (uint64_t)e);
+    else kept = masked ? elem_kept<R>(a, v.tid, v.t_hi, v.t_lo, g0 + (uint64_t)e) : true;
+    if (kept || ((nb >> e) & 1u)) sim_elem_as<R, DT, NOISE, PE>(a, v, T.theta, T.theta0, T.sim, gb + e, kept);
+  }
+}
+
+// Groups of the current chunk that need the element path, collected by all
+// threads of the CTA and drained by all of them after the chunk, so the rare
+// element work is spread over the whole CTA instead of serialising each
+// lane's own list. Tie-only groups fill it from the front, groups with a
+// Gaussian tail element from the back (one slot per group of a chunk, so it
+// cannot overflow). The counters are reset by the caller before the barrier
+// that precedes the chunk.
+struct ChunkQueue {
+  static constexpr int kGroups = kChunkElems / 16;
+  uint16_t e[kGroups];
+  int n_tie;
+  int n_tail;
+};
+
 template <int R, int DT, int NOISE, bool PE, bool IDENT, bool J0>
 __device__ __forceinline__ void sim_chunk(const KArgs& a, const TView& v, const DevTensor& T,
-                                          const Chunk& ch) {
+                                          const Chunk& ch, ChunkQueue& cq) {
   const bool vec = (v.flags & TF_VEC) != 0u;
   const bool masked = (v.flags & TF_MASK) != 0u;
-  TieList tl;
   for (int64_t i = ch.begin + 16 * (int64_t)threadIdx.x; i < ch.end; i += 16 * (int64_t)kBlock) {
     if (vec && i + 16 <= ch.end) {
-      sim_group16<R, DT, NOISE, PE, IDENT, J0>(a, v, T.theta, T.theta0, T.sim, i, (uint32_t)(i - ch.begin), tl);
+      Raw16<DT> th, t0;
+      load16<DT>(T.theta, i, th);
+      load16<DT>(T.theta0, i, t0);
+      const uint32_t f = sim_group16<R, DT, NOISE, PE, IDENT, J0>(a, v, th, t0, T.sim, i);
+      if (f) {
+        const uint32_t entry = (((uint32_t)(i - ch.begin) >> 4) << 2) | f;
+        if (f & kQueueTail)
+          cq.e[ChunkQueue::kGroups - 1 - atomicAdd(&cq.n_tail, 1)] = (uint16_t)entry;
+        else
+          cq.e[atomicAdd(&cq.n_tie, 1)] = (uint16_t)entry;
+      }
     } else {
       const int64_t e_end = (i + 16 < ch.end) ? i + 16 : ch.end;
       for (int64_t e = i; e < e_end; ++e) {
@@ -107,29 +181,23 @@ __device__ __forceinline__ void sim_chunk(const KArgs& a, const TView& v, const 
       }
     }
   }
-  // queued tie groups: rewrite the few elements that the low 24 bits keep
-#pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    if (k < tl.n) {
-      const int64_t gb = ch.begin + 16 * (int64_t)tl.at(k);
-      uint32_t tb = group_ties16<R, J0>(a, v.tid, v.t_hi, (uint64_t)(v.off + gb));
-      while (tb) {
-        const int e = __ffs(tb) - 1;
-        tb &= tb - 1u;
-        if (tie_kept<R, J0>(a, v.tid, v.t_lo, (uint64_t)(v.off + gb + e)))
-          sim_elem_as<R, DT, NOISE, PE>(a, v, T.theta, T.theta0, T.sim, gb + e, true);
-      }
-    }
+  // the barrier also orders every thread's group stores before the rewrites
+  __syncthreads();
+  const int nt = cq.n_tie, nn = cq.n_tail;
+#pragma unroll 1
+  for (int k = threadIdx.x; k < nt + nn; k += kBlock) {
+    const uint32_t q = (k < nt) ? cq.e[k] : cq.e[ChunkQueue::kGroups - nn + (k - nt)];
+    sim_resolve<R, DT, NOISE, PE, J0>(a, v, T, ch.begin + 16 * (int64_t)(q >> 2), q & 3u);
   }
 }
 
 template <int R, int DT, int NOISE, bool PE, bool IDENT, bool J0>
 __device__ __forceinline__ void sim_chunk_noise(const KArgs& a, const TView& v, const DevTensor& T,
-                                                const Chunk& ch) {
+                                                const Chunk& ch, ChunkQueue& cq) {
   if (v.has_noise)
-    sim_chunk<R, DT, NOISE, PE, IDENT, J0>(a, v, T, ch);
+    sim_chunk<R, DT, NOISE, PE, IDENT, J0>(a, v, T, ch, cq);
   else
-    sim_chunk<R, DT, NOISE_NONE, PE, IDENT, J0>(a, v, T, ch);
+    sim_chunk<R, DT, NOISE_NONE, PE, IDENT, J0>(a, v, T, ch, cq);
 }
 
 // ------------------------------------------- a2 + a3 fused (sigma_rel lists) ---
@@ -170,16 +238,17 @@ __device__ __forceinline__ bool wait_ready(const KArgs& a, int t) {
   }
 }
 
+// All threads of the CTA call this for the same chunk (it has a barrier).
 template <int R, int DT, int NOISE, bool PE>
 __device__ __forceinline__ void forward_chunk(const KArgs& a, const TView& v, const DevTensor& T,
-                                              const Chunk& ch) {
+                                              const Chunk& ch, ChunkQueue& cq) {
   const bool j0 = (uint64_t)(v.off + ch.end) <= (uint64_t(1) << 34);
   if (!PE && v.c == 1.0f) {
-    if (j0) sim_chunk_noise<R, DT, NOISE, PE, true, true>(a, v, T, ch);
-    else sim_chunk_noise<R, DT, NOISE, PE, true, false>(a, v, T, ch);
+    if (j0) sim_chunk_noise<R, DT, NOISE, PE, true, true>(a, v, T, ch, cq);
+    else sim_chunk_noise<R, DT, NOISE, PE, true, false>(a, v, T, ch, cq);
   } else {
-    if (j0) sim_chunk_noise<R, DT, NOISE, PE, false, true>(a, v, T, ch);
-    else sim_chunk_noise<R, DT, NOISE, PE, false, false>(a, v, T, ch);
+    if (j0) sim_chunk_noise<R, DT, NOISE, PE, false, true>(a, v, T, ch, cq);
+    else sim_chunk_noise<R, DT, NOISE, PE, false, false>(a, v, T, ch, cq);
   }
 }
 
@@ -190,8 +259,13 @@ __global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 3 : 2)
   __shared__ double sh_q[kBlock / 32];
   __shared__ int s_item;
   __shared__ int s_flag;
+  __shared__ ChunkQueue s_cq;
   for (;;) {
-    if (threadIdx.x == 0) s_item = atomicAdd(a.work_counter, 1);
+    if (threadIdx.x == 0) {
+      s_item = atomicAdd(a.work_counter, 1);
+      s_cq.n_tie = 0;
+      s_cq.n_tail = 0;
+    }
     __syncthreads();
     const int it = s_item;
     if (it >= a.n_items) break;  // same value in every thread
@@ -252,7 +326,7 @@ __global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 3 : 2)
         S.c = __ldcg(&a.scal[ch.tensor].c);
         S.sigma = __ldcg(&a.scal[ch.tensor].sigma);
         S.noise_scale = __ldcg(&a.scal[ch.tensor].noise_scale);
-        forward_chunk<R, DT, NOISE, PE>(a, make_view(T, S), T, ch);
+        forward_chunk<R, DT, NOISE, PE>(a, make_view(T, S), T, ch, s_cq);
       }
     }
     __syncthreads();  // s_item, s_flag and the shared sums are reused by the next item
@@ -261,11 +335,18 @@ __global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 3 : 2)
 
 template <int R, int DT, int NOISE, bool PE>
 __global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 3 : 2) simulate_kernel(const __grid_constant__ KArgs a) {
+  __shared__ ChunkQueue s_cq;
   for (int64_t ci = a.chunk_begin + blockIdx.x; ci < a.chunk_end; ci += gridDim.x) {
+    if (threadIdx.x == 0) {
+      s_cq.n_tie = 0;
+      s_cq.n_tail = 0;
+    }
+    __syncthreads();
     const Chunk ch = a.chunks[ci];
     const DevTensor& T = a.tensors[ch.tensor];
     const TView v = make_view(T, a.scal[ch.tensor]);
-    forward_chunk<R, DT, NOISE, PE>(a, v, T, ch);
+    forward_chunk<R, DT, NOISE, PE>(a, v, T, ch, s_cq);
+    __syncthreads();  // every thread has read the counters before the next reset
   }
 }
 
