@@ -95,7 +95,7 @@ typedef struct {
 } smat_tensor_desc;
 
 /* smat_config.flags */
-#define SMAT_FLAG_UNFUSED_STATS 1 /* run delta statistics as a separate pass before the forward */
+#define SMAT_FLAG_UNFUSED_STATS 1 /* run delta statistics as a separate pass, then a grid-stride forward */
 
 typedef struct {
   uint64_t seed;         /* Philox key */
@@ -126,10 +126,12 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
  * per-call scalars (and, for sigma_rel tensors, the delta statistics) and
  * writes theta~ into each tensor's `sim`. Requires the original storage to be
  * active (SMAT_ERR_STATE otherwise): the simulated state is rebuilt only
- * while the model reads theta. With sigma_rel tensors the statistics and the
- * forward run in one persistent launch by default (statistics of later
- * tensors beside the forward of earlier ones); SMAT_FLAG_UNFUSED_STATS runs
- * them as two passes. Results are identical either way. */
+ * while the model reads theta. By default the forward is one persistent
+ * launch whose CTAs take chunks of 2^18 elements from a work list in order;
+ * with sigma_rel tensors the statistics run in the same launch (statistics
+ * of later tensors beside the forward of earlier ones).
+ * SMAT_FLAG_UNFUSED_STATS runs the statistics as a separate pass and the
+ * forward as a grid-stride launch. Results are identical either way. */
 smat_status smat_simulate_multi(smat_ctx* ctx, uint32_t step, smat_stream_t stream);
 
 /* Gradient map (Eq. smat-gradient) at step `step`: for tensor k,

@@ -58,7 +58,7 @@ Layout layout_for(int32_t n, int64_t n_chunks, bool any_sigma_rel) {
   L.scal = off;    off = align_up(off + sizeof(DevScalars) * (size_t)n);
   L.partials = off; off = align_up(off + (any_sigma_rel ? sizeof(StatPartial) * (size_t)n_chunks : 0));
   L.grads = off;   off = align_up(off + sizeof(GradPtr) * (size_t)n);
-  L.items = off;   off = align_up(off + (any_sigma_rel ? sizeof(int32_t) * 2 * (size_t)n_chunks : 0));
+  L.items = off;   off = align_up(off + sizeof(int32_t) * (any_sigma_rel ? 2 : 1) * (size_t)n_chunks);
   L.sync = off;    off = align_up(off + sizeof(int32_t) * sync_words(n));
   L.total = off;
   return L;
@@ -169,7 +169,7 @@ struct smat_ctx {
   bool scalars_sigma = false; // the table's sigma_t are current
   std::vector<GradPtr> h_grads;
   bool grads_uploaded = false;
-  // fused statistics + forward
+  // work-list forward launch (with the statistics of sigma_rel tensors)
   bool fused = false;
   std::vector<int32_t> h_items;
   int32_t item_begin[kMaxRanges] = {0, 0};
@@ -344,9 +344,9 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
   c->d_scal = reinterpret_cast<DevScalars*>(ws + L.scal);
   c->d_partials = rel ? reinterpret_cast<StatPartial*>(ws + L.partials) : nullptr;
   c->d_grads = reinterpret_cast<GradPtr*>(ws + L.grads);
-  c->d_items = rel ? reinterpret_cast<int32_t*>(ws + L.items) : nullptr;
+  c->d_items = reinterpret_cast<int32_t*>(ws + L.items);
   c->d_sync = reinterpret_cast<int32_t*>(ws + L.sync);
-  c->fused = rel && !(cfg->flags & SMAT_FLAG_UNFUSED_STATS);
+  c->fused = !(cfg->flags & SMAT_FLAG_UNFUSED_STATS);
 
   c->h_tensors.resize(n_tensors);
   c->h_chunks.reserve((size_t)nc);
@@ -432,7 +432,8 @@ smat_status smat_simulate_multi(smat_ctx* c, uint32_t step, smat_stream_t stream
   if (c->active != 0)
     return fail(SMAT_ERR_STATE, "simulate called while the simulated storage is active; swap back first");
   if (c->fused) {
-    // a1 (alpha, c; sigma of fixed-sigma tensors; counter reset), then a2 + a3 in one launch
+    // a1 (alpha, c; sigma of fixed-sigma tensors; counter reset), then a3 (with a2
+    // for sigma_rel tensors) in one work-list launch
     smat_status st = run_scalars(c, step, false, stream);
     if (st != SMAT_OK) return st;
     c->scalars_sigma = true;

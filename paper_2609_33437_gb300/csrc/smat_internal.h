@@ -13,9 +13,13 @@ namespace smat {
 enum : uint32_t { S_MASK = 0, S_NOISE = 1, S_ALPHA_E = 2, S_ALPHA_T = 3, S_MASK_LO = 4 };
 constexpr uint32_t kGlobalAlphaTensor = 0x0FFFFFFFu;
 
-// Elements per work chunk of the multi-tensor launch (a multiple of 16, so a
-// chunk never splits a 16-element mask draw group of an aligned tensor).
-constexpr int64_t kChunkElems = int64_t(1) << 16;
+// Elements per work chunk of the multi-tensor launches (a multiple of 16, so
+// a chunk never splits a 16-element mask draw group of an aligned tensor).
+// Statistics and forward work items are whole chunks; the gradient map,
+// whose CTAs take chunks in a fixed grid-stride order, walks halves of
+// chunks (kGradUnitElems) so its CTAs end closer together.
+constexpr int64_t kChunkElems = int64_t(1) << 18;
+constexpr int64_t kGradUnitElems = kChunkElems / 2;
 constexpr int kMaxRounds = 10;
 
 enum : uint32_t {

@@ -6,9 +6,9 @@
 // partial sums live in a fixed file-scope device array instead of a
 // caller-provided workspace.
 //
-// The array holds kNoAllocMaxChunks partials (256 KiB); every GPU that loads
-// this library keeps it for the life of the process. Tensors of more than
-// kNoAllocMaxChunks * 2^16 elements are rejected.
+// The array holds kNoAllocMaxChunks partials (256 KiB), one per 2^16-element
+// chunk; every GPU that loads this library keeps it for the life of the
+// process. Tensors of more than kNoAllocMaxChunks * 2^16 elements are rejected.
 
 #include <mutex>
 
@@ -18,6 +18,7 @@
 namespace smat {
 namespace {
 
+constexpr int64_t kNoAllocChunkElems = int64_t(1) << 16;
 constexpr int64_t kNoAllocMaxChunks = 16384;
 constexpr int kMaxDevices = 64;
 
@@ -34,13 +35,13 @@ __global__ void __launch_bounds__(kBlock) noalloc_chunk_sums_kernel(const void* 
   T.theta = theta;
   T.theta0 = theta0;
   T.flags = vec ? TF_VEC : 0u;
-  const int64_t n_chunks = (numel + kChunkElems - 1) / kChunkElems;
+  const int64_t n_chunks = (numel + kNoAllocChunkElems - 1) / kNoAllocChunkElems;
   for (int64_t c = blockIdx.x; c < n_chunks; c += gridDim.x) {
     Chunk ch;
     ch.tensor = 0;
     ch.pad = 0;
-    ch.begin = c * kChunkElems;
-    ch.end = (c + 1) * kChunkElems < numel ? (c + 1) * kChunkElems : numel;
+    ch.begin = c * kNoAllocChunkElems;
+    ch.end = (c + 1) * kNoAllocChunkElems < numel ? (c + 1) * kNoAllocChunkElems : numel;
     double ds, dq;
     chunk_delta_sums<DT>(T, ch, sh_s, sh_q, ds, dq);
     if (threadIdx.x == 0) {
@@ -96,7 +97,7 @@ extern "C" smat_status smat_delta_sigma_noalloc(const void* d_theta, const void*
   if (dtype != SMAT_F32 && dtype != SMAT_BF16) return record_error(SMAT_ERR_UNSUPPORTED, "dtype not supported");
   if (numel < 0 || !(sigma_rel >= 0.0f) || sigma_rel > 3.0e38f)
     return record_error(SMAT_ERR_INVALID_ARG, "numel < 0 or sigma_rel invalid");
-  const int64_t n_chunks = (numel + kChunkElems - 1) / kChunkElems;
+  const int64_t n_chunks = (numel + kNoAllocChunkElems - 1) / kNoAllocChunkElems;
   if (n_chunks > kNoAllocMaxChunks)
     return record_error(SMAT_ERR_INVALID_ARG,
                         "numel exceeds the fixed scratch array of the allocation-free entry point "

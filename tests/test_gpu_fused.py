@@ -26,8 +26,8 @@ def _cuda():
 
 def _rel_list():
     specs = [W.TensorSpec(f"t{i}", (n,), "linear" if i % 2 else "other", 0.7 if i % 2 else 1.0, 0.0, 0.1)
-             for i, n in enumerate([70_001, 65_536 * 3 + 5, 17, 400_000, 4096])]
-    specs.append(W.TensorSpec("fixed", (100_003,), "linear", 0.5, 1e-3, 0.0))
+             for i, n in enumerate([70_001, 262_144 * 3 + 5, 17, 600_000, 4096])]
+    specs.append(W.TensorSpec("fixed", (300_003,), "linear", 0.5, 1e-3, 0.0))
     return W.Workload("rel_mix", specs, O.BF16, O.BF16, 0.3, 1.0, 1, O.NOISE_GAUSSIAN, 0.02, 3e-4, seed=11)
 
 

@@ -63,7 +63,8 @@ def test_scaled_backbone_lists(name):
 @pytest.mark.parametrize("alpha_mode", [O.ALPHA_GLOBAL, O.ALPHA_PER_TENSOR, O.ALPHA_PER_ELEMENT])
 @pytest.mark.parametrize("dtype", [O.F32, O.BF16])
 def test_modes_small_ragged_list(dtype, alpha_mode, noise):
-    sizes = [0, 1, 3, 15, 16, 17, 31, 33, 255, 4097, 65536, 65537, 200_003]
+    # work chunks are 2^18 elements (gradient-map units 2^17): sizes around both
+    sizes = [0, 1, 3, 15, 16, 17, 31, 33, 255, 131_073, 262_144, 262_145, 600_003]
     keeps = [0.5, 0.9, 0.1, 0.7, 1.0, 0.0, 0.3, 0.5, 0.7, 0.9, 0.3, 0.5 + 2**-10, 0.7]
     specs = [W.TensorSpec(f"t{i}", (n,), "linear", keeps[i], 2e-3 if i % 4 else 0.0) for i, n in enumerate(sizes)]
     w = W.Workload(f"ragged_{dtype}_{alpha_mode}_{noise}", specs, dtype, dtype, 0.2, 1.0, alpha_mode, noise, 0.02, 1e-3,
