@@ -250,7 +250,9 @@ def run_reference(args):
     if rank != 0:
         return 0
     w = workload(args)
-    per_step = int(min(8_000_000, max(200_000, 150.0 / max(1, args.steps + args.warmup) / 250e-9)))
+    # about 150 s in all: the oracle takes about 1 us per element (forward +
+    # gradient map on one Grace core) plus the sample's input generation
+    per_step = int(min(8_000_000, max(200_000, 150.0 / max(1, args.steps + args.warmup) / 1.1e-6)))
     for _ in range(args.warmup):
         oracle_run(w, per_step)
     tot_s, tot_b, tot_n = 0.0, 0, 0
