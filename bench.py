@@ -19,6 +19,13 @@ of all ranks over the slowest rank's time.
 
 --impl reference runs the CPU oracle (the reference arm of this benchmark)
 on a bounded sample of the same workload, on the host cores, rank 0 only.
+
+--sweep PATH measures the flat-tensor sweep instead (one tensor of n = 2^16
+.. 2^32 elements, fp32 and bf16, p_keep 0.1 .. 0.9, alpha per tensor or per
+element ~ U[0, 1), sigma 0 or 1e-4 Gaussian): forward alone and forward +
+gradient map, median of 20 CUDA-event-timed repetitions after 3 warm-ups,
+L2 flushed before each; one JSON line per point to PATH and a summary line
+on stdout.
 """
 
 import argparse
@@ -61,6 +68,9 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--sweep", metavar="PATH", default=None,
+                    help="run the flat-tensor sweep, one JSON line per point to PATH")
+    ap.add_argument("--sweep-max-log2n", type=int, default=32)
     return ap.parse_args()
 
 
@@ -459,10 +469,88 @@ def run_smat(args):
     return 0
 
 
+SWEEP_LOG2N = (16, 18, 20, 22, 24, 26, 28, 30, 32)
+SWEEP_KEEP = (0.1, 0.3, 0.5, 0.7, 0.9)
+SWEEP_ALPHA = (1, 2)  # per tensor, per element
+SWEEP_SIGMA = (0.0, 1e-4)
+
+
+def run_sweep(args):
+    """The flat-tensor sweep (one GPU): for each size and dtype the inputs are
+    generated once; each (p_keep, alpha mode, sigma) point gets its own session."""
+    from paper_2609_33437_gb300 import smat as S
+    S.load_library()
+    dev = torch.device("cuda")
+    peak, peak_kind = measured_peaks()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # twice the L2
+    stream = torch.cuda.current_stream()
+    clocks = None if args.no_clocks else ClockSampler(torch.cuda.current_device())
+    if clocks:
+        clocks.mark()
+    n_points, fracs = 0, []
+    with open(args.sweep, "w") as out:
+        for log2n in [x for x in SWEEP_LOG2N if x <= args.sweep_max_log2n]:
+            for dt in (W.F32, W.BF16):
+                w0 = W.flat_sweep(log2n, dt, 0.5, 1, 0.0)
+                th, t0, sim, gs, go = W.generate(w0, device=dev)
+                b = 2 if dt == W.BF16 else 4
+                n = 1 << log2n
+                for keep in SWEEP_KEEP:
+                    for am in SWEEP_ALPHA:
+                        for sig in SWEEP_SIGMA:
+                            w = W.flat_sweep(log2n, dt, keep, am, sig)
+                            sess = S.SmatSession(th, t0, sim, [keep], [sig], [0.0], seed=w.seed,
+                                                 alpha_min=w.alpha_min, alpha_max=w.alpha_max, alpha_mode=am,
+                                                 noise=w.noise)
+
+                            def fwd(s):
+                                sess.simulate_multi(s)
+
+                            def both(s):
+                                sess.simulate_multi(s)
+                                sess.swap()
+                                sess.grad_map_multi(s, gs, go)
+                                sess.swap()
+
+                            rec = {"log2n": log2n, "dtype": "bf16" if dt == W.BF16 else "f32", "keep": keep,
+                                   "alpha": "per-tensor" if am == 1 else "per-element", "sigma": sig}
+                            for name, fn, nbytes in (("fwd", fwd, 3 * b * n), ("fwd_grad", both, 5 * b * n)):
+                                times = []
+                                for r in range(23):
+                                    flush.zero_()
+                                    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                                    e0.record(stream)
+                                    fn(r)
+                                    e1.record(stream)
+                                    e1.synchronize()
+                                    if r >= 3:
+                                        times.append(e0.elapsed_time(e1))
+                                ms = statistics.median(times)
+                                rec[name + "_ms"] = ms
+                                rec[name + "_gbs"] = nbytes / (ms * 1e-3) / 1e9
+                                rec[name + "_frac"] = rec[name + "_gbs"] / peak
+                            sess.close()
+                            out.write(json.dumps(rec) + "\n")
+                            n_points += 2
+                            if log2n >= 28:
+                                fracs.append(rec["fwd_grad_frac"])
+                del th, t0, sim, gs, go
+                torch.cuda.empty_cache()
+    if clocks:
+        clocks.mark()
+    clk = clocks.stop() if clocks else None
+    print(json.dumps({"sweep": args.sweep, "points": n_points, "peak": peak, "peak_kind": peak_kind,
+                      "median_fwd_grad_frac_n_ge_2^28": statistics.median(fracs) if fracs else None,
+                      "clocks": clk, "l2": "256 MB written before every timed repetition"}))
+    return 0
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
+    if args.sweep:
+        return run_sweep(args)
     return run_smat(args)
 
 

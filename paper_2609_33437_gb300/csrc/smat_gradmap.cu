@@ -108,12 +108,12 @@ __device__ __forceinline__ void grad_chunk(const KArgs& a, const TView& v, const
 
 template <int R, int GDT, bool PE, bool ACC>
 __global__ void __launch_bounds__(kBlock, (GDT == DT_BF16 && !ACC) ? 3 : 2) gradmap_kernel(const __grid_constant__ KArgs a) {
-  constexpr int kUnits = (int)(kChunkElems / kGradUnitElems);
-  for (int64_t u = kUnits * a.chunk_begin + blockIdx.x; u < kUnits * a.chunk_end; u += gridDim.x) {
-    Chunk ch = a.chunks[u / kUnits];
-    ch.begin += (u % kUnits) * kGradUnitElems;
+  const int64_t units = a.grad_units;
+  for (int64_t u = units * a.chunk_begin + blockIdx.x; u < units * a.chunk_end; u += gridDim.x) {
+    Chunk ch = a.chunks[u / units];
+    ch.begin += (u % units) * a.grad_unit;
     if (ch.begin >= ch.end) continue;  // the tensor's last chunk is short
-    if (ch.begin + kGradUnitElems < ch.end) ch.end = ch.begin + kGradUnitElems;
+    if (ch.begin + a.grad_unit < ch.end) ch.end = ch.begin + a.grad_unit;
     const DevTensor& T = a.tensors[ch.tensor];
     const GradPtr G = a.grads[ch.tensor];
     const TView v = make_view(T, a.scal[ch.tensor]);

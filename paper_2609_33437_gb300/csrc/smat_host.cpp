@@ -48,7 +48,21 @@ struct Layout {
 // tensor_done and ready.
 size_t sync_words(int32_t n) { return 4 + 2 * (size_t)n; }
 
-int64_t chunks_of(int64_t numel) { return (numel + kChunkElems - 1) / kChunkElems; }
+int64_t chunks_of(int64_t numel, int64_t chunk_elems) { return (numel + chunk_elems - 1) / chunk_elems; }
+
+// The work-chunk size of a list: the largest power of two in
+// [kMinChunkElems, kMaxChunkElems] with at least kTargetChunks chunks' worth
+// of elements (a pure function of the list, so the workspace size and the
+// context agree).
+int64_t chunk_elems_for(const smat_tensor_desc* t, int32_t n, const smat_config* cfg) {
+  const int forced = (cfg->flags & SMAT_FLAG_CHUNK_LOG2_MASK) >> 8;
+  if (forced) return int64_t(1) << forced;
+  int64_t total = 0;
+  for (int32_t k = 0; k < n; ++k) total = std::min(total + t[k].numel, int64_t(1) << 62);
+  int64_t cs = kMaxChunkElems;
+  while (cs > kMinChunkElems && total < cs * kTargetChunks) cs /= 2;
+  return cs;
+}
 
 Layout layout_for(int32_t n, int64_t n_chunks, bool any_sigma_rel) {
   Layout L;
@@ -74,8 +88,11 @@ smat_status check_config(const smat_config* cfg) {
     return fail(SMAT_ERR_UNSUPPORTED, "noise %d not supported", cfg->noise);
   if (cfg->philox_rounds != 0 && cfg->philox_rounds != 7 && cfg->philox_rounds != 10)
     return fail(SMAT_ERR_UNSUPPORTED, "philox_rounds %d not supported (7 or 10)", cfg->philox_rounds);
-  if (cfg->flags & ~SMAT_FLAG_UNFUSED_STATS)
+  if (cfg->flags & ~(SMAT_FLAG_UNFUSED_STATS | SMAT_FLAG_CHUNK_LOG2_MASK))
     return fail(SMAT_ERR_UNSUPPORTED, "unknown flags 0x%x", cfg->flags);
+  const int chunk_log2 = (cfg->flags & SMAT_FLAG_CHUNK_LOG2_MASK) >> 8;
+  if (chunk_log2 != 0 && (chunk_log2 < 12 || chunk_log2 > 18))
+    return fail(SMAT_ERR_UNSUPPORTED, "chunk log2 %d not in [12, 18]", chunk_log2);
   if (!finite(cfg->alpha_min) || !finite(cfg->alpha_max) || cfg->alpha_min > cfg->alpha_max)
     return fail(SMAT_ERR_INVALID_ARG, "alpha range [%g, %g) invalid", cfg->alpha_min, cfg->alpha_max);
   return SMAT_OK;
@@ -86,7 +103,8 @@ bool overlaps(const void* a, size_t abytes, const void* b, size_t bbytes) {
   return x < y + bbytes && y < x + abytes;
 }
 
-smat_status check_tensors(const smat_tensor_desc* t, int32_t n, int64_t* n_chunks, bool* any_rel) {
+smat_status check_tensors(const smat_tensor_desc* t, int32_t n, const smat_config* cfg, int64_t* n_chunks,
+                          bool* any_rel, int64_t* chunk_elems) {
   if (n < 0) return fail(SMAT_ERR_INVALID_ARG, "n_tensors %d < 0", n);
   if (n > 0 && !t) return fail(SMAT_ERR_INVALID_ARG, "tensors is NULL");
   std::unordered_set<uint32_t> ids;
@@ -120,9 +138,11 @@ smat_status check_tensors(const smat_tensor_desc* t, int32_t n, int64_t* n_chunk
       if (overlaps(d.sim, bytes, d.theta, bytes) || overlaps(d.sim, bytes, d.theta0, bytes))
         return fail(SMAT_ERR_INVALID_ARG, "tensor %d: sim overlaps theta or theta0", k);
     }
-    nc += chunks_of(d.numel);
     rel = rel || d.sigma_rel > 0.0f;
   }
+  const int64_t cs = chunk_elems_for(t, n, cfg);
+  for (int32_t k = 0; k < n; ++k) nc += chunks_of(t[k].numel, cs);
+  *chunk_elems = cs;
   if (nc >= (int64_t(1) << 31)) return fail(SMAT_ERR_INVALID_ARG, "too many chunks (%lld)", (long long)nc);
   *n_chunks = nc;
   *any_rel = rel;
@@ -164,6 +184,7 @@ struct smat_ctx {
   GradPtr* d_grads = nullptr;
   RoundKeys keys;
   int sm_count = 1;
+  int64_t chunk_elems = kMaxChunkElems;  // work-chunk size of this list
   int32_t active = 0;
   int64_t scalars_step = -1;  // step whose scalars the table holds
   bool scalars_sigma = false; // the table's sigma_t are current
@@ -235,6 +256,8 @@ KArgs base_args(const smat_ctx* c, uint32_t step) {
   a.alpha_min = c->cfg.alpha_min;
   a.alpha_width = c->cfg.alpha_max - c->cfg.alpha_min;
   a.alpha_mode = c->cfg.alpha_mode;
+  a.grad_unit = std::min(c->chunk_elems, kMaxGradUnitElems);
+  a.grad_units = (int32_t)(c->chunk_elems / a.grad_unit);
   if (c->d_sync) {
     a.work_counter = c->d_sync;
     a.error = c->d_sync + 2;
@@ -311,7 +334,8 @@ size_t smat_workspace_bytes(const smat_tensor_desc* tensors, int32_t n_tensors, 
   if (check_config(cfg) != SMAT_OK) return 0;
   int64_t nc = 0;
   bool rel = false;
-  if (check_tensors(tensors, n_tensors, &nc, &rel) != SMAT_OK) return 0;
+  int64_t cs = 0;
+  if (check_tensors(tensors, n_tensors, cfg, &nc, &rel, &cs) != SMAT_OK) return 0;
   return layout_for(n_tensors, nc, rel).total;
 }
 
@@ -324,7 +348,8 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
   if (st != SMAT_OK) return st;
   int64_t nc = 0;
   bool rel = false;
-  st = check_tensors(tensors, n_tensors, &nc, &rel);
+  int64_t cs = 0;
+  st = check_tensors(tensors, n_tensors, cfg, &nc, &rel, &cs);
   if (st != SMAT_OK) return st;
   const Layout L = layout_for(n_tensors, nc, rel);
   if (!d_workspace) return fail(SMAT_ERR_WORKSPACE, "workspace is NULL");
@@ -337,6 +362,7 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
   c->cfg = *cfg;
   c->rounds = cfg->philox_rounds == 7 ? 7 : 10;
   c->any_sigma_rel = rel;
+  c->chunk_elems = cs;
   c->keys = make_keys(cfg->seed);
   char* ws = static_cast<char*>(d_workspace);
   c->d_tensors = reinterpret_cast<DevTensor*>(ws + L.tensors);
@@ -383,14 +409,14 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
       if (d.sigma_rel > 0.0f) flags |= TF_SIGMA_REL;
       T.flags = flags;
       T.chunk_first = (int32_t)c->h_chunks.size();
-      const int64_t m = chunks_of(d.numel);
+      const int64_t m = chunks_of(d.numel, cs);
       T.n_chunks = (int32_t)m;
       for (int64_t j = 0; j < m; ++j) {
         Chunk ch;
         ch.tensor = k;
         ch.pad = 0;
-        ch.begin = j * kChunkElems;
-        ch.end = (j + 1) * kChunkElems < d.numel ? (j + 1) * kChunkElems : d.numel;
+        ch.begin = j * cs;
+        ch.end = (j + 1) * cs < d.numel ? (j + 1) * cs : d.numel;
         c->h_chunks.push_back(ch);
       }
     }

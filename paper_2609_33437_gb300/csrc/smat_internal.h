@@ -13,13 +13,18 @@ namespace smat {
 enum : uint32_t { S_MASK = 0, S_NOISE = 1, S_ALPHA_E = 2, S_ALPHA_T = 3, S_MASK_LO = 4 };
 constexpr uint32_t kGlobalAlphaTensor = 0x0FFFFFFFu;
 
-// Elements per work chunk of the multi-tensor launches (a multiple of 16, so
-// a chunk never splits a 16-element mask draw group of an aligned tensor).
-// Statistics and forward work items are whole chunks; the gradient map,
-// whose CTAs take chunks in a fixed grid-stride order, walks halves of
-// chunks (kGradUnitElems) so its CTAs end closer together.
-constexpr int64_t kChunkElems = int64_t(1) << 18;
-constexpr int64_t kGradUnitElems = kChunkElems / 2;
+// Elements per work chunk of the multi-tensor launches: a power of two from
+// kMinChunkElems to kMaxChunkElems chosen per tensor list (the largest that
+// still gives kTargetChunks chunks, so small lists fill the GPU and large
+// ones pay few per-chunk costs); always a multiple of 16, so a chunk never
+// splits a 16-element mask draw group of an aligned tensor. Statistics and
+// forward work items are whole chunks; the gradient map, whose CTAs take
+// its units in a fixed grid-stride order, walks units of at most
+// kMaxGradUnitElems so its CTAs end closer together.
+constexpr int64_t kMinChunkElems = int64_t(1) << 12;
+constexpr int64_t kMaxChunkElems = int64_t(1) << 18;
+constexpr int64_t kTargetChunks = 4096;
+constexpr int64_t kMaxGradUnitElems = int64_t(1) << 17;
 constexpr int kMaxRounds = 10;
 
 enum : uint32_t {
@@ -87,6 +92,8 @@ struct KArgs {
   uint32_t* bits;        // mask_bits output
   int64_t chunk_begin;   // chunk-table range handled by this launch
   int64_t chunk_end;
+  int64_t grad_unit;     // gradient map: elements per unit (divides the chunk size)
+  int32_t grad_units;    // gradient map: units per chunk
   RoundKeys key;
   uint32_t step;
   int32_t n_tensors;

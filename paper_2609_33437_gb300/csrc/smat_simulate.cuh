@@ -149,7 +149,7 @@ __device__ __forceinline__ void sim_resolve(const KArgs& a, const TView& v, cons
 // cannot overflow). The counters are reset by the caller before the barrier
 // that precedes the chunk.
 struct ChunkQueue {
-  static constexpr int kGroups = kChunkElems / 16;
+  static constexpr int kGroups = kMaxChunkElems / 16;
   uint16_t e[kGroups];
   int n_tie;
   int n_tail;

@@ -52,6 +52,11 @@ class Config(ctypes.Structure):
 SMAT_FLAG_UNFUSED_STATS = 1
 
 
+def SMAT_FLAG_CHUNK_LOG2(k: int) -> int:
+    """Force the work-chunk size to 2^k elements (12 <= k <= 18)."""
+    return k << 8
+
+
 _lib = None
 
 

@@ -44,11 +44,11 @@ def orc_tensor(w: W.Workload, k: int, numel=None, elem_offset=0):
                     sigma_rel=t.sigma_rel, elem_offset=elem_offset)
 
 
-def session_for(w: W.Workload, th, t0, sim, rounds: int = 10, elem_offsets=None):
+def session_for(w: W.Workload, th, t0, sim, rounds: int = 10, elem_offsets=None, flags: int = 0):
     return S.SmatSession(th, t0, sim, [t.keep_prob for t in w.tensors], [t.sigma for t in w.tensors],
                          [t.sigma_rel for t in w.tensors], elem_offsets=elem_offsets, seed=w.seed,
                          alpha_min=w.alpha_min, alpha_max=w.alpha_max, alpha_mode=w.alpha_mode, noise=w.noise,
-                         philox_rounds=rounds)
+                         philox_rounds=rounds, flags=flags)
 
 
 def _ordered_bf16(b: np.ndarray) -> np.ndarray:
@@ -109,7 +109,7 @@ def compare(got_bits, ref_bits, dtype, noise, th=None, t0=None, what=""):
     assert not bad.any(), f"{what}: {int(bad.sum())} elements beyond 1e-6 relative (max ratio {float((err / scale).max())})"
 
 
-def run_and_check_full(w: W.Workload, steps=(0, 1, 2), rounds=10, accumulate=False, gdtype=None):
+def run_and_check_full(w: W.Workload, steps=(0, 1, 2), rounds=10, accumulate=False, gdtype=None, flags=0):
     """Generate w on the GPU, run simulate + gradient map for each step through
     the C ABI and compare every element with the oracle."""
     dev = torch.device("cuda")
@@ -118,7 +118,7 @@ def run_and_check_full(w: W.Workload, steps=(0, 1, 2), rounds=10, accumulate=Fal
         gs = [g.to(W.torch_dtype(gdtype)) for g in gs]
         go = [torch.empty_like(g) for g in gs]
     gdt = w.gdtype if gdtype is None else gdtype
-    sess = session_for(w, th, t0, sim, rounds=rounds)
+    sess = session_for(w, th, t0, sim, rounds=rounds, flags=flags)
     hth = [to_host(x) for x in th]
     ht0 = [to_host(x) for x in t0]
     hgs = [to_host(x) for x in gs]

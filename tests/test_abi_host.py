@@ -78,6 +78,30 @@ def test_workspace_size_scales_with_chunks(L):
     assert L.smat_workspace_bytes(None, 0, ctypes.byref(cfg())) >= 0
 
 
+def test_chunk_size_rule_and_override(L):
+    """Automatic chunk size: the largest power of two in [2^12, 2^18] with at
+    least 4096 chunks' worth of elements; the override forces 2^k. The chunk
+    count shows in the workspace size (24 B chunk table + 4 B work item per
+    chunk, up to section alignment)."""
+    def spaced(n):
+        d = desc(n)
+        d.theta0 = d.theta + 2 * n
+        d.sim = d.theta + 4 * n
+        return d
+
+    n = 1 << 26  # automatic: 2^14-element chunks, 4096 of them
+    auto = ws_bytes(L, [spaced(n)], cfg())
+    f12 = ws_bytes(L, [spaced(n)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(12)))
+    f14 = ws_bytes(L, [spaced(n)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(14)))
+    f13 = ws_bytes(L, [spaced(n)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(13)))
+    f18 = ws_bytes(L, [spaced(n)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(18)))
+    assert auto > 0 and f14 == auto and f13 > auto
+    assert f12 - f18 >= 28 * ((n >> 12) - (n >> 18)) - 4 * 256
+    big = 1 << 31  # automatic: 2^18 (8192 chunks)
+    assert ws_bytes(L, [spaced(big)], cfg()) == ws_bytes(L, [spaced(big)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(18)))
+    assert ws_bytes(L, [spaced(big)], cfg()) < ws_bytes(L, [spaced(big)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(17)))
+
+
 @pytest.mark.parametrize("bad,code", [
     (dict(keep=1.5), 1), (dict(keep=-0.1), 1), (dict(keep=float("nan")), 1), (dict(sigma=-1.0), 1),
     (dict(rel=float("inf")), 1), (dict(numel=-1), 1), (dict(numel=1 << 40), 1), (dict(tid=0x0FFFFFFF), 1),
@@ -96,6 +120,8 @@ def test_init_rejects_invalid_tensor(L, bad, code):
 @pytest.mark.parametrize("bad,code", [
     (dict(alpha_mode=3), 2), (dict(noise=2), 2), (dict(philox_rounds=8), 2),
     (dict(alpha_min=0.9, alpha_max=0.5), 1), (dict(alpha_min=float("nan")), 1),
+    (dict(flags=S.SMAT_FLAG_CHUNK_LOG2(11)), 2), (dict(flags=S.SMAT_FLAG_CHUNK_LOG2(19)), 2), (dict(flags=1 << 14), 2),
+    (dict(flags=2), 2),
 ])
 def test_init_rejects_invalid_config(L, bad, code):
     ctx = ctypes.c_void_p()

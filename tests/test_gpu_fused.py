@@ -31,15 +31,17 @@ def _rel_list():
     return W.Workload("rel_mix", specs, O.BF16, O.BF16, 0.3, 1.0, 1, O.NOISE_GAUSSIAN, 0.02, 3e-4, seed=11)
 
 
-def test_fused_and_unfused_give_identical_outputs():
+@pytest.mark.parametrize("chunk_log2", [0, 18])
+def test_fused_and_unfused_give_identical_outputs(chunk_log2):
     w = _rel_list()
     dev = torch.device("cuda")
     th, t0, sim_a, gs, go = W.generate(w, device=dev)
     sim_b = [torch.empty_like(x) for x in sim_a]
-    a = session_for(w, th, t0, sim_a)
+    chunk = S.SMAT_FLAG_CHUNK_LOG2(chunk_log2) if chunk_log2 else 0
+    a = session_for(w, th, t0, sim_a, flags=chunk)
     b = S.SmatSession(th, t0, sim_b, [t.keep_prob for t in w.tensors], [t.sigma for t in w.tensors],
                       [t.sigma_rel for t in w.tensors], seed=w.seed, alpha_min=w.alpha_min, alpha_max=w.alpha_max,
-                      alpha_mode=w.alpha_mode, noise=w.noise, flags=S.SMAT_FLAG_UNFUSED_STATS)
+                      alpha_mode=w.alpha_mode, noise=w.noise, flags=S.SMAT_FLAG_UNFUSED_STATS | chunk)
     for step in (0, 3):
         a.simulate_multi(step)
         b.simulate_multi(step)
@@ -49,8 +51,9 @@ def test_fused_and_unfused_give_identical_outputs():
     assert a.poll_errors() == 0 and b.poll_errors() == 0
 
 
-def test_fused_list_matches_oracle_and_reports_no_errors():
-    run_and_check_full(_rel_list(), steps=(0, 1, 5))
+@pytest.mark.parametrize("chunk_log2", [0, 18])
+def test_fused_list_matches_oracle_and_reports_no_errors(chunk_log2):
+    run_and_check_full(_rel_list(), steps=(0, 1, 5), flags=S.SMAT_FLAG_CHUNK_LOG2(chunk_log2) if chunk_log2 else 0)
 
 
 def test_bounded_wait_runs_out_and_reports():

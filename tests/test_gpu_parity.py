@@ -72,6 +72,20 @@ def test_modes_small_ragged_list(dtype, alpha_mode, noise):
     run_and_check_full(w, steps=(0, 7))
 
 
+@pytest.mark.parametrize("chunk_log2", [12, 16, 18])
+@pytest.mark.parametrize("noise", [O.NOISE_UNIFORM, O.NOISE_GAUSSIAN])
+def test_forced_chunk_sizes_ragged_list(chunk_log2, noise):
+    """The work-chunk size (chosen per list; forced here) changes no result:
+    ragged tensors around 2^12, 2^16, 2^17 (gradient-map unit) and 2^18
+    boundaries, bf16, elementwise against the oracle."""
+    sizes = [5, 4096, 4097, 65_536 + 17, 131_072, 262_144, 262_161, 600_003, 33]
+    keeps = [0.7, 0.5, 0.3, 0.7, 0.9, 0.1, 0.7, 0.5 + 2**-10, 1.0]
+    specs = [W.TensorSpec(f"t{i}", (n,), "linear", keeps[i], 2e-3 if i % 3 else 0.0) for i, n in enumerate(sizes)]
+    w = W.Workload(f"chunks_{chunk_log2}_{noise}", specs, O.BF16, O.BF16, 0.3, 1.0, O.ALPHA_PER_TENSOR, noise, 0.02,
+                   1e-3, seed=0x5EED_0018)
+    run_and_check_full(w, steps=(0, 3), flags=S.SMAT_FLAG_CHUNK_LOG2(chunk_log2))
+
+
 def test_philox_7_rounds_and_accumulate_and_f32_grads_on_bf16_params():
     specs = [W.TensorSpec("a", (70_001,), "linear", 0.7, 1e-3), W.TensorSpec("b", (9,), "other", 1.0, 1e-3)]
     w = W.Workload("r7", specs, O.BF16, O.BF16, 0.3, 1.0, 1, O.NOISE_UNIFORM, 0.02, 1e-3, seed=5)
