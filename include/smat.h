@@ -96,8 +96,8 @@ typedef struct {
 
 /* smat_config.flags */
 #define SMAT_FLAG_UNFUSED_STATS 1 /* run delta statistics as a separate pass, then a grid-stride forward */
-/* Work-chunk size. By default each list gets the largest power of two from
- * 2^12 to 2^18 elements that still gives 4096 chunks' worth of elements.
+/* Work-chunk size. By default each list gets the largest power of two cs from
+ * 2^12 to 2^18 elements with cs^2 / 64 <= its total number of elements.
  * SMAT_FLAG_CHUNK_LOG2(k), 12 <= k <= 18, forces 2^k (results do not depend
  * on it; tests use it to run small lists with large chunks). Pass the same
  * flags to smat_workspace_bytes and smat_init. */

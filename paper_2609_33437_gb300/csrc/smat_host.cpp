@@ -50,17 +50,17 @@ size_t sync_words(int32_t n) { return 4 + 2 * (size_t)n; }
 
 int64_t chunks_of(int64_t numel, int64_t chunk_elems) { return (numel + chunk_elems - 1) / chunk_elems; }
 
-// The work-chunk size of a list: the largest power of two in
-// [kMinChunkElems, kMaxChunkElems] with at least kTargetChunks chunks' worth
-// of elements (a pure function of the list, so the workspace size and the
-// context agree).
+// The work-chunk size of a list: the largest power of two cs in
+// [kMinChunkElems, kMaxChunkElems] with cs^2 / 64 <= total elements (a pure
+// function of the list and flags, so the workspace size and the context
+// agree).
 int64_t chunk_elems_for(const smat_tensor_desc* t, int32_t n, const smat_config* cfg) {
   const int forced = (cfg->flags & SMAT_FLAG_CHUNK_LOG2_MASK) >> 8;
   if (forced) return int64_t(1) << forced;
   int64_t total = 0;
   for (int32_t k = 0; k < n; ++k) total = std::min(total + t[k].numel, int64_t(1) << 62);
-  int64_t cs = kMaxChunkElems;
-  while (cs > kMinChunkElems && total < cs * kTargetChunks) cs /= 2;
+  int64_t cs = kMinChunkElems;
+  while (cs < kMaxChunkElems && (2 * cs) * (2 * cs) / 64 <= total) cs *= 2;
   return cs;
 }
 

@@ -14,16 +14,17 @@ enum : uint32_t { S_MASK = 0, S_NOISE = 1, S_ALPHA_E = 2, S_ALPHA_T = 3, S_MASK_
 constexpr uint32_t kGlobalAlphaTensor = 0x0FFFFFFFu;
 
 // Elements per work chunk of the multi-tensor launches: a power of two from
-// kMinChunkElems to kMaxChunkElems chosen per tensor list (the largest that
-// still gives kTargetChunks chunks, so small lists fill the GPU and large
-// ones pay few per-chunk costs); always a multiple of 16, so a chunk never
+// kMinChunkElems to kMaxChunkElems chosen per tensor list, about
+// sqrt(64 x total elements) (the largest cs with cs^2 / 64 <= total): large
+// chunks pay the per-item costs (work-list claim, descriptor loads, barriers,
+// the first loads' latency) less often, many chunks keep every CTA busy to
+// the end; measured best from 2^22 to 2^32 elements. Always a multiple of 16, so a chunk never
 // splits a 16-element mask draw group of an aligned tensor. Statistics and
 // forward work items are whole chunks; the gradient map, whose CTAs take
 // its units in a fixed grid-stride order, walks units of at most
 // kMaxGradUnitElems so its CTAs end closer together.
 constexpr int64_t kMinChunkElems = int64_t(1) << 12;
 constexpr int64_t kMaxChunkElems = int64_t(1) << 18;
-constexpr int64_t kTargetChunks = 4096;
 constexpr int64_t kMaxGradUnitElems = int64_t(1) << 17;
 constexpr int kMaxRounds = 10;
 

@@ -79,8 +79,8 @@ def test_workspace_size_scales_with_chunks(L):
 
 
 def test_chunk_size_rule_and_override(L):
-    """Automatic chunk size: the largest power of two in [2^12, 2^18] with at
-    least 4096 chunks' worth of elements; the override forces 2^k. The chunk
+    """Automatic chunk size: the largest power of two cs in [2^12, 2^18] with
+    cs^2 / 64 <= total elements; the override forces 2^k. The chunk
     count shows in the workspace size (24 B chunk table + 4 B work item per
     chunk, up to section alignment)."""
     def spaced(n):
@@ -89,15 +89,17 @@ def test_chunk_size_rule_and_override(L):
         d.sim = d.theta + 4 * n
         return d
 
-    n = 1 << 26  # automatic: 2^14-element chunks, 4096 of them
+    n = 1 << 26  # automatic: 2^16-element chunks (2^32 / 64 <= 2^26 < 2^34 / 64)
     auto = ws_bytes(L, [spaced(n)], cfg())
     f12 = ws_bytes(L, [spaced(n)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(12)))
-    f14 = ws_bytes(L, [spaced(n)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(14)))
-    f13 = ws_bytes(L, [spaced(n)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(13)))
+    f16 = ws_bytes(L, [spaced(n)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(16)))
+    f15 = ws_bytes(L, [spaced(n)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(15)))
     f18 = ws_bytes(L, [spaced(n)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(18)))
-    assert auto > 0 and f14 == auto and f13 > auto
+    assert auto > 0 and f16 == auto and f15 > auto
+    assert ws_bytes(L, [spaced(1 << 22)], cfg()) == ws_bytes(L, [spaced(1 << 22)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(14)))
+    assert ws_bytes(L, [spaced(100)], cfg()) == ws_bytes(L, [spaced(100)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(12)))
     assert f12 - f18 >= 28 * ((n >> 12) - (n >> 18)) - 4 * 256
-    big = 1 << 31  # automatic: 2^18 (8192 chunks)
+    big = 1 << 31  # automatic: 2^18
     assert ws_bytes(L, [spaced(big)], cfg()) == ws_bytes(L, [spaced(big)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(18)))
     assert ws_bytes(L, [spaced(big)], cfg()) < ws_bytes(L, [spaced(big)], cfg(flags=S.SMAT_FLAG_CHUNK_LOG2(17)))
 
