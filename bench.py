@@ -68,6 +68,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--philox-rounds", type=int, choices=[7, 10], default=10,
+                    help="Philox-4x32 rounds of the random streams (10 is the default stream definition)")
     ap.add_argument("--sweep", metavar="PATH", default=None,
                     help="run the flat-tensor sweep, one JSON line per point to PATH")
     ap.add_argument("--sweep-max-log2n", type=int, default=32)
@@ -365,7 +367,8 @@ def run_smat(args):
     def make_session(th, t0, sim):
         return S.SmatSession(th, t0, sim, [t.keep_prob for t in w.tensors], [t.sigma for t in w.tensors],
                              [t.sigma_rel for t in w.tensors], seed=w.seed, alpha_min=w.alpha_min,
-                             alpha_max=w.alpha_max, alpha_mode=w.alpha_mode, noise=w.noise)
+                             alpha_max=w.alpha_max, alpha_mode=w.alpha_mode, noise=w.noise,
+                             philox_rounds=args.philox_rounds)
 
     th, t0, sim, gs, go = W.generate(w, device=dev)
     sess = make_session(th, t0, sim)
@@ -436,6 +439,7 @@ def run_smat(args):
                           "param_dtype": "bf16" if w.dtype == W.BF16 else "f32",
                           "grad_dtype": "bf16" if w.gdtype == W.BF16 else "f32",
                           "noise": "gaussian" if w.noise == 1 else "uniform", "alpha": f"per-tensor U[{w.alpha_min}, {w.alpha_max})",
+                          "philox_rounds": args.philox_rounds,
                           "bytes_per_step": bytes_step, "l2": "inputs larger than L2 (no flush needed)",
                           "parallelism": f"{world} independent experts (one per GPU)"},
                "kernels": per_kernel,
