@@ -52,7 +52,7 @@ UNIT = "GB/s"
 FALLBACK_HBM_GBS = 6800.0
 NOMINAL_HBM_GBS = 8000.0
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2609_33437_gb300", "csrc", f)
-                  for f in ("smat_device.cuh", "smat_simulate.cuh", "smat_sim_bf16.cu", "smat_gradmap.cu",
+                  for f in ("smat_device.cuh", "smat_simulate.cuh", "smat_fused_bf16.cu", "smat_gradmap.cu",
                             "smat_internal.h")]
 
 
@@ -68,6 +68,10 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--theta0", choices=["device", "inplace", "host"], default="device",
+                    help="where theta0 lives: its own HBM buffer (default); in-place (the sim buffer holds theta0 "
+                         "and is refilled from pinned host memory every step, inside the timed region); pinned "
+                         "host memory read directly by the kernels")
     ap.add_argument("--philox-rounds", type=int, choices=[7, 10], default=10,
                     help="Philox-4x32 rounds of the random streams (10 is the default stream definition)")
     ap.add_argument("--sweep", metavar="PATH", default=None,
@@ -371,6 +375,12 @@ def run_smat(args):
                              philox_rounds=args.philox_rounds)
 
     th, t0, sim, gs, go = W.generate(w, device=dev)
+    host_t0 = None
+    if args.theta0 == "host":
+        t0 = [x.cpu().pin_memory() for x in t0]
+    elif args.theta0 == "inplace":
+        host_t0 = [x.cpu().pin_memory() for x in t0]
+        sim = t0  # one buffer per tensor: theta0, overwritten by theta~, refilled every step
     sess = make_session(th, t0, sim)
 
     def step(s):
@@ -378,6 +388,8 @@ def run_smat(args):
         sess.swap()
         sess.grad_map_multi(s, gs, go)
         sess.swap()
+        if host_t0 is not None:
+            sess.refill_theta0(host_t0)
 
     for s in range(args.warmup):
         step(s)
@@ -441,6 +453,7 @@ def run_smat(args):
                           "noise": "gaussian" if w.noise == 1 else "uniform", "alpha": f"per-tensor U[{w.alpha_min}, {w.alpha_max})",
                           "philox_rounds": args.philox_rounds,
                           "bytes_per_step": bytes_step, "l2": "inputs larger than L2 (no flush needed)",
+                          "theta0": args.theta0,
                           "parallelism": f"{world} independent experts (one per GPU)"},
                "kernels": per_kernel,
                "roofline": {"bound": "hbm", "kernel": "stats_simulate (fused)" if fused else "simulate",
@@ -449,7 +462,13 @@ def run_smat(args):
                             "traffic": traffic["dram_bytes_per_launch"] if traffic else None,
                             "algorithmic_bytes_per_launch": nb["simulate"]},
                "clocks": clk, "gpu_launches": launches}
-    if not args.no_e2e:
+    if out is not None and args.theta0 != "device":
+        kern_ms = sum(v["avg_ms"] * v["launches"] for v in per_kernel.values()) / args.steps
+        out["theta0_mode"] = {"kernel_ms_per_step": kern_ms, "other_ms_per_step": ms_step - kern_ms,
+                              "note": "in-place: the other time is the host-to-device refill of theta0 "
+                                      "(the paper hides it behind ordinary steps); host: theta0 is read "
+                                      "by the kernels from pinned host memory"}
+    if not args.no_e2e and args.theta0 == "device":
         need = 5 * 2 * w.numel
         avail = host_available_bytes() / max(1, world)
         ew = w

@@ -78,9 +78,15 @@ typedef enum {
 } smat_alpha_mode;
 
 /* One trainable tensor. theta (the expert's parameters, read), theta0 (the
- * shared initialisation, read) and sim (theta~, written) are device pointers
- * of `numel` elements of `dtype`, contiguous; they must stay valid from
- * smat_init to smat_destroy. sim must not overlap theta or theta0. */
+ * shared initialisation, read) and sim (theta~, written) are pointers of
+ * `numel` elements of `dtype`, contiguous, readable (theta, theta0) and
+ * writable (sim) by the GPU: device memory, or mapped pinned host memory for
+ * theta0; they must stay valid from smat_init to smat_destroy. sim must not
+ * overlap theta. sim == theta0 selects the in-place mode (Sec. 4.3: one extra
+ * buffer per tensor instead of two): the buffer holds theta0 until a forward
+ * overwrites it with theta~, and must be refilled with theta0
+ * (smat_refill_theta0 or smat_mark_theta0_resident) before the next forward.
+ * Any other overlap of sim and theta0 is an error. */
 typedef struct {
   const void* theta;
   const void* theta0;
@@ -133,7 +139,9 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
  * per-call scalars (and, for sigma_rel tensors, the delta statistics) and
  * writes theta~ into each tensor's `sim`. Requires the original storage to be
  * active (SMAT_ERR_STATE otherwise): the simulated state is rebuilt only
- * while the model reads theta. By default the forward is one persistent
+ * while the model reads theta; with in-place tensors it also requires theta0
+ * to be resident in their sim buffers (SMAT_ERR_STATE otherwise) and leaves
+ * theta~ there. By default the forward is one persistent
  * launch whose CTAs take chunks of 2^18 elements from a work list in order;
  * with sigma_rel tensors the statistics run in the same launch (statistics
  * of later tensors beside the forward of earlier ones).
@@ -158,6 +166,21 @@ smat_status smat_grad_map_multi(smat_ctx* ctx, uint32_t step, const void* const*
  * Host only: no device work, no copy. */
 smat_status smat_swap(smat_ctx* ctx, int32_t* active_out);
 
+/* In-place mode: copy theta0 back into the sim buffer of every in-place
+ * tensor (sim == theta0) from h_theta0[k], a HOST array of n_tensors host
+ * pointers (pinned memory for an asynchronous copy; entries of tensors that
+ * are not in-place are ignored and may be NULL), with one cudaMemcpyAsync per
+ * tensor on `stream`, and mark theta0 resident. The paper hides this copy
+ * behind ordinary training steps (Sec. 4.3, App. E); issue it on a side
+ * stream and order the next forward after it. SMAT_ERR_STATE while the
+ * simulated storage is active (the model reads those buffers). */
+smat_status smat_refill_theta0(smat_ctx* ctx, const void* const* h_theta0, smat_stream_t stream);
+
+/* In-place mode: the caller has put theta0 back into the sim buffers itself
+ * (ordered before the next forward). SMAT_ERR_STATE while the simulated
+ * storage is active. */
+smat_status smat_mark_theta0_resident(smat_ctx* ctx);
+
 /* Which storage is active (0 = theta, 1 = sim). */
 smat_status smat_active(const smat_ctx* ctx, int32_t* active_out);
 
@@ -171,7 +194,9 @@ smat_status smat_mask_bits(smat_ctx* ctx, uint32_t step, int32_t tensor_index, u
 /* Test hook: per-call scalars at `step` into the device buffer d_out of
  * 4 * n_tensors floats: {alpha_t, c_t = alpha_t / p_keep, sigma_t,
  * noise scale} per tensor (alpha_t and c_t are 0 in per-element mode).
- * Computes the delta statistics first for sigma_rel tensors. */
+ * Computes the delta statistics first for sigma_rel tensors (which, for
+ * in-place sigma_rel tensors, needs theta0 resident: SMAT_ERR_STATE
+ * otherwise). */
 smat_status smat_tensor_scalars(smat_ctx* ctx, uint32_t step, float* d_out, smat_stream_t stream);
 
 /* Release the host context (the caller still owns and frees the workspace

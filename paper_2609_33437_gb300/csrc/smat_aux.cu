@@ -131,9 +131,21 @@ __global__ void debug_noise_unit_kernel(const uint32_t* words, int64_t n, int no
 }  // namespace
 
 cudaError_t launch_simulate(const KArgs& a, int grid, int dtype, int noise, bool per_elem_alpha,
-                            int rounds, cudaStream_t s) {
+                            int rounds, bool inplace, cudaStream_t s) {
+  if (inplace)
+    return dtype == DT_BF16 ? launch_simulate_inplace_bf16(a, grid, noise, per_elem_alpha, rounds, s)
+                            : launch_simulate_inplace_f32(a, grid, noise, per_elem_alpha, rounds, s);
   return dtype == DT_BF16 ? launch_simulate_bf16(a, grid, noise, per_elem_alpha, rounds, s)
                           : launch_simulate_f32(a, grid, noise, per_elem_alpha, rounds, s);
+}
+
+cudaError_t launch_stats_simulate(const KArgs& a, int grid, int dtype, int noise, bool per_elem_alpha,
+                                  int rounds, bool inplace, cudaStream_t s) {
+  if (inplace)
+    return dtype == DT_BF16 ? launch_stats_simulate_inplace_bf16(a, grid, noise, per_elem_alpha, rounds, s)
+                            : launch_stats_simulate_inplace_f32(a, grid, noise, per_elem_alpha, rounds, s);
+  return dtype == DT_BF16 ? launch_stats_simulate_bf16(a, grid, noise, per_elem_alpha, rounds, s)
+                          : launch_stats_simulate_f32(a, grid, noise, per_elem_alpha, rounds, s);
 }
 
 int streaming_ctas_per_sm(int dtype, int noise, bool pe, int rounds) {

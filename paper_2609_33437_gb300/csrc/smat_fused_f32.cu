@@ -1,0 +1,15 @@
+// Rows a2 + a3 (the persistent work-list forward, with the delta statistics of
+// sigma_rel tensors) for f32 parameters. A translation unit of its own so the
+// forward kernels compile in parallel.
+#include "smat_simulate.cuh"
+
+namespace smat {
+
+cudaError_t launch_stats_simulate_f32(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
+                                      cudaStream_t s) {
+  if (a.n_items <= 0) return cudaSuccess;
+  return rounds == 7 ? fused_run<7, DT_F32, false>(a, grid, noise, per_elem_alpha, s)
+                     : fused_run<10, DT_F32, false>(a, grid, noise, per_elem_alpha, s);
+}
+
+}  // namespace smat

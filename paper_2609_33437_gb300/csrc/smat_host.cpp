@@ -135,8 +135,9 @@ smat_status check_tensors(const smat_tensor_desc* t, int32_t n, const smat_confi
       if ((uintptr_t)d.theta % es || (uintptr_t)d.theta0 % es || (uintptr_t)d.sim % es)
         return fail(SMAT_ERR_ALIGNMENT, "tensor %d: pointer not aligned to %zu bytes", k, es);
       const size_t bytes = es * (size_t)d.numel;
-      if (overlaps(d.sim, bytes, d.theta, bytes) || overlaps(d.sim, bytes, d.theta0, bytes))
-        return fail(SMAT_ERR_INVALID_ARG, "tensor %d: sim overlaps theta or theta0", k);
+      // sim == theta0 is the in-place mode; any other overlap is an error
+      if (overlaps(d.sim, bytes, d.theta, bytes) || (d.sim != d.theta0 && overlaps(d.sim, bytes, d.theta0, bytes)))
+        return fail(SMAT_ERR_INVALID_ARG, "tensor %d: sim overlaps theta, or theta0 without being equal to it", k);
     }
     rel = rel || d.sigma_rel > 0.0f;
   }
@@ -146,6 +147,32 @@ smat_status check_tensors(const smat_tensor_desc* t, int32_t n, const smat_confi
   if (nc >= (int64_t(1) << 31)) return fail(SMAT_ERR_INVALID_ARG, "too many chunks (%lld)", (long long)nc);
   *n_chunks = nc;
   *any_rel = rel;
+  return SMAT_OK;
+}
+
+// Every data pointer must be usable by the GPU's kernels as it is: device or
+// managed memory, host memory registered with CUDA (pinned; under unified
+// addressing its device address is the host address), or any host memory
+// when the device reads pageable memory directly (coherent CPU-GPU systems).
+smat_status check_gpu_access(const smat_tensor_desc* t, int32_t n) {
+  int dev = 0, pageable = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return fail(SMAT_ERR_CUDA, "no current CUDA device");
+  if (cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccess, dev) != cudaSuccess) pageable = 0;
+  for (int32_t k = 0; k < n; ++k) {
+    if (t[k].numel <= 0) continue;
+    const void* ptrs[3] = {t[k].theta, t[k].theta0, t[k].sim};
+    for (const void* p : ptrs) {
+      cudaPointerAttributes at;
+      if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+        cudaGetLastError();
+        return fail(SMAT_ERR_INVALID_ARG, "tensor %d: pointer attributes unavailable", k);
+      }
+      const bool ok = at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged ||
+                      (at.type == cudaMemoryTypeHost && at.devicePointer == p) ||
+                      (at.type == cudaMemoryTypeUnregistered && pageable);
+      if (!ok) return fail(SMAT_ERR_INVALID_ARG, "tensor %d: a data pointer is not accessible from the GPU", k);
+    }
+  }
   return SMAT_OK;
 }
 
@@ -177,6 +204,11 @@ struct smat_ctx {
   int64_t range_begin[2] = {0, 0};  // chunk range per dtype (F32, BF16)
   int64_t range_end[2] = {0, 0};
   bool any_sigma_rel = false;
+  // in-place tensors (sim == theta0): their sim buffers hold theta0 until a
+  // forward overwrites it; a refill makes them hold theta0 again
+  bool any_inplace = false;
+  bool any_inplace_rel = false;
+  bool theta0_resident = true;
   DevTensor* d_tensors = nullptr;
   Chunk* d_chunks = nullptr;
   DevScalars* d_scal = nullptr;
@@ -356,6 +388,8 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
   if ((uintptr_t)d_workspace % kAlign) return fail(SMAT_ERR_WORKSPACE, "workspace not 256-byte aligned");
   if (workspace_bytes < L.total)
     return fail(SMAT_ERR_WORKSPACE, "workspace %zu bytes < %zu needed", workspace_bytes, L.total);
+  st = check_gpu_access(tensors, n_tensors);
+  if (st != SMAT_OK) return st;
 
   smat_ctx* c = new smat_ctx();
   c->desc.assign(tensors, tensors + n_tensors);
@@ -407,6 +441,11 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
           ((uintptr_t)d.sim % 32 == 0) && (d.elem_offset % 16 == 0))
         flags |= TF_VEC;
       if (d.sigma_rel > 0.0f) flags |= TF_SIGMA_REL;
+      if (d.numel > 0 && d.sim == d.theta0) {
+        flags |= TF_INPLACE;
+        c->any_inplace = true;
+        c->any_inplace_rel = c->any_inplace_rel || d.sigma_rel > 0.0f;
+      }
       T.flags = flags;
       T.chunk_first = (int32_t)c->h_chunks.size();
       const int64_t m = chunks_of(d.numel, cs);
@@ -457,6 +496,9 @@ smat_status smat_simulate_multi(smat_ctx* c, uint32_t step, smat_stream_t stream
   if (!c) return fail(SMAT_ERR_INVALID_ARG, "ctx is NULL");
   if (c->active != 0)
     return fail(SMAT_ERR_STATE, "simulate called while the simulated storage is active; swap back first");
+  if (c->any_inplace && !c->theta0_resident)
+    return fail(SMAT_ERR_STATE, "in-place tensors: theta0 has not been refilled since the last forward");
+  c->theta0_resident = false;  // the forward below overwrites it
   if (c->fused) {
     // a1 (alpha, c; sigma of fixed-sigma tensors; counter reset), then a3 (with a2
     // for sigma_rel tensors) in one work-list launch
@@ -474,9 +516,8 @@ smat_status smat_simulate_multi(smat_ctx* c, uint32_t step, smat_stream_t stream
       a.work_counter = c->d_sync + dt;
       const int grid = grid_for(c, c->range_end[dt] - c->range_begin[dt], dt);
       Timed t(c, 2, stream);
-      const cudaError_t e = dt == SMAT_BF16
-          ? launch_stats_simulate_bf16(a, grid, c->cfg.noise, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT, c->rounds, stream)
-          : launch_stats_simulate_f32(a, grid, c->cfg.noise, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT, c->rounds, stream);
+      const cudaError_t e = launch_stats_simulate(a, grid, dt, c->cfg.noise, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT,
+                                                  c->rounds, c->any_inplace, stream);
       t.done();
       if (e != cudaSuccess) return cuda_fail(e, "fused statistics + forward launch");
     }
@@ -491,7 +532,8 @@ smat_status smat_simulate_multi(smat_ctx* c, uint32_t step, smat_stream_t stream
     if (a.chunk_end <= a.chunk_begin) continue;
     Timed t(c, 2, stream);
     const cudaError_t e = launch_simulate(a, grid_for(c, a.chunk_end - a.chunk_begin, dt), dt, c->cfg.noise,
-                                          c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT, c->rounds, stream);
+                                          c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT, c->rounds, c->any_inplace,
+                                          stream);
     t.done();
     if (e != cudaSuccess) return cuda_fail(e, "simulate launch");
   }
@@ -559,6 +601,35 @@ smat_status smat_swap(smat_ctx* c, int32_t* active_out) {
   return SMAT_OK;
 }
 
+smat_status smat_refill_theta0(smat_ctx* c, const void* const* h_theta0, smat_stream_t stream) {
+  if (!c) return fail(SMAT_ERR_INVALID_ARG, "ctx is NULL");
+  if (c->active != 0)
+    return fail(SMAT_ERR_STATE, "refill while the simulated storage is active: the model reads those buffers");
+  const int32_t n = (int32_t)c->desc.size();
+  if (c->any_inplace && !h_theta0) return fail(SMAT_ERR_INVALID_ARG, "h_theta0 is NULL");
+  for (int32_t k = 0; k < n; ++k) {
+    if (!(c->h_tensors[(size_t)k].flags & TF_INPLACE)) continue;
+    if (!h_theta0[k]) return fail(SMAT_ERR_INVALID_ARG, "tensor %d: h_theta0 entry is NULL", k);
+  }
+  for (int32_t k = 0; k < n; ++k) {
+    const smat_tensor_desc& d = c->desc[(size_t)k];
+    if (!(c->h_tensors[(size_t)k].flags & TF_INPLACE)) continue;
+    const cudaError_t e = cudaMemcpyAsync(d.sim, h_theta0[k], elem_size(d.dtype) * (size_t)d.numel,
+                                          cudaMemcpyHostToDevice, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "theta0 refill copy");
+  }
+  c->theta0_resident = true;
+  return SMAT_OK;
+}
+
+smat_status smat_mark_theta0_resident(smat_ctx* c) {
+  if (!c) return fail(SMAT_ERR_INVALID_ARG, "ctx is NULL");
+  if (c->active != 0)
+    return fail(SMAT_ERR_STATE, "the simulated storage is active: its buffers hold theta~");
+  c->theta0_resident = true;
+  return SMAT_OK;
+}
+
 smat_status smat_active(const smat_ctx* c, int32_t* active_out) {
   if (!c || !active_out) return fail(SMAT_ERR_INVALID_ARG, "NULL argument");
   *active_out = c->active;
@@ -588,6 +659,8 @@ smat_status smat_tensor_scalars(smat_ctx* c, uint32_t step, float* d_out, smat_s
   if (n == 0) return SMAT_OK;
   if (!d_out) return fail(SMAT_ERR_INVALID_ARG, "d_out is NULL");
   if ((uintptr_t)d_out % 4) return fail(SMAT_ERR_ALIGNMENT, "d_out not 4-byte aligned");
+  if (c->any_inplace_rel && !c->theta0_resident)
+    return fail(SMAT_ERR_STATE, "in-place sigma_rel tensors: theta0 is not resident (refill it first)");
   const smat_status st = run_scalars(c, step, true, stream);
   if (st != SMAT_OK) return st;
   const cudaError_t e = cudaMemcpyAsync(d_out, c->d_scal, sizeof(DevScalars) * n, cudaMemcpyDeviceToDevice, stream);
@@ -599,6 +672,7 @@ smat_status smat_debug_fused(smat_ctx* c, uint32_t step, const int32_t* d_items,
                              uint32_t epoch_skew, smat_stream_t stream) {
   if (!c) return fail(SMAT_ERR_INVALID_ARG, "ctx is NULL");
   if (!c->any_sigma_rel) return fail(SMAT_ERR_STATE, "context has no sigma_rel tensor");
+  if (c->any_inplace) return fail(SMAT_ERR_STATE, "test hook not available with in-place tensors");
   if (n_items < 0 || (n_items > 0 && !d_items)) return fail(SMAT_ERR_INVALID_ARG, "bad item list");
   if (c->range_end[SMAT_BF16] <= c->range_begin[SMAT_BF16]) return fail(SMAT_ERR_STATE, "no bf16 tensors");
   // items must name chunks of the bf16 range; checked on the host copy the caller passes through

@@ -1,0 +1,17 @@
+// Rows a2 + a3 (work-list launch) for bf16 parameters in lists with in-place
+// tensors (sim == theta0): the launch of smat_fused_bf16.cu instantiated
+// with the in-place path (flagged groups are recomputed whole after the chunk
+// instead of rewritten element by element, since their theta0 is still
+// needed), so the launches of other lists carry none of its code.
+#include "smat_simulate.cuh"
+
+namespace smat {
+
+cudaError_t launch_stats_simulate_inplace_bf16(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
+                                              cudaStream_t s) {
+  if (a.n_items <= 0) return cudaSuccess;
+  return rounds == 7 ? fused_run<7, DT_BF16, true>(a, grid, noise, per_elem_alpha, s)
+                     : fused_run<10, DT_BF16, true>(a, grid, noise, per_elem_alpha, s);
+}
+
+}  // namespace smat

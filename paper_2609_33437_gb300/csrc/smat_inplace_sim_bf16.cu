@@ -1,0 +1,15 @@
+// Row a3 (grid-stride launch, SMAT_FLAG_UNFUSED_STATS) for bf16 parameters in
+// lists with in-place tensors: the launch of smat_sim_bf16.cu instantiated with
+// the in-place path (see smat_inplace_bf16.cu).
+#include "smat_simulate.cuh"
+
+namespace smat {
+
+cudaError_t launch_simulate_inplace_bf16(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
+                                        cudaStream_t s) {
+  if (a.chunk_end <= a.chunk_begin) return cudaSuccess;
+  return rounds == 7 ? sim_run<7, DT_BF16, true>(a, grid, noise, per_elem_alpha, s)
+                     : sim_run<10, DT_BF16, true>(a, grid, noise, per_elem_alpha, s);
+}
+
+}  // namespace smat

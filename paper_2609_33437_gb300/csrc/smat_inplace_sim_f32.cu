@@ -1,0 +1,15 @@
+// Row a3 (grid-stride launch, SMAT_FLAG_UNFUSED_STATS) for f32 parameters in
+// lists with in-place tensors: the launch of smat_sim_f32.cu instantiated with
+// the in-place path (see smat_inplace_f32.cu).
+#include "smat_simulate.cuh"
+
+namespace smat {
+
+cudaError_t launch_simulate_inplace_f32(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
+                                        cudaStream_t s) {
+  if (a.chunk_end <= a.chunk_begin) return cudaSuccess;
+  return rounds == 7 ? sim_run<7, DT_F32, true>(a, grid, noise, per_elem_alpha, s)
+                     : sim_run<10, DT_F32, true>(a, grid, noise, per_elem_alpha, s);
+}
+
+}  // namespace smat

@@ -32,6 +32,7 @@ enum : uint32_t {
   TF_MASK = 1u,       // T = floor(p_keep 2^32) < 2^32: the mask stream is consulted
   TF_VEC = 2u,        // 32-byte aligned pointers and elem_offset % 16 == 0
   TF_SIGMA_REL = 4u,  // sigma_t from delta statistics
+  TF_INPLACE = 8u,    // sim == theta0: the forward overwrites theta0 with theta~
 };
 
 struct DevTensor {  // 80 bytes
@@ -121,7 +122,9 @@ constexpr int kMaxRanges = 2;  // one item list per parameter dtype
 cudaError_t launch_delta_stats(const KArgs& a, int grid, int dtype, cudaStream_t s);
 cudaError_t launch_scalars(const KArgs& a, int noise, int rounds, cudaStream_t s);
 cudaError_t launch_simulate(const KArgs& a, int grid, int dtype, int noise, bool per_elem_alpha,
-                            int rounds, cudaStream_t s);
+                            int rounds, bool inplace, cudaStream_t s);
+cudaError_t launch_stats_simulate(const KArgs& a, int grid, int dtype, int noise, bool per_elem_alpha,
+                                  int rounds, bool inplace, cudaStream_t s);
 cudaError_t launch_gradmap(const KArgs& a, int grid, int gdtype, bool per_elem_alpha, bool accumulate,
                            int rounds, cudaStream_t s);
 cudaError_t launch_simulate_f32(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
@@ -134,6 +137,15 @@ cudaError_t launch_stats_simulate_f32(const KArgs& a, int grid, int noise, bool 
                                       cudaStream_t s);
 cudaError_t launch_stats_simulate_bf16(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
                                        cudaStream_t s);
+// the same launches for lists with in-place tensors (smat_inplace_*.cu)
+cudaError_t launch_stats_simulate_inplace_f32(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
+                                              cudaStream_t s);
+cudaError_t launch_stats_simulate_inplace_bf16(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
+                                               cudaStream_t s);
+cudaError_t launch_simulate_inplace_f32(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
+                                        cudaStream_t s);
+cudaError_t launch_simulate_inplace_bf16(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
+                                         cudaStream_t s);
 cudaError_t launch_mask_bits(const KArgs& a, int64_t numel, int rounds, cudaStream_t s);
 cudaError_t launch_debug_philox(const uint32_t* ctr, int64_t n, const RoundKeys& key, int rounds,
                                 uint32_t* out, uint32_t* out_ref, cudaStream_t s);

@@ -1,4 +1,4 @@
-// Row a3 (forward) for bf16 parameters.
+// Row a3 (forward, grid-stride launch with SMAT_FLAG_UNFUSED_STATS) for bf16 parameters.
 #include "smat_simulate.cuh"
 
 namespace smat {
@@ -6,15 +6,8 @@ namespace smat {
 cudaError_t launch_simulate_bf16(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
                                   cudaStream_t s) {
   if (a.chunk_end <= a.chunk_begin) return cudaSuccess;
-  return rounds == 7 ? sim_run<7, DT_BF16>(a, grid, noise, per_elem_alpha, s)
-                     : sim_run<10, DT_BF16>(a, grid, noise, per_elem_alpha, s);
-}
-
-cudaError_t launch_stats_simulate_bf16(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
-                                      cudaStream_t s) {
-  if (a.n_items <= 0) return cudaSuccess;
-  return rounds == 7 ? fused_run<7, DT_BF16>(a, grid, noise, per_elem_alpha, s)
-                     : fused_run<10, DT_BF16>(a, grid, noise, per_elem_alpha, s);
+  return rounds == 7 ? sim_run<7, DT_BF16, false>(a, grid, noise, per_elem_alpha, s)
+                     : sim_run<10, DT_BF16, false>(a, grid, noise, per_elem_alpha, s);
 }
 
 int simulate_ctas_per_sm_bf16(int noise, bool per_elem_alpha, int rounds) {

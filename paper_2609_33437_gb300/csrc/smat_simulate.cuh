@@ -14,8 +14,11 @@ constexpr uint32_t kQueueTail = 2u;  // the group has a Gaussian tail element
 // (kept elements are theta itself); only used without per-element alpha.
 // Tie elements are written as dropped and Gaussian noise takes the central
 // polynomial for every element; the returned flags (kQueueTie, kQueueTail)
-// say whether some element needs the element path afterwards.
-template <int R, int DT, int NOISE, bool PE, bool IDENT, bool J0>
+// say whether some element needs the element path afterwards. A flagged
+// group of an in-place tensor (sim == theta0) is not stored at all, since its
+// theta0 is still needed; the chunk's drain recomputes it with EXACT, which
+// decides ties at once and takes the full erfinv (tail included).
+template <int R, int DT, int NOISE, bool PE, bool IDENT, bool J0, bool EXACT = false, bool IP = false>
 __device__ __forceinline__ uint32_t sim_group16(const KArgs& a, const TView& v, const Raw16<DT>& th,
                                                 const Raw16<DT>& t0, void* sim_p, int64_t i) {
   const uint64_t g0 = (uint64_t)(v.off + i);
@@ -23,7 +26,11 @@ __device__ __forceinline__ uint32_t sim_group16(const KArgs& a, const TView& v, 
   uint32_t flags = 0u;
   if (v.flags & TF_MASK) {
     const bool tie = group_keep16<R, J0>(a, v.tid, v.t_hi, g0, kw);
-    flags = (v.t_lo != 0u && tie) ? kQueueTie : 0u;
+    if (EXACT) {
+      if (v.t_lo != 0u && tie) resolve_group_ties<R, J0>(a, v.tid, v.t_hi, v.t_lo, g0, kw);
+    } else {
+      flags = (v.t_lo != 0u && tie) ? kQueueTie : 0u;
+    }
   }
   float out[16];
   float minL = 0.0f;
@@ -66,7 +73,8 @@ __device__ __forceinline__ uint32_t sim_group16(const KArgs& a, const TView& v, 
       float x0 = kept_of(kw, e0) ? kv.x : t02.x;
       float x1 = kept_of(kw, e0 + 1) ? kv.y : t02.y;
       if (NOISE != NOISE_NONE) {
-        const float2 eps = noise_group2<NOISE>(u[2 * h], u[2 * h + 1], scale2, minL);
+        const float2 eps = EXACT ? noise_of2<NOISE>(u[2 * h], u[2 * h + 1], scale2)
+                                 : noise_group2<NOISE>(u[2 * h], u[2 * h + 1], scale2, minL);
         x0 = __fadd_rn(x0, eps.x);
         x1 = __fadd_rn(x1, eps.y);
       }
@@ -74,8 +82,8 @@ __device__ __forceinline__ uint32_t sim_group16(const KArgs& a, const TView& v, 
       out[e0 + 1] = x1;
     }
   }
-  store16<DT>(sim_p, i, out);
-  if (NOISE == NOISE_GAUSSIAN && minL < -8.0f) flags |= kQueueTail;
+  if (!EXACT && NOISE == NOISE_GAUSSIAN && minL < -8.0f) flags |= kQueueTail;
+  if (!(IP && flags && (v.flags & TF_INPLACE))) store16<DT>(sim_p, i, out);
   return flags;
 }
 
@@ -155,7 +163,9 @@ struct ChunkQueue {
   int n_tail;
 };
 
-template <int R, int DT, int NOISE, bool PE, bool IDENT, bool J0>
+// IP: the launch may hold in-place tensors (a separate instantiation, so the
+// launches without any carry none of the in-place code).
+template <int R, int DT, int NOISE, bool PE, bool IDENT, bool J0, bool IP>
 __device__ __forceinline__ void sim_chunk(const KArgs& a, const TView& v, const DevTensor& T,
                                           const Chunk& ch, ChunkQueue& cq) {
   const bool vec = (v.flags & TF_VEC) != 0u;
@@ -165,7 +175,7 @@ __device__ __forceinline__ void sim_chunk(const KArgs& a, const TView& v, const 
       Raw16<DT> th, t0;
       load16<DT>(T.theta, i, th);
       load16<DT>(T.theta0, i, t0);
-      const uint32_t f = sim_group16<R, DT, NOISE, PE, IDENT, J0>(a, v, th, t0, T.sim, i);
+      const uint32_t f = sim_group16<R, DT, NOISE, PE, IDENT, J0, false, IP>(a, v, th, t0, T.sim, i);
       if (f) {
         const uint32_t entry = (((uint32_t)(i - ch.begin) >> 4) << 2) | f;
         if (f & kQueueTail)
@@ -184,20 +194,30 @@ __device__ __forceinline__ void sim_chunk(const KArgs& a, const TView& v, const 
   // the barrier also orders every thread's group stores before the rewrites
   __syncthreads();
   const int nt = cq.n_tie, nn = cq.n_tail;
+  const bool inplace = IP && (v.flags & TF_INPLACE) != 0u;
 #pragma unroll 1
   for (int k = threadIdx.x; k < nt + nn; k += kBlock) {
     const uint32_t q = (k < nt) ? cq.e[k] : cq.e[ChunkQueue::kGroups - nn + (k - nt)];
-    sim_resolve<R, DT, NOISE, PE, J0>(a, v, T, ch.begin + 16 * (int64_t)(q >> 2), q & 3u);
+    const int64_t gb = ch.begin + 16 * (int64_t)(q >> 2);
+    if (inplace) {
+      // the group was not stored: its theta0 is intact; recompute it whole
+      Raw16<DT> th, t0;
+      load16<DT>(T.theta, gb, th);
+      load16<DT>(T.theta0, gb, t0);
+      sim_group16<R, DT, NOISE, PE, IDENT, J0, true, IP>(a, v, th, t0, T.sim, gb);
+    } else {
+      sim_resolve<R, DT, NOISE, PE, J0>(a, v, T, gb, q & 3u);
+    }
   }
 }
 
-template <int R, int DT, int NOISE, bool PE, bool IDENT, bool J0>
+template <int R, int DT, int NOISE, bool PE, bool IDENT, bool J0, bool IP>
 __device__ __forceinline__ void sim_chunk_noise(const KArgs& a, const TView& v, const DevTensor& T,
                                                 const Chunk& ch, ChunkQueue& cq) {
   if (v.has_noise)
-    sim_chunk<R, DT, NOISE, PE, IDENT, J0>(a, v, T, ch, cq);
+    sim_chunk<R, DT, NOISE, PE, IDENT, J0, IP>(a, v, T, ch, cq);
   else
-    sim_chunk<R, DT, NOISE_NONE, PE, IDENT, J0>(a, v, T, ch, cq);
+    sim_chunk<R, DT, NOISE_NONE, PE, IDENT, J0, IP>(a, v, T, ch, cq);
 }
 
 // ------------------------------------------- a2 + a3 fused (sigma_rel lists) ---
@@ -239,20 +259,20 @@ __device__ __forceinline__ bool wait_ready(const KArgs& a, int t) {
 }
 
 // All threads of the CTA call this for the same chunk (it has a barrier).
-template <int R, int DT, int NOISE, bool PE>
+template <int R, int DT, int NOISE, bool PE, bool IP>
 __device__ __forceinline__ void forward_chunk(const KArgs& a, const TView& v, const DevTensor& T,
                                               const Chunk& ch, ChunkQueue& cq) {
   const bool j0 = (uint64_t)(v.off + ch.end) <= (uint64_t(1) << 34);
   if (!PE && v.c == 1.0f) {
-    if (j0) sim_chunk_noise<R, DT, NOISE, PE, true, true>(a, v, T, ch, cq);
-    else sim_chunk_noise<R, DT, NOISE, PE, true, false>(a, v, T, ch, cq);
+    if (j0) sim_chunk_noise<R, DT, NOISE, PE, true, true, IP>(a, v, T, ch, cq);
+    else sim_chunk_noise<R, DT, NOISE, PE, true, false, IP>(a, v, T, ch, cq);
   } else {
-    if (j0) sim_chunk_noise<R, DT, NOISE, PE, false, true>(a, v, T, ch, cq);
-    else sim_chunk_noise<R, DT, NOISE, PE, false, false>(a, v, T, ch, cq);
+    if (j0) sim_chunk_noise<R, DT, NOISE, PE, false, true, IP>(a, v, T, ch, cq);
+    else sim_chunk_noise<R, DT, NOISE, PE, false, false, IP>(a, v, T, ch, cq);
   }
 }
 
-template <int R, int DT, int NOISE, bool PE>
+template <int R, int DT, int NOISE, bool PE, bool IP>
 __global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 3 : 2)
     stats_simulate_kernel(const __grid_constant__ KArgs a) {
   __shared__ double sh_s[kBlock / 32];
@@ -326,14 +346,14 @@ __global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 3 : 2)
         S.c = __ldcg(&a.scal[ch.tensor].c);
         S.sigma = __ldcg(&a.scal[ch.tensor].sigma);
         S.noise_scale = __ldcg(&a.scal[ch.tensor].noise_scale);
-        forward_chunk<R, DT, NOISE, PE>(a, make_view(T, S), T, ch, s_cq);
+        forward_chunk<R, DT, NOISE, PE, IP>(a, make_view(T, S), T, ch, s_cq);
       }
     }
     __syncthreads();  // s_item, s_flag and the shared sums are reused by the next item
   }
 }
 
-template <int R, int DT, int NOISE, bool PE>
+template <int R, int DT, int NOISE, bool PE, bool IP>
 __global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 3 : 2) simulate_kernel(const __grid_constant__ KArgs a) {
   __shared__ ChunkQueue s_cq;
   for (int64_t ci = a.chunk_begin + blockIdx.x; ci < a.chunk_end; ci += gridDim.x) {
@@ -345,25 +365,25 @@ __global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 3 : 2) simula
     const Chunk ch = a.chunks[ci];
     const DevTensor& T = a.tensors[ch.tensor];
     const TView v = make_view(T, a.scal[ch.tensor]);
-    forward_chunk<R, DT, NOISE, PE>(a, v, T, ch, s_cq);
+    forward_chunk<R, DT, NOISE, PE, IP>(a, v, T, ch, s_cq);
     __syncthreads();  // every thread has read the counters before the next reset
   }
 }
 
 
-template <int R, int DT, int NOISE, bool PE>
+template <int R, int DT, int NOISE, bool PE, bool IP>
 struct FusedVariant {
   static cudaError_t run(const KArgs& a, int grid, cudaStream_t s) {
-    stats_simulate_kernel<R, DT, NOISE, PE><<<grid, kBlock, 0, s>>>(a);
+    stats_simulate_kernel<R, DT, NOISE, PE, IP><<<grid, kBlock, 0, s>>>(a);
     return cudaGetLastError();
   }
 };
 
-template <int R, int DT>
+template <int R, int DT, bool IP>
 cudaError_t fused_run(const KArgs& a, int grid, int noise, bool pe, cudaStream_t s) {
   if (noise == NOISE_GAUSSIAN)
-    return pe ? FusedVariant<R, DT, NOISE_GAUSSIAN, true>::run(a, grid, s) : FusedVariant<R, DT, NOISE_GAUSSIAN, false>::run(a, grid, s);
-  return pe ? FusedVariant<R, DT, NOISE_UNIFORM, true>::run(a, grid, s) : FusedVariant<R, DT, NOISE_UNIFORM, false>::run(a, grid, s);
+    return pe ? FusedVariant<R, DT, NOISE_GAUSSIAN, true, IP>::run(a, grid, s) : FusedVariant<R, DT, NOISE_GAUSSIAN, false, IP>::run(a, grid, s);
+  return pe ? FusedVariant<R, DT, NOISE_UNIFORM, true, IP>::run(a, grid, s) : FusedVariant<R, DT, NOISE_UNIFORM, false, IP>::run(a, grid, s);
 }
 
 template <typename Kernel>
@@ -373,30 +393,30 @@ int occupancy_of(Kernel k) {
   return v;
 }
 
-template <int R, int DT, int NOISE, bool PE>
+template <int R, int DT, int NOISE, bool PE, bool IP>
 struct SimVariant {
   static int occ() {
-    static int v = occupancy_of(simulate_kernel<R, DT, NOISE, PE>);
+    static int v = occupancy_of(simulate_kernel<R, DT, NOISE, PE, IP>);
     return v;
   }
   static cudaError_t run(const KArgs& a, int grid, cudaStream_t s) {
-    simulate_kernel<R, DT, NOISE, PE><<<grid, kBlock, 0, s>>>(a);
+    simulate_kernel<R, DT, NOISE, PE, IP><<<grid, kBlock, 0, s>>>(a);
     return cudaGetLastError();
   }
 };
 
-template <int R, int DT>
+template <int R, int DT, bool IP>
 cudaError_t sim_run(const KArgs& a, int grid, int noise, bool pe, cudaStream_t s) {
   if (noise == NOISE_GAUSSIAN)
-    return pe ? SimVariant<R, DT, NOISE_GAUSSIAN, true>::run(a, grid, s) : SimVariant<R, DT, NOISE_GAUSSIAN, false>::run(a, grid, s);
-  return pe ? SimVariant<R, DT, NOISE_UNIFORM, true>::run(a, grid, s) : SimVariant<R, DT, NOISE_UNIFORM, false>::run(a, grid, s);
+    return pe ? SimVariant<R, DT, NOISE_GAUSSIAN, true, IP>::run(a, grid, s) : SimVariant<R, DT, NOISE_GAUSSIAN, false, IP>::run(a, grid, s);
+  return pe ? SimVariant<R, DT, NOISE_UNIFORM, true, IP>::run(a, grid, s) : SimVariant<R, DT, NOISE_UNIFORM, false, IP>::run(a, grid, s);
 }
 
 template <int R, int DT>
 int sim_occ(int noise, bool pe) {
   if (noise == NOISE_GAUSSIAN)
-    return pe ? SimVariant<R, DT, NOISE_GAUSSIAN, true>::occ() : SimVariant<R, DT, NOISE_GAUSSIAN, false>::occ();
-  return pe ? SimVariant<R, DT, NOISE_UNIFORM, true>::occ() : SimVariant<R, DT, NOISE_UNIFORM, false>::occ();
+    return pe ? SimVariant<R, DT, NOISE_GAUSSIAN, true, false>::occ() : SimVariant<R, DT, NOISE_GAUSSIAN, false, false>::occ();
+  return pe ? SimVariant<R, DT, NOISE_UNIFORM, true, false>::occ() : SimVariant<R, DT, NOISE_UNIFORM, false, false>::occ();
 }
 
 }  // namespace

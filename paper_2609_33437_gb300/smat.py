@@ -85,6 +85,8 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
     L.smat_mask_bits.argtypes = [P, U32, I32, P, P]
     L.smat_tensor_scalars.argtypes = [P, U32, P, P]
     L.smat_destroy.argtypes = [P]
+    L.smat_refill_theta0.argtypes = [P, P, P]
+    L.smat_mark_theta0_resident.argtypes = [P]
     L.smat_debug_philox.argtypes = [P, I64, U64, I32, P, P, P]
     L.smat_debug_noise_unit.argtypes = [P, I64, I32, P, P]
     L.smat_poll_errors.argtypes = [P, P, ctypes.POINTER(I32)]
@@ -100,7 +102,8 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
     L.smat_abi_version.restype = I32
     for name in ("smat_init", "smat_simulate_multi", "smat_grad_map_multi", "smat_swap", "smat_active",
                  "smat_mask_bits", "smat_tensor_scalars", "smat_destroy", "smat_debug_philox", "smat_debug_noise_unit",
-                 "smat_poll_errors", "smat_debug_fused", "smat_timing_enable", "smat_timing_read"):
+                 "smat_poll_errors", "smat_debug_fused", "smat_timing_enable", "smat_timing_read",
+                 "smat_refill_theta0", "smat_mark_theta0_resident"):
         getattr(L, name).restype = I32
     _lib = L
     return L
@@ -155,8 +158,9 @@ class SmatSession:
         for k in range(n):
             th, t0, sm = thetas[k], theta0s[k], sims[k]
             for t in (th, t0, sm):
-                if not t.is_cuda or not t.is_contiguous():
-                    raise ValueError(f"tensor {k}: must be a contiguous CUDA tensor")
+                # theta0 may live in pinned host memory: the kernels read it there
+                if not t.is_contiguous() or not (t.is_cuda or (t is t0 and t.is_pinned())):
+                    raise ValueError(f"tensor {k}: must be a contiguous CUDA tensor (theta0: or pinned host)")
             if th.dtype != t0.dtype or th.dtype != sm.dtype or th.numel() != t0.numel() or th.numel() != sm.numel():
                 raise ValueError(f"tensor {k}: theta / theta0 / sim differ in dtype or numel")
             d = descs[k]
@@ -225,6 +229,25 @@ class SmatSession:
         a = ctypes.c_int32()
         check("smat_active", self._L.smat_active(self._ctx, ctypes.byref(a)))
         return a.value
+
+    # -- in-place mode (a tensor passed with sim == theta0) --------------------
+    def refill_theta0(self, host_theta0s: Sequence[Optional[torch.Tensor]],
+                      stream: Optional[torch.cuda.Stream] = None):
+        """Copy theta0 from host tensors (pinned for an asynchronous copy) back
+        into the sim buffers of the in-place tensors; other entries may be None."""
+        if len(host_theta0s) != self.n:
+            raise ValueError("one entry per tensor")
+        ptrs = (ctypes.c_void_p * max(self.n, 1))()
+        for k, h in enumerate(host_theta0s):
+            if h is not None:
+                if h.is_cuda or not h.is_contiguous() or h.numel() != self.numels[k]:
+                    raise ValueError(f"tensor {k}: host theta0 must be a contiguous CPU tensor of the same size")
+                ptrs[k] = h.data_ptr()
+        self._hkeep = list(host_theta0s)  # the copies read them asynchronously
+        check("smat_refill_theta0", self._L.smat_refill_theta0(self._ctx, ptrs, _stream_handle(stream)))
+
+    def mark_theta0_resident(self):
+        check("smat_mark_theta0_resident", self._L.smat_mark_theta0_resident(self._ctx))
 
     # -- test hooks ----------------------------------------------------------
     def mask_bits(self, step: int, k: int, stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:

@@ -78,6 +78,20 @@ def test_workspace_size_scales_with_chunks(L):
     assert L.smat_workspace_bytes(None, 0, ctypes.byref(cfg())) >= 0
 
 
+def test_inplace_accepted_partial_overlap_rejected(L):
+    """sim == theta0 is the in-place mode (Sec. 4.3); any other overlap of sim
+    with theta0, or any overlap with theta, is rejected."""
+    d = desc(4096)
+    d.sim = d.theta0
+    assert ws_bytes(L, [d], cfg()) > 0
+    d.sim = d.theta0 + 64
+    assert ws_bytes(L, [d], cfg()) == 0
+    d.sim = d.theta
+    assert ws_bytes(L, [d], cfg()) == 0
+    assert L.smat_refill_theta0(None, None, None) == 1
+    assert L.smat_mark_theta0_resident(None) == 1
+
+
 def test_chunk_size_rule_and_override(L):
     """Automatic chunk size: the largest power of two cs in [2^12, 2^18] with
     cs^2 / 64 <= total elements; the override forces 2^k. The chunk
