@@ -77,6 +77,8 @@ def parse():
     ap.add_argument("--sweep", metavar="PATH", default=None,
                     help="run the flat-tensor sweep, one JSON line per point to PATH")
     ap.add_argument("--sweep-max-log2n", type=int, default=32)
+    ap.add_argument("--schedule", action="store_true",
+                    help="training-loop overhead of periodic SMAT (Sec. 4.3) over plain fine-tuning, synthetic model")
     return ap.parse_args()
 
 
@@ -568,12 +570,111 @@ def run_sweep(args):
     return 0
 
 
+def run_schedule(args, d=4096, layers=8, tokens=8192, period=4, steps=32, warmup=4, rounds=3):
+    """Training-loop overhead of the periodic schedule (Sec. 4.3: t = 4, one
+    simulated-loss step per period) over plain fine-tuning, on a synthetic
+    bf16 MLP stack (layers x [d -> 4d -> d] with residuals, about 1.07e9
+    parameters) with fused AdamW (weight decay 1e-3) and random tokens: the
+    paper's method settings (uniform Perturb, drop probability 0.5 on the
+    matrices, global alpha ~ U[0.3, 1)). Three loops of `steps` steps each:
+    plain, SMAT with theta0 in HBM, SMAT in-place with theta0 in pinned host
+    memory (refilled on a side stream during the ordinary steps). The three
+    loops run `rounds` times interleaved (clocks and power drift between
+    runs); the median of each is reported, with the clocks seen."""
+    from paper_2609_33437_gb300 import smat as S
+    from paper_2609_33437_gb300.schedule import PeriodicSmat
+    S.load_library()
+    dev = torch.device("cuda")
+
+    class Block(torch.nn.Module):
+        def __init__(self):
+            super().__init__()
+            self.up = torch.nn.Linear(d, 4 * d)
+            self.down = torch.nn.Linear(4 * d, d)
+
+        def forward(self, x):
+            return x + self.down(torch.nn.functional.gelu(self.up(x)))
+
+    def build():
+        torch.manual_seed(0)
+        return torch.nn.Sequential(*[Block() for _ in range(layers)]).to(device=dev, dtype=torch.bfloat16)
+
+    x = torch.randn(tokens, d, device=dev, dtype=torch.bfloat16)
+
+    def run(mode):
+        model = build()
+        ps = list(model.parameters())
+        opt = torch.optim.AdamW(ps, lr=1e-5, weight_decay=1e-3, fused=True)
+        sched = None
+        if mode != "ft":
+            theta0 = [p.detach().clone() for p in ps]
+            keeps = [0.5 if p.dim() == 2 else 1.0 for p in ps]
+            kw = dict(seed=1, alpha_min=0.3, alpha_max=1.0, alpha_mode=S.SMAT_ALPHA_GLOBAL,
+                      noise=S.SMAT_NOISE_UNIFORM, period=period)
+            if mode == "smat":
+                sched = PeriodicSmat(ps, keeps, [1e-4] * len(ps), theta0=theta0, **kw)
+            else:
+                sched = PeriodicSmat(ps, keeps, [1e-4] * len(ps), host_theta0=[t.cpu().pin_memory() for t in theta0],
+                                     **kw)
+                del theta0
+
+        def one(step):
+            if sched:
+                sched.before_forward(step)
+            model(x).float().square().mean().backward()
+            if sched:
+                sched.after_backward(step)
+            opt.step()
+            opt.zero_grad(set_to_none=False)
+
+        for s in range(warmup):
+            one(s)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for s in range(warmup, warmup + steps):
+            one(s)
+        if sched is not None and sched.refilled is not None:
+            torch.cuda.current_stream().wait_event(sched.refilled)
+        e1.record()
+        torch.cuda.synchronize()
+        n = sum(p.numel() for p in ps)
+        if sched:
+            sched.close()
+        del model, opt, sched
+        torch.cuda.empty_cache()
+        return e0.elapsed_time(e1) / steps, n
+
+    clocks = None if args.no_clocks else ClockSampler(torch.cuda.current_device())
+    if clocks:
+        clocks.mark()
+    times = {"ft": [], "smat": [], "inplace": []}
+    n = 0
+    for _ in range(rounds):
+        for mode in times:
+            t, n = run(mode)
+            times[mode].append(t)
+    if clocks:
+        clocks.mark()
+    clk = clocks.stop() if clocks else None
+    ft, smat, inpl = (statistics.median(times[m]) for m in ("ft", "smat", "inplace"))
+    print(json.dumps({"schedule": "periodic SMAT, t = %d" % period, "params": n, "tokens_per_step": tokens,
+                      "model": f"{layers} x MLP block d={d} (bf16, residual), fused AdamW",
+                      "ft_ms_per_step": ft, "smat_ms_per_step": smat, "smat_inplace_ms_per_step": inpl,
+                      "overhead_pct": 100.0 * (smat - ft) / ft, "overhead_inplace_pct": 100.0 * (inpl - ft) / ft,
+                      "speed_vs_ft": ft / smat, "speed_vs_ft_inplace": ft / inpl,
+                      "runs_ms_per_step": times, "steps": steps, "warmup": warmup, "clocks": clk}))
+    return 0
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
     if args.sweep:
         return run_sweep(args)
+    if args.schedule:
+        return run_schedule(args)
     return run_smat(args)
 
 
