@@ -18,7 +18,7 @@ from . import build as _build
 
 F32, BF16 = 0, 1
 ALPHA_GLOBAL, ALPHA_PER_TENSOR, ALPHA_PER_ELEMENT = 0, 1, 2
-NOISE_UNIFORM, NOISE_GAUSSIAN = 0, 1
+NOISE_UNIFORM, NOISE_GAUSSIAN, NOISE_LAPLACE = 0, 1, 2
 S_MASK, S_NOISE, S_ALPHA_E, S_ALPHA_T, S_MASK_LO = 0, 1, 2, 3, 4
 GLOBAL_ALPHA_ID = 0x0FFFFFFF
 
@@ -58,12 +58,14 @@ def lib():
         L.orc_gradmap_at.argtypes = [P, P, ctypes.c_int32, ctypes.c_int32, P, ctypes.c_int64, P, P, P]
         L.orc_mask_bits.argtypes = [P, P, P]
         L.orc_gauss_z.argtypes = [P, P, P, ctypes.c_int64, P]
+        L.orc_noise_z.argtypes = [P, P, P, ctypes.c_int64, P]
+        L.orc_laplace.argtypes = [P, ctypes.c_int64, P]
         L.orc_simulate_f64.argtypes = [P, P, ctypes.c_float, P, P, P]
         L.orc_gradmap_f64.argtypes = [P, P, P, P]
         for name in ("orc_philox", "orc_stream_words", "orc_f32_to_bf16", "orc_erfinv", "orc_scalars",
                      "orc_delta_stats", "orc_simulate", "orc_simulate_at", "orc_gradmap",
                      "orc_gradmap_at", "orc_mask_bits", "orc_gauss_z", "orc_simulate_f64",
-                     "orc_gradmap_f64"):
+                     "orc_gradmap_f64", "orc_noise_z", "orc_laplace"):
             getattr(L, name).restype = None
         _lib = L
     return _lib
@@ -117,6 +119,14 @@ def erfinv(v):
     v = _c(v, np.float64).ravel()
     out = np.zeros(v.shape[0], np.float64)
     lib().orc_erfinv(_p(v), v.shape[0], _p(out))
+    return out
+
+
+def laplace(v):
+    """-sign(v) ln(1 - |v|) in double (the Laplace inverse-CDF transform)."""
+    v = _c(v, np.float64).ravel()
+    out = np.zeros(v.shape[0], np.float64)
+    lib().orc_laplace(_p(v), v.shape[0], _p(out))
     return out
 
 
@@ -202,6 +212,14 @@ def gauss_z(cfg, t, gidx):
     g = _c(gidx, np.uint64)
     out = np.zeros(g.shape[0], np.float64)
     lib().orc_gauss_z(ctypes.byref(cfg), ctypes.byref(t), _p(g), g.shape[0], _p(out))
+    return out
+
+
+def noise_z(cfg, t, gidx):
+    """Unit-variance variates of the elements' noise under the config's law."""
+    g = _c(gidx, np.uint64)
+    out = np.zeros(g.shape[0], np.float64)
+    lib().orc_noise_z(ctypes.byref(cfg), ctypes.byref(t), _p(g), g.shape[0], _p(out))
     return out
 
 

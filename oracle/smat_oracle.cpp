@@ -39,6 +39,10 @@
 //     uniform   eps = fl(sqrt3 sigma) * sym24(u)
 //     Gaussian  eps = fl(sqrt2 sigma) * fl(erfinv(sym24(u)))  (inverse-CDF transform:
 //               sqrt2 erfinv(v) is N(0, 1) for v uniform on (-1, 1))
+//     Laplace   eps = fl(sigma / sqrt2) * fl(-sign(v) ln(1 - |v|)), v = sym24(u)
+//               (inverse-CDF transform: -sign(v) ln(1 - |v|) is Laplace(0, 1),
+//               variance 2, for v uniform on (-1, 1); the scale sigma / sqrt2 gives
+//               RMS sigma, the matched-RMS comparison of Sec. 4.1 "Perturb")
 //   Alpha:  per tensor  alpha = fma(amax - amin, u01(W(ALPHA_T, t_a, 0)[0]), amin)
 //           t_a = 0x0FFFFFFF (one alpha for all tensors) or the tensor id;
 //           per element alpha = fma(amax - amin, u01(W(ALPHA_E, tid, gidx >> 2)[gidx & 3]), amin)
@@ -89,7 +93,7 @@ enum { S_MASK = 0, S_NOISE = 1, S_ALPHA_E = 2, S_ALPHA_T = 3, S_MASK_LO = 4 };
 const uint32_t kGlobalAlphaId = 0x0FFFFFFFu;
 
 enum { ALPHA_GLOBAL = 0, ALPHA_PER_TENSOR = 1, ALPHA_PER_ELEMENT = 2 };
-enum { NOISE_UNIFORM = 0, NOISE_GAUSSIAN = 1 };
+enum { NOISE_UNIFORM = 0, NOISE_GAUSSIAN = 1, NOISE_LAPLACE = 2 };
 enum { DT_F32 = 0, DT_BF16 = 1 };
 
 }  // namespace
@@ -102,7 +106,7 @@ struct OrcConfig {
   uint32_t step;
   int32_t rounds;      // Philox rounds (10 by default)
   int32_t alpha_mode;  // ALPHA_GLOBAL / ALPHA_PER_TENSOR / ALPHA_PER_ELEMENT
-  int32_t noise;       // NOISE_UNIFORM / NOISE_GAUSSIAN
+  int32_t noise;       // NOISE_UNIFORM / NOISE_GAUSSIAN / NOISE_LAPLACE
   float alpha_min;
   float alpha_max;
 };
@@ -180,7 +184,7 @@ struct Scalars {
   float c;            // alpha * inv_keep
   uint64_t T;         // keep threshold on the 32-bit mask uniform
   float sigma;        // Perturb RMS for this call
-  float noise_scale;  // fl(sqrt3 sigma) (uniform) or fl(sqrt2 sigma) (Gaussian)
+  float noise_scale;  // fl(sqrt3 sigma) (uniform), fl(sqrt2 sigma) (Gaussian), fl(sigma / sqrt2) (Laplace)
 };
 
 // Population mean and centred second moment of delta = theta - theta0 (each
@@ -228,7 +232,8 @@ Scalars make_scalars(const OrcConfig& cfg, const OrcTensor& t, float sigma) {
   s.c = s.alpha * s.inv_keep;
   s.T = (uint64_t)std::floor((double)t.keep_prob * 4294967296.0);
   s.sigma = sigma;
-  s.noise_scale = (float)(std::sqrt(cfg.noise == NOISE_UNIFORM ? 3.0 : 2.0) * (double)sigma);
+  s.noise_scale = (float)(std::sqrt(cfg.noise == NOISE_UNIFORM ? 3.0 : cfg.noise == NOISE_GAUSSIAN ? 2.0 : 0.5) *
+                          (double)sigma);
   return s;
 }
 
@@ -289,6 +294,12 @@ uint32_t noise_field(const OrcConfig& cfg, const OrcTensor& t, uint64_t gidx) {
 float sym24(uint32_t u24) { return (float)(2 * (int32_t)u24 + 1 - (1 << 24)) * kTwoPow24Inv; }
 double sym24_d(uint32_t u24) { return (double)(2 * (int64_t)u24 + 1 - (1 << 24)) * 0x1p-24; }
 
+// Laplace(0, 1) variate of v in (-1, 1) by the inverse CDF: -sign(v) ln(1 - |v|).
+double laplace_d(double v) {
+  const double z = -std::log1p(-std::fabs(v));
+  return v < 0.0 ? -z : z;
+}
+
 // Unit-variance normal variate of element gidx: sqrt2 erfinv(sym24(u)).
 double gauss_z(const OrcConfig& cfg, const OrcTensor& t, uint64_t gidx) {
   return std::sqrt(2.0) * erfinv_d(sym24_d(noise_field(cfg, t, gidx)));
@@ -297,6 +308,7 @@ double gauss_z(const OrcConfig& cfg, const OrcTensor& t, uint64_t gidx) {
 float noise_eps(const OrcConfig& cfg, const OrcTensor& t, const Scalars& s, uint64_t gidx) {
   const uint32_t u = noise_field(cfg, t, gidx);
   if (cfg.noise == NOISE_UNIFORM) return s.noise_scale * sym24(u);
+  if (cfg.noise == NOISE_LAPLACE) return s.noise_scale * (float)laplace_d(sym24_d(u));
   return s.noise_scale * (float)erfinv_d(sym24_d(u));
 }
 
@@ -347,6 +359,23 @@ void orc_f32_to_bf16(const float* x, int64_t n, uint16_t* out) {
 // erfinv in double (the Gaussian transform's definition), for its pin.
 void orc_erfinv(const double* v, int64_t n, double* out) {
   for (int64_t i = 0; i < n; ++i) out[i] = erfinv_d(v[i]);
+}
+
+// The Laplace transform -sign(v) ln(1 - |v|) in double, for its pins.
+void orc_laplace(const double* v, int64_t n, double* out) {
+  for (int64_t i = 0; i < n; ++i) out[i] = laplace_d(v[i]);
+}
+
+// Unit-variance variate of each element's noise under the config's law:
+// sqrt3 sym24(u) (uniform), sqrt2 erfinv(sym24(u)) (Gaussian),
+// laplace(sym24(u)) / sqrt2 (Laplace).
+void orc_noise_z(const OrcConfig* cfg, const OrcTensor* t, const uint64_t* gidx, int64_t n, double* z) {
+  for (int64_t k = 0; k < n; ++k) {
+    const double v = sym24_d(noise_field(*cfg, *t, gidx[k]));
+    z[k] = cfg->noise == NOISE_UNIFORM    ? std::sqrt(3.0) * v
+           : cfg->noise == NOISE_GAUSSIAN ? std::sqrt(2.0) * erfinv_d(v)
+                                          : laplace_d(v) / std::sqrt(2.0);
+  }
 }
 
 // Per-call scalars: out = {alpha, inv_keep, c, T, sigma_t, noise_scale}.
@@ -452,6 +481,8 @@ void orc_simulate_f64(const OrcConfig* cfg, const OrcTensor* t, float sigma_t, c
       const uint32_t u = noise_field(*cfg, *t, gidx);
       if (cfg->noise == NOISE_UNIFORM)
         x += (double)s.noise_scale * (double)sym24(u);
+      else if (cfg->noise == NOISE_LAPLACE)
+        x += (double)s.noise_scale * laplace_d(sym24_d(u));
       else
         x += (double)s.noise_scale * erfinv_d(sym24_d(u));
     }

@@ -44,6 +44,8 @@ def main():
                                                alpha_mode=O.ALPHA_GLOBAL, alpha_min=0.3),
              O.tensor(3, n, O.BF16, keep_prob=0.7, sigma_rel=0.1), O.f32_to_bf16(th), O.f32_to_bf16(t0),
              O.f32_to_bf16(gs), O.BF16),
+        case("f32_laplace_per_tensor", O.config(seed=11, step=5, noise=O.NOISE_LAPLACE, alpha_min=0.3),
+             O.tensor(6, n, O.F32, keep_prob=0.7, sigma=2e-3), th, t0, gs, O.F32),
     ]
     doc = {"about": "CPU-oracle outputs on fixed inputs; regression guard for the oracle "
                     "(written by tests/golden/make_golden.py, oracle/ only)",

@@ -350,6 +350,55 @@ def test_gaussian_z_matches_noise_of_simulate():
     assert np.allclose(eps, zz, rtol=3 * 2.0**-24, atol=0)
 
 
+def test_laplace_transform_closed_forms():
+    """Laplace inverse-CDF transform z(v) = -sign(v) ln(1 - |v|): z(+-1/2) =
+    +-ln 2, z(1 - 2^-k) = k ln 2 (both exact in double), z(0) = 0, exactly odd
+    and strictly increasing over the noise grid sym24(u)."""
+    k = np.arange(1, 25)
+    v = np.concatenate([[0.5, -0.5, 0.0], 1 - 2.0**-k])
+    z = O.laplace(v)
+    assert z[0] == math.log(2) and z[1] == -math.log(2) and z[2] == 0.0
+    assert np.allclose(z[3:], k * math.log(2), rtol=1e-15, atol=0)
+    u = np.arange(0, 1 << 24, 4099, dtype=np.int64)
+    g = (2 * u + 1 - (1 << 24)).astype(np.float64) * 2.0**-24
+    zg = O.laplace(g)
+    assert np.array_equal(O.laplace(-g), -zg)
+    assert np.all(np.diff(zg) > 0)
+
+
+def test_laplace_law_on_the_noise_grid():
+    """Over all 2^24 values of sym24(u), z(v) is Laplace(0, 1): its CDF is
+    within the grid's 2^-24 steps of 1/2 e^x (x < 0) / 1 - 1/2 e^-x, its mean
+    is 0 and its variance 2 (matched RMS: eps = (sigma / sqrt2) z has variance
+    sigma^2)."""
+    u = np.arange(1 << 24, dtype=np.int64)
+    v = (2 * u + 1 - (1 << 24)).astype(np.float64) * 2.0**-24
+    z = O.laplace(v)  # increasing in u
+    x = np.array([-6.0, -2.0, -0.5, -0.1, 0.0, 0.1, 0.5, 2.0, 6.0])
+    emp = np.searchsorted(z, x, side="right") / z.size
+    cdf = np.where(x < 0, 0.5 * np.exp(x), 1 - 0.5 * np.exp(-x))
+    assert np.max(np.abs(emp - cdf)) <= 2.0**-23
+    assert abs(z.mean()) < 1e-12
+    assert abs(z.var() - 2.0) < 1e-4
+
+
+def test_laplace_noise_law_in_simulate():
+    """Laplace Perturb through the full forward: RMS sigma, the Laplace
+    kurtosis 6 (uniform: 1.8, Gaussian: 3), KS against Laplace(0, 1/sqrt2) of
+    eps / sigma, and the unit variates of noise_z match eps / sigma."""
+    n, sigma = 200_000, 1e-4
+    t = O.tensor(8, n, keep_prob=0.0, sigma=sigma)
+    zero = np.zeros(n, np.float32)
+    cfg = O.config(seed=6, noise=O.NOISE_LAPLACE)
+    eps = O.simulate(cfg, t, zero, zero).astype(np.float64) / sigma
+    assert abs(eps.var() - 1) < 5 * math.sqrt(5.0 / n)
+    kurt = np.mean(eps**4) / eps.var() ** 2
+    assert abs(kurt - 6.0) < 0.3
+    assert stats.kstest(eps, "laplace", args=(0.0, 1 / math.sqrt(2))).pvalue > 1e-4
+    z = O.noise_z(cfg, t, np.arange(n))
+    assert np.allclose(eps, z, rtol=4 * 2.0**-24, atol=1e-12)
+
+
 # ------------------------------------------- Prop. moments (App. C) ---
 
 def test_state_moments_proposition():
