@@ -63,7 +63,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["smat", "reference"], default="smat")
     ap.add_argument("--workload", default="llama_7b", choices=["llama_7b", "dec_0p5b", "vl_7b", "tiny_flat"])
-    ap.add_argument("--noise", choices=["gaussian", "uniform"], default="gaussian")
+    ap.add_argument("--noise", choices=["gaussian", "uniform", "laplace"], default="gaussian")
     ap.add_argument("--scale", type=int, default=0, help="cut the list to about this many elements (profiling)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -82,13 +82,17 @@ def parse():
     return ap.parse_args()
 
 
+NOISE_CODE = {"uniform": 0, "gaussian": 1, "laplace": 2}
+NOISE_NAME = {v: k for k, v in NOISE_CODE.items()}
+
+
 def workload(args) -> W.Workload:
     if args.workload == "llama_7b":
-        w = W.llama_7b(noise=1 if args.noise == "gaussian" else 0)
+        w = W.llama_7b(noise=NOISE_CODE[args.noise])
     else:
         w = W.WORKLOADS[args.workload]()
-        if args.noise == "uniform":
-            w.noise = 0
+        if args.noise != "gaussian":
+            w.noise = NOISE_CODE[args.noise]
     if args.scale:
         w = W.scaled(w, args.scale)
     return w
@@ -286,7 +290,7 @@ def run_reference(args):
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
            "data": "synthetic", "params_per_s": tot_n / tot_s,
            "config": {"workload": w.name, "elements_per_step_sample": tot_n // args.steps,
-                      "noise": "gaussian" if w.noise == 1 else "uniform"},
+                      "noise": NOISE_NAME[w.noise]},
            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                             "sample": f"each step: {sample} (single-threaded C++ oracle, forward + gradient map)"},
            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -452,7 +456,7 @@ def run_smat(args):
                "config": {"workload": w.name, "tensors": len(w.tensors), "elements": w.numel,
                           "param_dtype": "bf16" if w.dtype == W.BF16 else "f32",
                           "grad_dtype": "bf16" if w.gdtype == W.BF16 else "f32",
-                          "noise": "gaussian" if w.noise == 1 else "uniform", "alpha": f"per-tensor U[{w.alpha_min}, {w.alpha_max})",
+                          "noise": NOISE_NAME[w.noise], "alpha": f"per-tensor U[{w.alpha_min}, {w.alpha_max})",
                           "philox_rounds": args.philox_rounds,
                           "bytes_per_step": bytes_step, "l2": "inputs larger than L2 (no flush needed)",
                           "theta0": args.theta0,

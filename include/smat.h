@@ -65,8 +65,12 @@ typedef enum {
 
 typedef enum { SMAT_F32 = 0, SMAT_BF16 = 1 } smat_dtype;
 
-/* Perturb law. Uniform on [-sqrt3 sigma, sqrt3 sigma] is the paper's (Sec. 4.1). */
-typedef enum { SMAT_NOISE_UNIFORM = 0, SMAT_NOISE_GAUSSIAN = 1 } smat_noise;
+/* Perturb law, each at RMS sigma. Uniform on [-sqrt3 sigma, sqrt3 sigma] is the
+ * paper's (Sec. 4.1); Gaussian N(0, sigma^2) and Laplace(0, sigma / sqrt2) are
+ * the alternatives its "Perturb" comparison uses (Laplace: 10 Philox rounds
+ * only). Gaussian and Laplace are inverse-CDF transforms of the same 24-bit
+ * uniform noise field. */
+typedef enum { SMAT_NOISE_UNIFORM = 0, SMAT_NOISE_GAUSSIAN = 1, SMAT_NOISE_LAPLACE = 2 } smat_noise;
 
 /* Scale granularity. The paper shares one alpha across all coordinates
  * (Sec. 4.1, App. A): SMAT_ALPHA_GLOBAL. Per tensor and per element are
@@ -213,8 +217,9 @@ smat_status smat_debug_philox(const uint32_t* d_ctr, int64_t n, uint64_t seed, i
 
 /* Test hook: the unit noise transform of n raw noise words d_words (device):
  * d_out[i] = sym(w) = (2 (w >> 8) + 1 - 2^24) 2^-24 for SMAT_NOISE_UNIFORM,
- * or erfinv(sym(w)) as the forward evaluates it for SMAT_NOISE_GAUSSIAN
- * (the forward scales these by fl(sqrt3 sigma) and fl(sqrt2 sigma)). */
+ * erfinv(sym(w)) as the forward evaluates it for SMAT_NOISE_GAUSSIAN, or
+ * -sign(v) ln(1 - |v|), v = sym(w), for SMAT_NOISE_LAPLACE (the forward scales
+ * these by fl(sqrt3 sigma), fl(sqrt2 sigma) and fl(sigma / sqrt2)). */
 smat_status smat_debug_noise_unit(const uint32_t* d_words, int64_t n, int32_t noise, float* d_out,
                                   smat_stream_t stream);
 

@@ -60,7 +60,7 @@ __global__ void scalars_kernel(const __grid_constant__ KArgs a) {
       S.c = __fmul_rn(S.alpha, T.inv_keep);
     }
     S.sigma = sigma;
-    S.noise_scale = (float)(sqrt(NOISE == NOISE_UNIFORM ? 3.0 : 2.0) * (double)sigma);
+    S.noise_scale = noise_scale_of<NOISE>(sigma);
     a.scal[t] = S;
   }
 }
@@ -123,7 +123,7 @@ __global__ void debug_noise_unit_kernel(const uint32_t* words, int64_t n, int no
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * blockDim.x) {
     const float x = sym24(words[i] >> 8);
-    out[i] = (noise == NOISE_GAUSSIAN) ? erfinv_poly(x) : x;
+    out[i] = (noise == NOISE_GAUSSIAN) ? erfinv_poly(x) : (noise == NOISE_LAPLACE) ? laplace_unit(x) : x;
   }
 }
 
@@ -132,6 +132,9 @@ __global__ void debug_noise_unit_kernel(const uint32_t* words, int64_t n, int no
 
 cudaError_t launch_simulate(const KArgs& a, int grid, int dtype, int noise, bool per_elem_alpha,
                             int rounds, bool inplace, cudaStream_t s) {
+  if (noise == NOISE_LAPLACE)  // built for 10 rounds (the host refuses 7 with Laplace)
+    return dtype == DT_BF16 ? launch_laplace_bf16(a, grid, false, per_elem_alpha, inplace, s)
+                            : launch_laplace_f32(a, grid, false, per_elem_alpha, inplace, s);
   if (inplace)
     return dtype == DT_BF16 ? launch_simulate_inplace_bf16(a, grid, noise, per_elem_alpha, rounds, s)
                             : launch_simulate_inplace_f32(a, grid, noise, per_elem_alpha, rounds, s);
@@ -141,6 +144,9 @@ cudaError_t launch_simulate(const KArgs& a, int grid, int dtype, int noise, bool
 
 cudaError_t launch_stats_simulate(const KArgs& a, int grid, int dtype, int noise, bool per_elem_alpha,
                                   int rounds, bool inplace, cudaStream_t s) {
+  if (noise == NOISE_LAPLACE)
+    return dtype == DT_BF16 ? launch_laplace_bf16(a, grid, true, per_elem_alpha, inplace, s)
+                            : launch_laplace_f32(a, grid, true, per_elem_alpha, inplace, s);
   if (inplace)
     return dtype == DT_BF16 ? launch_stats_simulate_inplace_bf16(a, grid, noise, per_elem_alpha, rounds, s)
                             : launch_stats_simulate_inplace_f32(a, grid, noise, per_elem_alpha, rounds, s);
@@ -166,9 +172,11 @@ cudaError_t launch_scalars(const KArgs& a, int noise, int rounds, cudaStream_t s
   if (a.n_tensors <= 0) return cudaSuccess;
   if (rounds == 7) {
     if (noise == NOISE_GAUSSIAN) scalars_kernel<7, NOISE_GAUSSIAN><<<a.n_tensors, 32, 0, s>>>(a);
+    else if (noise == NOISE_LAPLACE) scalars_kernel<7, NOISE_LAPLACE><<<a.n_tensors, 32, 0, s>>>(a);
     else scalars_kernel<7, NOISE_UNIFORM><<<a.n_tensors, 32, 0, s>>>(a);
   } else {
     if (noise == NOISE_GAUSSIAN) scalars_kernel<10, NOISE_GAUSSIAN><<<a.n_tensors, 32, 0, s>>>(a);
+    else if (noise == NOISE_LAPLACE) scalars_kernel<10, NOISE_LAPLACE><<<a.n_tensors, 32, 0, s>>>(a);
     else scalars_kernel<10, NOISE_UNIFORM><<<a.n_tensors, 32, 0, s>>>(a);
   }
   return cudaGetLastError();

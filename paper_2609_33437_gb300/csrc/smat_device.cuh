@@ -35,7 +35,15 @@ constexpr uint32_t kMulB = 0xCD9E8D57u;
 
 constexpr int NOISE_UNIFORM = 0;
 constexpr int NOISE_GAUSSIAN = 1;
-constexpr int NOISE_NONE = 2;  // sigma_t == 0: no add at all (chunk-level choice)
+constexpr int NOISE_LAPLACE = 2;
+constexpr int NOISE_NONE = 3;  // sigma_t == 0: no add at all (chunk-level choice)
+
+// Noise scale of each law at RMS sigma: uniform on [-sqrt3 sigma, sqrt3
+// sigma], Gaussian sqrt2 sigma erfinv(v), Laplace (sigma / sqrt2) z(v).
+template <int NOISE>
+__device__ __forceinline__ float noise_scale_of(float sigma) {
+  return (float)(sqrt(NOISE == NOISE_UNIFORM ? 3.0 : NOISE == NOISE_GAUSSIAN ? 2.0 : 0.5) * (double)sigma);
+}
 constexpr int DT_F32 = 0;
 constexpr int DT_BF16 = 1;
 
@@ -213,6 +221,13 @@ __device__ __forceinline__ float2 erfinv_poly2(float2 x) {
   return make_float2(erfinv_poly(x.x), erfinv_poly(x.y));
 }
 
+// Laplace(0, 1) variate of v in (-1, 1) by the inverse CDF, -sign(v) ln(1 -
+// |v|): 1 - |v| is exact in fp32 for every noise-grid v, and log1pf of -|v|
+// keeps full relative accuracy for small |v|.
+__device__ __forceinline__ float laplace_unit(float v) {
+  return copysignf(-log1pf(-fabsf(v)), v);
+}
+
 // The group path's erfinv of a pair: the central polynomial only (packed,
 // branch free). minL collects the smallest L = log2(1 - x^2) seen, computed
 // exactly as erfinv_poly computes it; an element with L < -8 belongs to the
@@ -240,6 +255,10 @@ template <int NOISE>
 __device__ __forceinline__ float2 noise_group2(uint32_t n0, uint32_t n1, float2 scale, float& minL) {
   if (NOISE == NOISE_UNIFORM) return mul2_rn(scale, sym2<false>(n0, n1));
   if (NOISE == NOISE_GAUSSIAN) return mul2_rn(scale, erfinv_central2(sym2<true>(n0, n1), minL));
+  if (NOISE == NOISE_LAPLACE) {
+    const float2 v = sym2<true>(n0, n1);
+    return mul2_rn(scale, make_float2(laplace_unit(v.x), laplace_unit(v.y)));
+  }
   return splat(0.0f);
 }
 
@@ -252,6 +271,10 @@ template <int NOISE>
 __device__ __forceinline__ float2 noise_of2(uint32_t n0, uint32_t n1, float2 scale) {
   if (NOISE == NOISE_UNIFORM) return mul2_rn(scale, sym2<false>(n0, n1));
   if (NOISE == NOISE_GAUSSIAN) return mul2_rn(scale, erfinv_poly2(sym2<true>(n0, n1)));
+  if (NOISE == NOISE_LAPLACE) {
+    const float2 v = sym2<true>(n0, n1);
+    return mul2_rn(scale, make_float2(laplace_unit(v.x), laplace_unit(v.y)));
+  }
   return splat(0.0f);
 }
 
@@ -259,6 +282,7 @@ template <int NOISE>
 __device__ __forceinline__ float noise_of(uint32_t u24, float scale) {
   if (NOISE == NOISE_UNIFORM) return __fmul_rn(scale, sym24(u24));
   if (NOISE == NOISE_GAUSSIAN) return __fmul_rn(scale, erfinv_poly(sym24(u24)));
+  if (NOISE == NOISE_LAPLACE) return __fmul_rn(scale, laplace_unit(sym24(u24)));
   return 0.0f;
 }
 

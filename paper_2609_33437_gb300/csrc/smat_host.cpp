@@ -84,8 +84,10 @@ smat_status check_config(const smat_config* cfg) {
   if (!cfg) return fail(SMAT_ERR_INVALID_ARG, "cfg is NULL");
   if (cfg->alpha_mode < SMAT_ALPHA_GLOBAL || cfg->alpha_mode > SMAT_ALPHA_PER_ELEMENT)
     return fail(SMAT_ERR_UNSUPPORTED, "alpha_mode %d not supported", cfg->alpha_mode);
-  if (cfg->noise != SMAT_NOISE_UNIFORM && cfg->noise != SMAT_NOISE_GAUSSIAN)
+  if (cfg->noise != SMAT_NOISE_UNIFORM && cfg->noise != SMAT_NOISE_GAUSSIAN && cfg->noise != SMAT_NOISE_LAPLACE)
     return fail(SMAT_ERR_UNSUPPORTED, "noise %d not supported", cfg->noise);
+  if (cfg->noise == SMAT_NOISE_LAPLACE && cfg->philox_rounds == 7)
+    return fail(SMAT_ERR_UNSUPPORTED, "Laplace noise is built for 10 Philox rounds");
   if (cfg->philox_rounds != 0 && cfg->philox_rounds != 7 && cfg->philox_rounds != 10)
     return fail(SMAT_ERR_UNSUPPORTED, "philox_rounds %d not supported (7 or 10)", cfg->philox_rounds);
   if (cfg->flags & ~(SMAT_FLAG_UNFUSED_STATS | SMAT_FLAG_CHUNK_LOG2_MASK))
@@ -770,7 +772,7 @@ smat_status smat_debug_noise_unit(const uint32_t* d_words, int64_t n, int32_t no
   if (n < 0) return fail(SMAT_ERR_INVALID_ARG, "n < 0");
   if (n == 0) return SMAT_OK;
   if (!d_words || !d_out) return fail(SMAT_ERR_INVALID_ARG, "NULL pointer");
-  if (noise != SMAT_NOISE_UNIFORM && noise != SMAT_NOISE_GAUSSIAN)
+  if (noise != SMAT_NOISE_UNIFORM && noise != SMAT_NOISE_GAUSSIAN && noise != SMAT_NOISE_LAPLACE)
     return fail(SMAT_ERR_UNSUPPORTED, "noise %d not supported", noise);
   const cudaError_t e = launch_debug_noise_unit(d_words, n, noise, d_out, stream);
   if (e != cudaSuccess) return cuda_fail(e, "noise transform launch");

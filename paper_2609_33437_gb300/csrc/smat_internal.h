@@ -137,6 +137,10 @@ cudaError_t launch_stats_simulate_f32(const KArgs& a, int grid, int noise, bool 
                                       cudaStream_t s);
 cudaError_t launch_stats_simulate_bf16(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
                                        cudaStream_t s);
+// Laplace noise (10 rounds; smat_laplace_*.cu): the work-list launch when
+// `fused`, else the grid-stride one; in-place instantiations when `inplace`.
+cudaError_t launch_laplace_f32(const KArgs& a, int grid, bool fused, bool per_elem_alpha, bool inplace, cudaStream_t s);
+cudaError_t launch_laplace_bf16(const KArgs& a, int grid, bool fused, bool per_elem_alpha, bool inplace, cudaStream_t s);
 // the same launches for lists with in-place tensors (smat_inplace_*.cu)
 cudaError_t launch_stats_simulate_inplace_f32(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
                                               cudaStream_t s);

@@ -326,8 +326,7 @@ __global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 3 : 2)
           }
           const float sigma = sigma_from_sums(ts, tq, T.numel, T.sigma_rel);
           a.scal[ch.tensor].sigma = sigma;
-          a.scal[ch.tensor].noise_scale =
-              (float)(sqrt(NOISE == NOISE_UNIFORM ? 3.0 : 2.0) * (double)sigma);
+          a.scal[ch.tensor].noise_scale = noise_scale_of<NOISE>(sigma);
           __threadfence();
           st_release(a.ready + ch.tensor, a.epoch);
         }

@@ -19,7 +19,7 @@ import torch
 from . import build as _build
 
 SMAT_F32, SMAT_BF16 = 0, 1
-SMAT_NOISE_UNIFORM, SMAT_NOISE_GAUSSIAN = 0, 1
+SMAT_NOISE_UNIFORM, SMAT_NOISE_GAUSSIAN, SMAT_NOISE_LAPLACE = 0, 1, 2
 SMAT_ALPHA_GLOBAL, SMAT_ALPHA_PER_TENSOR, SMAT_ALPHA_PER_ELEMENT = 0, 1, 2
 
 EXPORTED = ("smat_workspace_bytes", "smat_init", "smat_simulate_multi", "smat_grad_map_multi",

@@ -134,7 +134,8 @@ def test_init_rejects_invalid_tensor(L, bad, code):
 
 
 @pytest.mark.parametrize("bad,code", [
-    (dict(alpha_mode=3), 2), (dict(noise=2), 2), (dict(philox_rounds=8), 2),
+    (dict(alpha_mode=3), 2), (dict(noise=3), 2), (dict(philox_rounds=8), 2),
+    (dict(noise=S.SMAT_NOISE_LAPLACE, philox_rounds=7), 2),
     (dict(alpha_min=0.9, alpha_max=0.5), 1), (dict(alpha_min=float("nan")), 1),
     (dict(flags=S.SMAT_FLAG_CHUNK_LOG2(11)), 2), (dict(flags=S.SMAT_FLAG_CHUNK_LOG2(19)), 2), (dict(flags=1 << 14), 2),
     (dict(flags=2), 2),

@@ -37,7 +37,7 @@ def _bits(t):
 
 @pytest.mark.parametrize("chunk_log2", [12, 18])
 @pytest.mark.parametrize("rel", [False, True])
-@pytest.mark.parametrize("noise", [O.NOISE_UNIFORM, O.NOISE_GAUSSIAN])
+@pytest.mark.parametrize("noise", [O.NOISE_UNIFORM, O.NOISE_GAUSSIAN, O.NOISE_LAPLACE])
 @pytest.mark.parametrize("dtype", [O.BF16, O.F32])
 def test_inplace_forward_equals_two_buffer_forward(dtype, noise, rel, chunk_log2):
     w = _list(dtype, noise, rel)

@@ -59,7 +59,7 @@ def test_scaled_backbone_lists(name):
     run_and_check_full(w, steps=(0, 2))
 
 
-@pytest.mark.parametrize("noise", [O.NOISE_UNIFORM, O.NOISE_GAUSSIAN])
+@pytest.mark.parametrize("noise", [O.NOISE_UNIFORM, O.NOISE_GAUSSIAN, O.NOISE_LAPLACE])
 @pytest.mark.parametrize("alpha_mode", [O.ALPHA_GLOBAL, O.ALPHA_PER_TENSOR, O.ALPHA_PER_ELEMENT])
 @pytest.mark.parametrize("dtype", [O.F32, O.BF16])
 def test_modes_small_ragged_list(dtype, alpha_mode, noise):
@@ -73,7 +73,7 @@ def test_modes_small_ragged_list(dtype, alpha_mode, noise):
 
 
 @pytest.mark.parametrize("chunk_log2", [12, 16, 18])
-@pytest.mark.parametrize("noise", [O.NOISE_UNIFORM, O.NOISE_GAUSSIAN])
+@pytest.mark.parametrize("noise", [O.NOISE_UNIFORM, O.NOISE_GAUSSIAN, O.NOISE_LAPLACE])
 def test_forced_chunk_sizes_ragged_list(chunk_log2, noise):
     """The work-chunk size (chosen per list; forced here) changes no result:
     ragged tensors around 2^12, 2^16, 2^17 (gradient-map unit) and 2^18
