@@ -20,6 +20,7 @@ F32, BF16 = 0, 1
 ALPHA_GLOBAL, ALPHA_PER_TENSOR, ALPHA_PER_ELEMENT = 0, 1, 2
 NOISE_UNIFORM, NOISE_GAUSSIAN, NOISE_LAPLACE = 0, 1, 2
 S_MASK, S_NOISE, S_ALPHA_E, S_ALPHA_T, S_MASK_LO = 0, 1, 2, 3, 4
+MERGE_WA, MERGE_TA, MERGE_DARE_TA, MERGE_TIES = 0, 1, 2, 3
 GLOBAL_ALPHA_ID = 0x0FFFFFFF
 
 
@@ -35,6 +36,12 @@ class OrcTensor(ctypes.Structure):
                 ("numel", ctypes.c_int64), ("elem_offset", ctypes.c_int64),
                 ("keep_prob", ctypes.c_float), ("sigma", ctypes.c_float),
                 ("sigma_rel", ctypes.c_float)]
+
+
+class OrcMerge(ctypes.Structure):
+    _fields_ = [("seed", ctypes.c_uint64), ("rounds", ctypes.c_int32), ("method", ctypes.c_int32),
+                ("n_experts", ctypes.c_int32), ("gamma", ctypes.c_float), ("p_drop", ctypes.c_float),
+                ("retention", ctypes.c_float)]
 
 
 _lib = None
@@ -60,12 +67,13 @@ def lib():
         L.orc_gauss_z.argtypes = [P, P, P, ctypes.c_int64, P]
         L.orc_noise_z.argtypes = [P, P, P, ctypes.c_int64, P]
         L.orc_laplace.argtypes = [P, ctypes.c_int64, P]
+        L.orc_merge.argtypes = [P, ctypes.c_uint32, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64, P, P, P, P]
         L.orc_simulate_f64.argtypes = [P, P, ctypes.c_float, P, P, P]
         L.orc_gradmap_f64.argtypes = [P, P, P, P]
         for name in ("orc_philox", "orc_stream_words", "orc_f32_to_bf16", "orc_erfinv", "orc_scalars",
                      "orc_delta_stats", "orc_simulate", "orc_simulate_at", "orc_gradmap",
                      "orc_gradmap_at", "orc_mask_bits", "orc_gauss_z", "orc_simulate_f64",
-                     "orc_gradmap_f64", "orc_noise_z", "orc_laplace"):
+                     "orc_gradmap_f64", "orc_noise_z", "orc_laplace", "orc_merge"):
             getattr(L, name).restype = None
         _lib = L
     return _lib
@@ -248,3 +256,22 @@ def stored_to_f32(bits, dtype):
 
 def library_path():
     return os.path.abspath(_build.LIB)
+
+
+def merge(method, theta0, experts, dtype=F32, gamma=1.0, p_drop=0.0, retention=1.0, seed=0, tensor_id=0,
+          elem_offset=0, rounds=10):
+    """Eq. merged-state over the K experts (WA, TA, DARE + TA or TIES); returns
+    (theta_merge in storage form, the K TIES threshold keys)."""
+    dt = _store_dtype(dtype)
+    t0 = _c(theta0, dt).ravel()
+    ex = [_c(x, dt).ravel() for x in experts]
+    n = t0.size
+    assert all(x.size == n for x in ex)
+    K = len(ex)
+    m = OrcMerge(seed, rounds, method, K, gamma, p_drop, retention)
+    ptrs = (ctypes.c_void_p * K)(*[x.ctypes.data for x in ex])
+    out = np.zeros(n, dt)
+    thr = np.zeros(K, np.uint32)
+    lib().orc_merge(ctypes.byref(m), tensor_id, dtype, n, elem_offset, _p(t0), ctypes.cast(ptrs, ctypes.c_void_p),
+                    _p(out), _p(thr))
+    return out, thr

@@ -47,12 +47,29 @@
 //           t_a = 0x0FFFFFFF (one alpha for all tensors) or the tensor id;
 //           per element alpha = fma(amax - amin, u01(W(ALPHA_E, tid, gidx >> 2)[gidx & 3]), amin)
 //
+// Merging (the evaluation side, Eq. merged-state): theta_merge = theta0 +
+// sum_j alpha_j (.) m_j (.) Delta_j over K experts, Delta_j = theta_j - theta0
+// (one fp32 subtraction), accumulated over j = 0 .. K-1 in that order:
+//   WA    acc = fma(fl(1/K), Delta_j, acc)             (weight averaging, Sec. 3.1)
+//   TA    acc = fma(gamma, Delta_j, acc)               (Task Arithmetic, Sec. 3.1)
+//   DARE  acc = fma(c, Delta_j, acc) for kept j only,  c = fl(gamma * fl(1 / p_keep)),
+//         p_keep = fl(1 - p_drop); expert j's keep decision is the Mask stream
+//         above with step = j (same threshold rule, same Philox draws)
+//   TIES  trim: keep Delta_j where key(|Delta_j|) >= the r-th largest key of the
+//         tensor's expert j, r = ceil(retention n) (key = the bits of |x| as
+//         uint32; ties at the threshold are kept); elect s = sign of the fp32
+//         sum over j of the trimmed values; merged = the fp32 mean of the
+//         trimmed values of sign s (0 if none), acc = fl(gamma * merged)
+//   theta_merge = fl(theta0 + acc), rounded to the storage dtype.
+//
 // Build: g++ -O2 -ffp-contract=off -shared -fPIC (no fast-math: every float
 // operation below is one IEEE binary32 operation, round to nearest even).
 
+#include <algorithm>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
+#include <functional>
 #include <vector>
 
 namespace {
@@ -495,6 +512,131 @@ void orc_gradmap_f64(const OrcConfig* cfg, const OrcTensor* t, const double* gsi
   for (int64_t i = 0; i < t->numel; ++i) {
     const uint64_t gidx = (uint64_t)(t->elem_offset + i);
     out[i] = is_kept(*cfg, *t, s, gidx) ? (double)element_c(*cfg, *t, s, gidx) * gsim[i] : 0.0;
+  }
+}
+
+}  // extern "C"
+
+// ------------------------------------------------------------- merging ---
+namespace {
+
+enum { MERGE_WA = 0, MERGE_TA = 1, MERGE_DARE_TA = 2, MERGE_TIES = 3 };
+
+}  // namespace
+
+extern "C" {
+
+// Layout mirrored by the ctypes wrapper (oracle/__init__.py).
+struct OrcMerge {
+  uint64_t seed;
+  int32_t rounds;
+  int32_t method;     // MERGE_*
+  int32_t n_experts;  // K >= 1
+  float gamma;        // merging coefficient (TA, DARE, TIES)
+  float p_drop;       // DARE drop probability in [0, 1)
+  float retention;    // TIES fraction kept per expert, (0, 1]
+};
+
+}  // extern "C"
+
+namespace {
+
+uint32_t abs_key(float x) {
+  uint32_t b;
+  std::memcpy(&b, &x, 4);
+  return b & 0x7FFFFFFFu;
+}
+
+// The r-th largest key of one expert's task vector, r = ceil(retention n)
+// clamped to [1, n] (sort in descending order and index: plain, not fast).
+uint32_t orc_ties_threshold_of(const std::vector<float>& delta, double retention) {
+  const int64_t n = (int64_t)delta.size();
+  if (n == 0) return 0u;
+  int64_t r = (int64_t)std::ceil(retention * (double)n);
+  if (r < 1) r = 1;
+  if (r > n) r = n;
+  std::vector<uint32_t> keys((size_t)n);
+  for (int64_t i = 0; i < n; ++i) keys[(size_t)i] = abs_key(delta[(size_t)i]);
+  std::sort(keys.begin(), keys.end(), std::greater<uint32_t>());
+  return keys[(size_t)(r - 1)];
+}
+
+}  // namespace
+
+extern "C" {
+
+// One tensor: theta0 and the K experts (dtype storage, n elements each) into
+// out; thresholds_out (K entries, may be NULL) receives the TIES keys.
+void orc_merge(const OrcMerge* m, uint32_t tensor_id, int32_t dtype, int64_t n, int64_t elem_offset,
+               const void* theta0, const void* const* experts, void* out, uint32_t* thresholds_out) {
+  const int K = m->n_experts;
+  std::vector<std::vector<float>> delta((size_t)K, std::vector<float>((size_t)n));
+  for (int e = 0; e < K; ++e)
+    for (int64_t i = 0; i < n; ++i)
+      delta[(size_t)e][(size_t)i] = load_elem(experts[e], dtype, i) - load_elem(theta0, dtype, i);
+  std::vector<uint32_t> thr((size_t)K, 0u);
+  if (m->method == MERGE_TIES)
+    for (int e = 0; e < K; ++e) thr[(size_t)e] = orc_ties_threshold_of(delta[(size_t)e], (double)m->retention);
+  if (thresholds_out)
+    for (int e = 0; e < K; ++e) thresholds_out[e] = thr[(size_t)e];
+  // DARE: the Mask stream of Eq. smat-mask at step = expert index
+  const float keep = 1.0f - m->p_drop;
+  OrcTensor mt;
+  mt.tensor_id = tensor_id;
+  mt.dtype = dtype;
+  mt.numel = n;
+  mt.elem_offset = elem_offset;
+  mt.keep_prob = keep;
+  mt.sigma = 0.0f;
+  mt.sigma_rel = 0.0f;
+  const float inv_keep = keep > 0.0f ? (float)(1.0 / (double)keep) : 0.0f;
+  const float c_dare = m->gamma * inv_keep;
+  const float c_wa = (float)(1.0 / (double)K);
+  for (int64_t i = 0; i < n; ++i) {
+    const uint64_t gidx = (uint64_t)(elem_offset + i);
+    float acc = 0.0f;
+    if (m->method == MERGE_TIES) {
+      float sum = 0.0f;
+      for (int e = 0; e < K; ++e) {
+        const float d = delta[(size_t)e][(size_t)i];
+        if (abs_key(d) >= thr[(size_t)e]) sum = sum + d;
+      }
+      const int s = sum > 0.0f ? 1 : (sum < 0.0f ? -1 : 0);
+      float part = 0.0f;
+      int cnt = 0;
+      for (int e = 0; e < K; ++e) {
+        const float d = delta[(size_t)e][(size_t)i];
+        if (abs_key(d) < thr[(size_t)e]) continue;
+        if ((s > 0 && d > 0.0f) || (s < 0 && d < 0.0f)) {
+          part = part + d;
+          ++cnt;
+        }
+      }
+      const float merged = cnt > 0 ? part / (float)cnt : 0.0f;
+      acc = m->gamma * merged;
+    } else {
+      for (int e = 0; e < K; ++e) {
+        const float d = delta[(size_t)e][(size_t)i];
+        if (m->method == MERGE_WA) {
+          acc = std::fma(c_wa, d, acc);
+        } else if (m->method == MERGE_TA) {
+          acc = std::fma(m->gamma, d, acc);
+        } else {
+          OrcConfig cfg;
+          cfg.seed = m->seed;
+          cfg.step = (uint32_t)e;
+          cfg.rounds = m->rounds;
+          cfg.alpha_mode = ALPHA_PER_TENSOR;
+          cfg.noise = NOISE_UNIFORM;
+          cfg.alpha_min = 0.0f;
+          cfg.alpha_max = 1.0f;
+          Scalars s;
+          s.T = (uint64_t)std::floor((double)keep * 4294967296.0);
+          if (is_kept(cfg, mt, s, gidx)) acc = std::fma(c_dare, d, acc);
+        }
+      }
+    }
+    store_elem(out, dtype, i, load_elem(theta0, dtype, i) + acc);
   }
 }
 

@@ -609,3 +609,94 @@ def test_oracle_regression_fixture():
         assert sim.tolist() == c["sim_bits"], c["name"]
         assert g.tolist() == c["g_bits"], c["name"]
         assert O.mask_bits(cfg, t).tolist() == c["mask_words"], c["name"]
+
+
+# ------------------------------------------- merging (Eq. merged-state) ---
+
+def _dyadic(r, n, scale=2.0**-6):
+    """Small multiples of 2^-10: differences, sums and products by the
+    coefficients below are exact in fp32, so results equal exact rationals."""
+    return (r.integers(-64, 65, n) * scale / 16).astype(np.float32)
+
+
+def test_merge_ta_wa_closed_forms_and_identities():
+    """TA: theta0 + gamma sum_j Delta_j, WA: theta0 + (1/K) sum_j Delta_j
+    (Sec. 3.1), against exact rational arithmetic on dyadic inputs; gamma = 0
+    gives theta0; permuting the experts changes nothing (exact sums)."""
+    r = rng(30)
+    n, K = 257, 4
+    t0 = _dyadic(r, n)
+    ex = [_dyadic(r, n) for _ in range(K)]
+    exact_sum = sum(e.astype(np.float64) - t0 for e in ex)
+    ta, _ = O.merge(O.MERGE_TA, t0, ex, gamma=0.5)
+    assert np.array_equal(ta.astype(np.float64), t0 + 0.5 * exact_sum)
+    wa, _ = O.merge(O.MERGE_WA, t0, ex)
+    assert np.array_equal(wa.astype(np.float64), t0 + exact_sum / K)
+    z, _ = O.merge(O.MERGE_TA, t0, ex, gamma=0.0)
+    assert np.array_equal(z, t0)
+    perm, _ = O.merge(O.MERGE_TA, t0, ex[::-1], gamma=0.5)
+    assert np.array_equal(perm, ta)
+
+
+def test_merge_dare_masks_are_the_smat_mask_stream():
+    """DARE (Yu et al.) drops each coordinate of Delta_j with probability p and
+    rescales the rest by 1/(1-p); expert j's mask is the SMAT Mask stream at
+    step j: with one expert at a time, the kept set equals mask_bits at that
+    step, the keep rate is binomial, p = 0 is TA exactly, and the merge is
+    unbiased over seeds."""
+    r = rng(31)
+    n, K, p = 20_000, 3, 0.3
+    t0 = _dyadic(r, n)
+    ex = [_dyadic(r, n) + np.float32(1.0) for _ in range(K)]  # Delta never 0
+    for j in range(K):
+        one = [t0.copy() for _ in range(K)]
+        one[j] = ex[j]
+        out, _ = O.merge(O.MERGE_DARE_TA, t0, one, gamma=1.0, p_drop=p, seed=77, tensor_id=5)
+        kept = out != t0
+        bits = O.unpack_bits(O.mask_bits(O.config(seed=77, step=j), O.tensor(5, n, keep_prob=np.float32(1 - p))), n)
+        assert np.array_equal(kept, bits.astype(bool)), j
+        assert abs(kept.sum() - n * (1 - p)) < 5 * math.sqrt(n * p * (1 - p))
+    d0, _ = O.merge(O.MERGE_DARE_TA, t0, ex, gamma=0.7, p_drop=0.0, seed=1)
+    ta, _ = O.merge(O.MERGE_TA, t0, ex, gamma=0.7)
+    assert np.array_equal(d0, ta)
+    m = 600
+    small = [e[:64] for e in ex]
+    mean = np.mean([O.merge(O.MERGE_DARE_TA, t0[:64], small, gamma=1.0, p_drop=0.5, seed=s)[0].astype(np.float64)
+                    for s in range(m)], axis=0)
+    target = O.merge(O.MERGE_TA, t0[:64], small, gamma=1.0)[0].astype(np.float64)
+    spread = np.sqrt(sum((e[:64].astype(np.float64) - t0[:64]) ** 2 for e in ex) / m)  # sd of the mean, p = 0.5
+    assert np.all(np.abs(mean - target) < 5 * spread + 1e-6)
+
+
+def test_merge_ties_hand_example():
+    """TIES (Yadav et al.): trim, elect sign, disjoint mean, worked by hand.
+    Delta_1 = (1, -2, 3, 0.5), Delta_2 = (2, 1, -1, -0.5), Delta_3 = (-4, 1, -1,
+    0.5). No trimming: sums (-1, 0, 1, 0.5), merged (-4, 0, 3, 0.5). Retention
+    0.5 (r = 2 of 4): thresholds 2, 1, 1 (ties kept: Delta_2 keeps 2, 1, -1),
+    trimmed sums (-2, 0, 1, 0), merged (-4, 0, 3, 0)."""
+    t0 = np.zeros(4, np.float32)
+    ex = [np.array([1, -2, 3, 0.5], np.float32), np.array([2, 1, -1, -0.5], np.float32),
+          np.array([-4, 1, -1, 0.5], np.float32)]
+    out, _ = O.merge(O.MERGE_TIES, t0, ex, gamma=1.0, retention=1.0)
+    assert np.array_equal(out, np.array([-4, 0, 3, 0.5], np.float32))
+    out, thr = O.merge(O.MERGE_TIES, t0, ex, gamma=1.0, retention=0.5)
+    assert np.array_equal(out, np.array([-4, 0, 3, 0], np.float32))
+    assert np.array_equal(thr.view(np.float32), np.array([2, 1, 1], np.float32))
+    out, _ = O.merge(O.MERGE_TIES, t0 + np.float32(0.25), [e + np.float32(0.25) for e in ex], gamma=0.5,
+                     retention=1.0)
+    assert np.array_equal(out, np.array([-1.75, 0.25, 1.75, 0.5], np.float32))
+
+
+def test_merge_ties_threshold_is_the_rth_largest_magnitude():
+    """The trim threshold equals the ceil(k n)-th largest |Delta| of numpy's
+    sort, and exactly the entries at or above it survive."""
+    r = rng(32)
+    n, K = 1001, 3
+    t0 = (r.standard_normal(n) * 0.02).astype(np.float32)
+    ex = [(t0 + r.standard_normal(n).astype(np.float32) * np.float32(1e-3)).astype(np.float32) for _ in range(K)]
+    for k in (0.1, 0.3, 0.5, 1.0):
+        _, thr = O.merge(O.MERGE_TIES, t0, ex, retention=k)
+        for j in range(K):
+            d = np.abs(ex[j] - t0)
+            ref = np.sort(d)[::-1][min(n, max(1, math.ceil(k * n))) - 1]
+            assert thr.view(np.float32)[j] == ref
