@@ -77,6 +77,9 @@ def parse():
     ap.add_argument("--sweep", metavar="PATH", default=None,
                     help="run the flat-tensor sweep, one JSON line per point to PATH")
     ap.add_argument("--sweep-max-log2n", type=int, default=32)
+    ap.add_argument("--merge", choices=["wa", "ta", "dare", "ties"], default=None,
+                    help="time merging K experts of the chosen list (Eq. merged-state) instead of the SMAT step")
+    ap.add_argument("--experts", type=int, default=8)
     ap.add_argument("--schedule", action="store_true",
                     help="training-loop overhead of periodic SMAT (Sec. 4.3) over plain fine-tuning, synthetic model")
     return ap.parse_args()
@@ -671,8 +674,55 @@ def run_schedule(args, d=4096, layers=8, tokens=8192, period=4, steps=32, warmup
     return 0
 
 
+def run_merge(args):
+    """Merging K synthetic experts of the chosen list (theta_j = theta0 +
+    delta_j, delta_j ~ N(0, delta_std^2) per the list's recipe) with the given
+    method: gamma 0.3 (TA, DARE, TIES), DARE drop 0.3, TIES retention 0.5 (the
+    paper's calibrated settings, App. B). Algorithmic bytes per element: the
+    merge reads theta0 and the K experts and writes the result, (K + 2) b; TIES
+    adds three radix-select passes reading theta0 and each expert, 6 K b."""
+    from paper_2609_33437_gb300 import smat as S
+    S.load_library()
+    dev = torch.device("cuda")
+    w = workload(args)
+    K = args.experts
+    method = {"wa": S.SMAT_MERGE_WA, "ta": S.SMAT_MERGE_TA, "dare": S.SMAT_MERGE_DARE_TA, "ties": S.SMAT_MERGE_TIES}[args.merge]
+    tdt = W.torch_dtype(w.dtype)
+    t0s, exs, outs = [], [], []
+    for k, spec in enumerate(w.tensors):
+        g = torch.Generator(device=dev).manual_seed(w.data_seed * 100003 + k)
+        t0 = torch.randn(spec.numel, generator=g, device=dev) * w.theta0_std
+        ex = [(t0 + torch.randn(spec.numel, generator=g, device=dev) * w.delta_std).to(tdt) for _ in range(K)]
+        t0s.append(t0.to(tdt))
+        exs.append(ex)
+        outs.append(torch.empty(spec.numel, dtype=tdt, device=dev))
+        del t0
+    kw = dict(gamma=0.3, p_drop=0.3, retention=0.5, seed=1)
+    for _ in range(max(1, args.warmup)):
+        S.merge(t0s, exs, outs, method, **kw)
+    torch.cuda.synchronize()
+    times = []
+    for _ in range(args.steps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        S.merge(t0s, exs, outs, method, **kw)
+        e1.record()
+        e1.synchronize()
+        times.append(e0.elapsed_time(e1))
+    ms = statistics.median(times)
+    b = 2 if w.dtype == W.BF16 else 4
+    nbytes = (K + 2) * b * w.numel + (6 * K * b * w.numel if method == S.SMAT_MERGE_TIES else 0)
+    peak, peak_kind = measured_peaks()
+    print(json.dumps({"merge": args.merge, "experts": K, "workload": w.name, "elements": w.numel,
+                      "ms": ms, "gbs": nbytes / (ms * 1e-3) / 1e9, "frac_of_measured_peak": nbytes / (ms * 1e-3) / 1e9 / peak,
+                      "algorithmic_bytes": nbytes, "runs_ms": times, "settings": kw}))
+    return 0
+
+
 def main():
     args = parse()
+    if args.merge:
+        return run_merge(args)
     if args.impl == "reference":
         return run_reference(args)
     if args.sweep:

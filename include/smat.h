@@ -280,6 +280,76 @@ const char* smat_status_string(smat_status s);
 /* Message describing the last failure on the calling thread ("" if none). */
 const char* smat_last_error(void);
 
+/* ---------------------------------------------------------------- merging ---
+ * The evaluation side (Eq. merged-state): theta_merge = theta0 + sum_j
+ * alpha_j (.) m_j (.) Delta_j over K experts, Delta_j = theta_j - theta0, for
+ * the merging methods the paper evaluates with (Sec. 5): weight averaging
+ * (alpha_j = 1/K), Task Arithmetic (alpha_j = gamma), DARE followed by Task
+ * Arithmetic (m_j drops each coordinate with probability p_drop and rescales
+ * the rest by 1 / (1 - p_drop); the masks are the SMAT Mask stream of this
+ * library with the expert index as the step, so they are the same Philox
+ * draws), and TIES (per tensor and expert keep the ceil(retention n) largest
+ * |Delta_j|, ties at the threshold kept; elect the sign of the sum of the
+ * kept values; average the kept values of that sign; scale by gamma).
+ * One dtype per call. Arithmetic: fp32, experts accumulated in index order with one fused
+ * multiply-add each (TIES: sums and one division), then fl(theta0 + acc)
+ * rounded to the storage dtype; results are bit-identical to the CPU oracle. */
+typedef enum {
+  SMAT_MERGE_WA = 0,
+  SMAT_MERGE_TA = 1,
+  SMAT_MERGE_DARE_TA = 2,
+  SMAT_MERGE_TIES = 3
+} smat_merge_method;
+
+#define SMAT_MERGE_MAX_EXPERTS 16
+
+/* One tensor to merge: theta0 and n_experts expert tensors (GPU-readable,
+ * numel elements of dtype each) into out (GPU memory). experts is a HOST
+ * array of n_experts pointers. out may equal theta0 (merged in place); it
+ * must not overlap an expert or overlap theta0 otherwise. tensor_id (<
+ * 0x0FFFFFFF, unique) and elem_offset key the DARE masks like the SMAT
+ * descriptors do. */
+typedef struct {
+  const void* theta0;
+  const void* const* experts;
+  void* out;
+  int64_t numel;
+  int64_t elem_offset;
+  uint32_t tensor_id;
+  int32_t dtype;
+} smat_merge_tensor;
+
+typedef struct {
+  int32_t method;        /* smat_merge_method */
+  int32_t n_experts;     /* 1 .. SMAT_MERGE_MAX_EXPERTS, the same for every tensor */
+  float gamma;           /* merging coefficient (TA, DARE + TA, TIES); finite */
+  float p_drop;          /* DARE drop probability in [0, 1) */
+  float retention;       /* TIES fraction kept per tensor and expert, (0, 1] */
+  uint64_t seed;         /* DARE mask key */
+  int32_t philox_rounds; /* 10 (default) or 7 */
+  int32_t flags;         /* 0 */
+} smat_merge_config;
+
+/* Bytes of device workspace smat_merge needs (0 on invalid arguments). */
+size_t smat_merge_workspace_bytes(const smat_merge_tensor* tensors, int32_t n_tensors,
+                                  const smat_merge_config* cfg);
+
+/* Merge every tensor on `stream` (asynchronous; the host arrays are read
+ * before return). d_workspace: device memory of at least
+ * smat_merge_workspace_bytes bytes, 256-byte aligned, not in use by another
+ * call until this one's work on `stream` has finished. TIES first selects
+ * each tensor's per-expert threshold exactly (three passes of a radix
+ * select over the magnitudes), then merges. */
+smat_status smat_merge(const smat_merge_tensor* tensors, int32_t n_tensors, const smat_merge_config* cfg,
+                       void* d_workspace, size_t workspace_bytes, smat_stream_t stream);
+
+/* Test hook: the TIES threshold keys (bits of the kept magnitude's lower
+ * bound, n_tensors * n_experts uint32, tensor-major) that the last TIES
+ * smat_merge on this workspace selected, copied to the device buffer d_out. */
+smat_status smat_merge_ties_thresholds(const smat_merge_tensor* tensors, int32_t n_tensors,
+                                       const smat_merge_config* cfg, const void* d_workspace,
+                                       uint32_t* d_out, smat_stream_t stream);
+
 /* SMAT_ABI_VERSION of the loaded library. */
 int32_t smat_abi_version(void);
 

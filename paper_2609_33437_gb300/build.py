@@ -17,7 +17,7 @@ LIB = os.path.join(PKG, "libsmat.so")
 
 SOURCES = ["smat_fused_bf16.cu", "smat_fused_f32.cu", "smat_sim_bf16.cu", "smat_sim_f32.cu",
            "smat_inplace_bf16.cu", "smat_inplace_f32.cu", "smat_inplace_sim_bf16.cu", "smat_inplace_sim_f32.cu",
-           "smat_laplace_bf16.cu", "smat_laplace_f32.cu", "smat_gradmap.cu", "smat_aux.cu", "smat_noalloc.cu",
+           "smat_laplace_bf16.cu", "smat_laplace_f32.cu", "smat_merge.cu", "smat_gradmap.cu", "smat_aux.cu", "smat_noalloc.cu",
            "smat_host.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-fmad=false", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",

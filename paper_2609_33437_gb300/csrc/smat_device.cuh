@@ -69,9 +69,14 @@ __device__ __forceinline__ uint4 philox(uint32_t c0, uint32_t c1, uint32_t c2, u
 // caller guarantees j < 2^32, so counter word 1 is the constant 0 and the
 // loop-invariant part of the first two rounds can be hoisted.
 template <int R, bool J0 = false>
+__device__ __forceinline__ uint4 stream_block_at(const RoundKeys& key, uint32_t step, uint32_t stream,
+                                                 uint32_t tid, uint64_t j) {
+  return philox<R>((uint32_t)j, J0 ? 0u : (uint32_t)(j >> 32), (stream << 28) | tid, step, key);
+}
+template <int R, bool J0 = false>
 __device__ __forceinline__ uint4 stream_block(const KArgs& a, uint32_t stream, uint32_t tid,
                                               uint64_t j) {
-  return philox<R>((uint32_t)j, J0 ? 0u : (uint32_t)(j >> 32), (stream << 28) | tid, a.step, a.key);
+  return stream_block_at<R, J0>(a.key, a.step, stream, tid, j);
 }
 
 __device__ __forceinline__ uint32_t pick(const uint4& w, unsigned i) {
@@ -333,10 +338,7 @@ __device__ __forceinline__ bool kept_of(const uint32_t (&kw)[4], int e) {
 // a tie is decided by the low 24 bits of the uniform (MASK_LO stream), which
 // the caller resolves (group_ties16 / resolve_group_ties); its flag is left
 // clear here.
-template <int R, bool J0>
-__device__ __forceinline__ bool group_keep16(const KArgs& a, uint32_t tid, uint32_t t_hi, uint64_t gidx0,
-                                             uint32_t (&kw)[4]) {
-  const uint4 w = stream_block<R, J0>(a, S_MASK, tid, gidx0 >> 4);
+__device__ __forceinline__ bool keep_bytes16(const uint4& w, uint32_t t_hi, uint32_t (&kw)[4]) {
   const uint32_t words[4] = {w.x, w.y, w.z, w.w};
   const uint32_t tt = t_hi * 0x01010101u;
   const uint32_t tl = tt & 0x7F7F7F7Fu;
@@ -352,12 +354,15 @@ __device__ __forceinline__ bool group_keep16(const KArgs& a, uint32_t tid, uint3
   }
   return anytie != 0u;
 }
+template <int R, bool J0>
+__device__ __forceinline__ bool group_keep16(const KArgs& a, uint32_t tid, uint32_t t_hi, uint64_t gidx0,
+                                             uint32_t (&kw)[4]) {
+  return keep_bytes16(stream_block<R, J0>(a, S_MASK, tid, gidx0 >> 4), t_hi, kw);
+}
 
 // Tie elements of the 16-element group at gidx0: bit e set iff element e's
 // mask byte equals the threshold's high byte.
-template <int R, bool J0>
-__device__ __forceinline__ uint32_t group_ties16(const KArgs& a, uint32_t tid, uint32_t t_hi, uint64_t gidx0) {
-  const uint4 w = stream_block<R, J0>(a, S_MASK, tid, gidx0 >> 4);
+__device__ __forceinline__ uint32_t tie_bits16(const uint4& w, uint32_t t_hi) {
   const uint32_t words[4] = {w.x, w.y, w.z, w.w};
   const uint32_t tt = t_hi * 0x01010101u;
   uint32_t tbits = 0u;
@@ -369,6 +374,10 @@ __device__ __forceinline__ uint32_t group_ties16(const KArgs& a, uint32_t tid, u
     tbits |= ((((eq >> 7) * 0x00204081u) >> 21) & 0xFu) << (4 * q);
   }
   return tbits;
+}
+template <int R, bool J0>
+__device__ __forceinline__ uint32_t group_ties16(const KArgs& a, uint32_t tid, uint32_t t_hi, uint64_t gidx0) {
+  return tie_bits16(stream_block<R, J0>(a, S_MASK, tid, gidx0 >> 4), t_hi);
 }
 
 // Low-24-bit test of one tie element.

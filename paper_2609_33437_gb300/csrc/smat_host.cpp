@@ -157,40 +157,56 @@ smat_status check_tensors(const smat_tensor_desc* t, int32_t n, const smat_confi
 // addressing its device address is the host address), or any host memory
 // when the device reads pageable memory directly (coherent CPU-GPU systems).
 smat_status check_gpu_access(const smat_tensor_desc* t, int32_t n) {
-  int dev = 0, pageable = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return fail(SMAT_ERR_CUDA, "no current CUDA device");
-  if (cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccess, dev) != cudaSuccess) pageable = 0;
   for (int32_t k = 0; k < n; ++k) {
     if (t[k].numel <= 0) continue;
     const void* ptrs[3] = {t[k].theta, t[k].theta0, t[k].sim};
     for (const void* p : ptrs) {
-      cudaPointerAttributes at;
-      if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
-        cudaGetLastError();
-        return fail(SMAT_ERR_INVALID_ARG, "tensor %d: pointer attributes unavailable", k);
-      }
-      const bool ok = at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged ||
-                      (at.type == cudaMemoryTypeHost && at.devicePointer == p) ||
-                      (at.type == cudaMemoryTypeUnregistered && pageable);
+      const int ok = gpu_can_access(p);
+      if (ok < 0) return fail(SMAT_ERR_CUDA, "no current CUDA device or pointer attributes unavailable");
       if (!ok) return fail(SMAT_ERR_INVALID_ARG, "tensor %d: a data pointer is not accessible from the GPU", k);
     }
   }
   return SMAT_OK;
 }
 
-RoundKeys make_keys(uint64_t seed) {
+RoundKeys make_keys(uint64_t seed) { return make_round_keys(seed); }
+
+}  // namespace
+
+// 1 if the kernels can dereference p as it is: device or managed memory, host
+// memory registered with CUDA (pinned; under unified addressing its device
+// address is the host address), or any host memory when the device reads
+// pageable memory directly (coherent CPU-GPU systems); 0 if not; -1 on a
+// CUDA error.
+int smat::gpu_can_access(const void* p) {
+  int dev = 0, pageable = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return -1;
+  if (cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccess, dev) != cudaSuccess) pageable = 0;
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return -1;
+  }
+  return (at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged ||
+          (at.type == cudaMemoryTypeHost && at.devicePointer == p) ||
+          (at.type == cudaMemoryTypeUnregistered && pageable))
+             ? 1
+             : 0;
+}
+
+// Philox round keys of a seed: key = (seed mod 2^32, seed div 2^32), each
+// round's key advanced by the Weyl increments of the key schedule.
+RoundKeys smat::make_round_keys(uint64_t seed) {
   RoundKeys k;
   uint32_t a = (uint32_t)(seed & 0xFFFFFFFFu), b = (uint32_t)(seed >> 32);
   for (int r = 0; r < kMaxRounds; ++r) {
     k.k0[r] = a;
     k.k1[r] = b;
-    a += 0x9E3779B9u;  // Weyl increments of the Philox key schedule
+    a += 0x9E3779B9u;
     b += 0xBB67AE85u;
   }
   return k;
 }
-
-}  // namespace
 
 int smat::record_error_code(int status, const char* msg) {
   g_last_error = msg;

@@ -162,5 +162,9 @@ constexpr int kBlock = 256;
 
 // Record `msg` as this thread's smat_last_error() text; returns `status`.
 int record_error_code(int status, const char* msg);
+// 1 if kernels can dereference p as it is, 0 if not, -1 on a CUDA error.
+int gpu_can_access(const void* p);
+// Philox round keys of a seed (smat_host.cpp).
+RoundKeys make_round_keys(uint64_t seed);
 
 }  // namespace smat

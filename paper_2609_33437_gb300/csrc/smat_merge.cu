@@ -1,0 +1,587 @@
+// Merging over K experts (the evaluation side, Eq. merged-state):
+// theta_merge = theta0 + sum_j alpha_j (.) m_j (.) Delta_j, Delta_j = theta_j -
+// theta0, for weight averaging, Task Arithmetic, DARE followed by Task
+// Arithmetic and TIES (the merging methods of Sec. 5). Elementwise and bound
+// by HBM bandwidth: each element reads theta0 and the K experts once and
+// writes the result once (TIES first reads every expert three more times to
+// select its per-tensor trim thresholds exactly).
+//
+// Arithmetic, identical to the CPU oracle: Delta_j one fp32 subtraction;
+// experts accumulated in index order, one fused multiply-add each (WA 1/K,
+// TA gamma, DARE gamma / p_keep on the kept coordinates); TIES sums the kept
+// values, elects the sign of that sum, averages the kept values of that sign
+// (one fp32 division) and scales by gamma; then fl(theta0 + acc) rounded to
+// the storage dtype. DARE's mask of expert j is the library's Mask stream
+// with step = j.
+//
+// TIES trim threshold of each (tensor, expert): the r-th largest key of
+// |Delta_j| (key = the bits of the magnitude as uint32, r = ceil(retention
+// n)), found by a most-significant-digit radix select in three passes of 11,
+// 11 and 10 bits: each pass histograms the digit of the keys that match the
+// digits decided so far (shared-memory histograms per chunk, flushed into
+// 64-bit global bins), then one CTA per (tensor, expert) picks the digit
+// whose bin holds the r-th largest and the rank within it.
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <unordered_set>
+#include <vector>
+
+#include "smat.h"
+#include "smat_device.cuh"
+
+namespace smat {
+namespace {
+
+constexpr int kMergeMaxExperts = SMAT_MERGE_MAX_EXPERTS;
+constexpr int64_t kMergeChunk = int64_t(1) << 16;
+constexpr int kHistBins = 2048;
+constexpr int kPasses = 3;
+constexpr int kPassShift[kPasses] = {21, 10, 0};
+constexpr int kPassWidth[kPasses] = {11, 11, 10};
+constexpr size_t kMergeAlign = 256;
+
+struct MTensor {
+  const void* theta0;
+  void* out;
+  int64_t numel;
+  int64_t elem_offset;
+  uint32_t tid, flags, t_hi, t_lo;
+  int32_t dtype, pad;
+};
+
+struct MArgs {
+  const MTensor* tensors;
+  const Chunk* chunks;
+  const void* const* experts;  // [tensor * K + e]
+  uint32_t* thr;               // [tensor * K + e] TIES threshold keys
+  uint32_t* prefix;            // radix select: the digits decided so far
+  int64_t* rank;               // radix select: rank among keys with that prefix (1 = largest)
+  unsigned long long* hist;    // [(tensor * K + e) * kHistBins]
+  int64_t n_chunks;
+  RoundKeys key;
+  int32_t K, method;
+  float gamma, c;              // c: per-expert coefficient (WA 1/K, TA gamma, DARE gamma / p_keep)
+  int32_t shift, width;        // current radix pass
+  uint32_t decided;            // mask of the key bits decided before this pass
+  int32_t last_pass;
+};
+
+__device__ __forceinline__ uint32_t abs_key(float x) { return __float_as_uint(x) & 0x7FFFFFFFu; }
+
+// DARE keep flags of the 16-element group at g0 for expert e: the Mask
+// stream at step e; the rare byte ties are decided at once.
+template <int R>
+__device__ __forceinline__ void dare_keep16(const MArgs& m, const MTensor& T, uint32_t e, uint64_t g0,
+                                            uint32_t (&kw)[4]) {
+  const uint4 w = stream_block_at<R>(m.key, e, S_MASK, T.tid, g0 >> 4);
+  if (keep_bytes16(w, T.t_hi, kw) && T.t_lo != 0u) {
+    uint32_t tb = tie_bits16(w, T.t_hi);
+    while (tb) {
+      const int k = __ffs(tb) - 1;
+      tb &= tb - 1u;
+      const uint64_t g = g0 + (uint64_t)k;
+      const uint4 l = stream_block_at<R>(m.key, e, S_MASK_LO, T.tid, g >> 2);
+      if ((pick(l, (unsigned)(g & 3)) >> 8) < T.t_lo) set_kept(kw, k);
+    }
+  }
+}
+
+template <int R>
+__device__ __forceinline__ bool dare_kept1(const MArgs& m, const MTensor& T, uint32_t e, uint64_t g) {
+  const uint4 w = stream_block_at<R>(m.key, e, S_MASK, T.tid, g >> 4);
+  const uint32_t hi = (pick(w, (unsigned)((g >> 2) & 3)) >> (8u * (unsigned)(g & 3))) & 0xFFu;
+  if (hi != T.t_hi) return hi < T.t_hi;
+  if (T.t_lo == 0u) return false;
+  const uint4 l = stream_block_at<R>(m.key, e, S_MASK_LO, T.tid, g >> 2);
+  return (pick(l, (unsigned)(g & 3)) >> 8) < T.t_lo;
+}
+
+// WA / TA / DARE on one 16-element group (vector path).
+template <int R, int DT, int METHOD>
+__device__ __forceinline__ void merge_linear16(const MArgs& m, const MTensor& T, int t, int64_t i) {
+  Raw16<DT> t0;
+  load16<DT>(T.theta0, i, t0);
+  float2 acc[8];
+#pragma unroll
+  for (int h = 0; h < 8; ++h) acc[h] = splat(0.0f);
+  const float2 c2 = splat(m.c);
+  const uint64_t g0 = (uint64_t)(T.elem_offset + i);
+  const bool masked = METHOD == SMAT_MERGE_DARE_TA && (T.flags & TF_MASK) != 0u;
+#pragma unroll 1
+  for (int e = 0; e < m.K; ++e) {
+    Raw16<DT> x;
+    load16<DT>(m.experts[t * m.K + e], i, x);
+    uint32_t kw[4] = {0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u};
+    if (masked) dare_keep16<R>(m, T, (uint32_t)e, g0, kw);
+#pragma unroll
+    for (int h = 0; h < 8; ++h) {
+      const float2 b = t0.pair(h);
+      const float2 d = add2_rn(x.pair(h), make_float2(-b.x, -b.y));
+      const float2 f = fma2_rn(c2, d, acc[h]);
+      acc[h] = make_float2(kept_of(kw, 2 * h) ? f.x : acc[h].x, kept_of(kw, 2 * h + 1) ? f.y : acc[h].y);
+    }
+  }
+  float out[16];
+#pragma unroll
+  for (int h = 0; h < 8; ++h) {
+    const float2 o = add2_rn(t0.pair(h), acc[h]);
+    out[2 * h] = o.x;
+    out[2 * h + 1] = o.y;
+  }
+  store16<DT>(T.out, i, out);
+}
+
+// TIES on one 16-element group: elect, then the disjoint mean (the experts
+// are read twice; the second read is served by the L2).
+template <int DT>
+__device__ __forceinline__ void merge_ties16(const MArgs& m, const MTensor& T, int t, int64_t i) {
+  Raw16<DT> t0;
+  load16<DT>(T.theta0, i, t0);
+  float sum[16];
+#pragma unroll
+  for (int k = 0; k < 16; ++k) sum[k] = 0.0f;
+#pragma unroll 1
+  for (int e = 0; e < m.K; ++e) {
+    Raw16<DT> x;
+    load16<DT>(m.experts[t * m.K + e], i, x);
+    const uint32_t thr = m.thr[t * m.K + e];
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      const float d = __fsub_rn(x.at(k), t0.at(k));
+      if (abs_key(d) >= thr) sum[k] = __fadd_rn(sum[k], d);
+    }
+  }
+  float part[16];
+  uint32_t cnt[4] = {0u, 0u, 0u, 0u};  // four 8-bit counts per word (K <= 16)
+#pragma unroll
+  for (int k = 0; k < 16; ++k) part[k] = 0.0f;
+#pragma unroll 1
+  for (int e = 0; e < m.K; ++e) {
+    Raw16<DT> x;
+    load16<DT>(m.experts[t * m.K + e], i, x);
+    const uint32_t thr = m.thr[t * m.K + e];
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      const float d = __fsub_rn(x.at(k), t0.at(k));
+      const bool agree = abs_key(d) >= thr && ((sum[k] > 0.0f && d > 0.0f) || (sum[k] < 0.0f && d < 0.0f));
+      if (agree) {
+        part[k] = __fadd_rn(part[k], d);
+        cnt[k >> 2] += 1u << (8 * (k & 3));
+      }
+    }
+  }
+  float out[16];
+#pragma unroll
+  for (int k = 0; k < 16; ++k) {
+    const uint32_t n = (cnt[k >> 2] >> (8 * (k & 3))) & 0xFFu;
+    const float merged = n ? __fdiv_rn(part[k], (float)n) : 0.0f;
+    out[k] = __fadd_rn(t0.at(k), __fmul_rn(m.gamma, merged));
+  }
+  store16<DT>(T.out, i, out);
+}
+
+// Any method, one element (any alignment).
+template <int R, int DT, int METHOD>
+__device__ __forceinline__ void merge_elem(const MArgs& m, const MTensor& T, int t, int64_t i) {
+  const float t0 = load1<DT>(T.theta0, i);
+  const uint64_t g = (uint64_t)(T.elem_offset + i);
+  float acc = 0.0f;
+  if (METHOD == SMAT_MERGE_TIES) {
+    float sum = 0.0f, part = 0.0f;
+    int n = 0;
+    for (int e = 0; e < m.K; ++e) {
+      const float d = __fsub_rn(load1<DT>(m.experts[t * m.K + e], i), t0);
+      if (abs_key(d) >= m.thr[t * m.K + e]) sum = __fadd_rn(sum, d);
+    }
+    for (int e = 0; e < m.K; ++e) {
+      const float d = __fsub_rn(load1<DT>(m.experts[t * m.K + e], i), t0);
+      if (abs_key(d) >= m.thr[t * m.K + e] && ((sum > 0.0f && d > 0.0f) || (sum < 0.0f && d < 0.0f))) {
+        part = __fadd_rn(part, d);
+        ++n;
+      }
+    }
+    acc = __fmul_rn(m.gamma, n ? __fdiv_rn(part, (float)n) : 0.0f);
+  } else {
+    for (int e = 0; e < m.K; ++e) {
+      const float d = __fsub_rn(load1<DT>(m.experts[t * m.K + e], i), t0);
+      const bool kept = METHOD != SMAT_MERGE_DARE_TA || !(T.flags & TF_MASK) || dare_kept1<R>(m, T, (uint32_t)e, g);
+      if (kept) acc = __fmaf_rn(m.c, d, acc);
+    }
+  }
+  store1<DT>(T.out, i, __fadd_rn(t0, acc));
+}
+
+template <int R, int DT, int METHOD>
+__global__ void __launch_bounds__(kBlock, 2) merge_kernel(const __grid_constant__ MArgs m) {
+  for (int64_t ci = blockIdx.x; ci < m.n_chunks; ci += gridDim.x) {
+    const Chunk ch = m.chunks[ci];
+    const MTensor& T = m.tensors[ch.tensor];
+    const bool vec = (T.flags & TF_VEC) != 0u;
+    for (int64_t i = ch.begin + 16 * (int64_t)threadIdx.x; i < ch.end; i += 16 * (int64_t)kBlock) {
+      if (vec && i + 16 <= ch.end) {
+        if (METHOD == SMAT_MERGE_TIES)
+          merge_ties16<DT>(m, T, ch.tensor, i);
+        else
+          merge_linear16<R, DT, METHOD>(m, T, ch.tensor, i);
+      } else {
+        const int64_t e_end = (i + 16 < ch.end) ? i + 16 : ch.end;
+        for (int64_t e = i; e < e_end; ++e) merge_elem<R, DT, METHOD>(m, T, ch.tensor, e);
+      }
+    }
+  }
+}
+
+// One radix pass of the TIES threshold selection: work items are (chunk,
+// expert) pairs.
+template <int DT>
+__global__ void __launch_bounds__(kBlock) ties_hist_kernel(const __grid_constant__ MArgs m) {
+  __shared__ uint32_t h[kHistBins];
+  const int64_t items = m.n_chunks * m.K;
+  const uint32_t digit = (1u << m.width) - 1u;
+  for (int64_t w = blockIdx.x; w < items; w += gridDim.x) {
+    const int64_t ci = w / m.K;
+    const int e = (int)(w % m.K);
+    const Chunk ch = m.chunks[ci];
+    const MTensor& T = m.tensors[ch.tensor];
+    const int slot = ch.tensor * m.K + e;
+    for (int b = threadIdx.x; b < kHistBins; b += kBlock) h[b] = 0u;
+    __syncthreads();
+    const uint32_t P = m.prefix[slot];
+    const void* xp = m.experts[slot];
+    const bool vec = (T.flags & TF_VEC) != 0u;
+    for (int64_t i = ch.begin + 16 * (int64_t)threadIdx.x; i < ch.end; i += 16 * (int64_t)kBlock) {
+      if (vec && i + 16 <= ch.end) {
+        Raw16<DT> t0, x;
+        load16<DT>(T.theta0, i, t0);
+        load16<DT>(xp, i, x);
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          const uint32_t key = abs_key(__fsub_rn(x.at(k), t0.at(k)));
+          if ((key & m.decided) == P) atomicAdd(&h[(key >> m.shift) & digit], 1u);
+        }
+      } else {
+        const int64_t e_end = (i + 16 < ch.end) ? i + 16 : ch.end;
+        for (int64_t k = i; k < e_end; ++k) {
+          const uint32_t key = abs_key(__fsub_rn(load1<DT>(xp, k), load1<DT>(T.theta0, k)));
+          if ((key & m.decided) == P) atomicAdd(&h[(key >> m.shift) & digit], 1u);
+        }
+      }
+    }
+    __syncthreads();
+    unsigned long long* gh = m.hist + (size_t)slot * kHistBins;
+    for (int b = threadIdx.x; b < kHistBins; b += kBlock)
+      if (h[b]) atomicAdd(gh + b, (unsigned long long)h[b]);
+    __syncthreads();
+  }
+}
+
+// After a pass: one CTA per (tensor, expert) picks the digit whose bin holds
+// the rank-th largest key (bins scanned from the top), records it and the
+// rank within that bin, and clears the histogram for the next pass.
+__global__ void __launch_bounds__(kBlock) ties_select_kernel(const __grid_constant__ MArgs m) {
+  __shared__ unsigned long long s_sum[kBlock];
+  __shared__ int s_digit;
+  __shared__ long long s_above;
+  const int slot = blockIdx.x;
+  unsigned long long* gh = m.hist + (size_t)slot * kHistBins;
+  const long long r = m.rank[slot];
+  const int nb = 1 << m.width;
+  const int per = nb / kBlock;  // bins per thread, highest bins in thread 0
+  unsigned long long local = 0;
+  const int top = nb - 1 - threadIdx.x * per;
+  for (int k = 0; k < per; ++k) local += gh[top - k];
+  s_sum[threadIdx.x] = local;
+  if (threadIdx.x == 0) {
+    s_digit = -1;
+    s_above = 0;
+  }
+  __syncthreads();
+  // inclusive scan from the top (Hillis-Steele; 8 steps over 256 entries)
+  for (int o = 1; o < kBlock; o <<= 1) {
+    const unsigned long long v = threadIdx.x >= o ? s_sum[threadIdx.x - o] : 0ull;
+    __syncthreads();
+    s_sum[threadIdx.x] += v;
+    __syncthreads();
+  }
+  const unsigned long long incl = s_sum[threadIdx.x];
+  const unsigned long long excl = incl - local;
+  if (r > 0 && (long long)excl < r && r <= (long long)incl) {
+    unsigned long long acc = excl;
+    for (int k = 0; k < per; ++k) {
+      const unsigned long long c = gh[top - k];
+      if ((long long)(acc + c) >= r) {
+        s_digit = top - k;
+        s_above = (long long)acc;
+        break;
+      }
+      acc += c;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && r > 0 && s_digit >= 0) {
+    const uint32_t p = m.prefix[slot] | ((uint32_t)s_digit << m.shift);
+    m.prefix[slot] = p;
+    m.rank[slot] = r - s_above;
+    if (m.last_pass) m.thr[slot] = p;
+  }
+  for (int b = threadIdx.x; b < kHistBins; b += kBlock) gh[b] = 0ull;
+}
+
+template <int R, int DT>
+cudaError_t merge_method(const MArgs& m, int grid, cudaStream_t s) {
+  switch (m.method) {
+    case SMAT_MERGE_WA: merge_kernel<R, DT, SMAT_MERGE_WA><<<grid, kBlock, 0, s>>>(m); break;
+    case SMAT_MERGE_TA: merge_kernel<R, DT, SMAT_MERGE_TA><<<grid, kBlock, 0, s>>>(m); break;
+    case SMAT_MERGE_DARE_TA: merge_kernel<R, DT, SMAT_MERGE_DARE_TA><<<grid, kBlock, 0, s>>>(m); break;
+    default: merge_kernel<R, DT, SMAT_MERGE_TIES><<<grid, kBlock, 0, s>>>(m); break;
+  }
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------- host ---
+struct MLayout {
+  size_t tensors, chunks, experts, thr, prefix, rank, hist, total;
+};
+
+size_t align_m(size_t x) { return (x + kMergeAlign - 1) / kMergeAlign * kMergeAlign; }
+
+MLayout merge_layout(int32_t n, int64_t n_chunks, int K, bool ties) {
+  MLayout L;
+  size_t off = 0;
+  const size_t slots = (size_t)n * (size_t)K;
+  L.tensors = off; off = align_m(off + sizeof(MTensor) * (size_t)n);
+  L.chunks = off;  off = align_m(off + sizeof(Chunk) * (size_t)n_chunks);
+  L.experts = off; off = align_m(off + sizeof(void*) * slots);
+  L.thr = off;     off = align_m(off + sizeof(uint32_t) * slots);
+  L.prefix = off;  off = align_m(off + sizeof(uint32_t) * slots);
+  L.rank = off;    off = align_m(off + sizeof(int64_t) * slots);
+  L.hist = off;    off = align_m(off + (ties ? sizeof(unsigned long long) * kHistBins * slots : 0));
+  L.total = off;
+  return L;
+}
+
+smat_status mfail(smat_status s, const char* fmt, ...) {
+  char buf[256];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  return (smat_status)record_error_code((int)s, buf);
+}
+
+bool m_overlaps(const void* a, size_t na, const void* b, size_t nb) {
+  const uintptr_t x = (uintptr_t)a, y = (uintptr_t)b;
+  return x < y + nb && y < x + na;
+}
+
+// Host-side validation (no device access); returns the chunk count and the
+// list's dtype (one dtype per call).
+smat_status merge_check(const smat_merge_tensor* t, int32_t n, const smat_merge_config* cfg, int64_t* n_chunks,
+                        int32_t* dtype_out) {
+  if (!cfg) return mfail(SMAT_ERR_INVALID_ARG, "cfg is NULL");
+  if (cfg->method < SMAT_MERGE_WA || cfg->method > SMAT_MERGE_TIES)
+    return mfail(SMAT_ERR_UNSUPPORTED, "merge method %d not supported", cfg->method);
+  if (cfg->n_experts < 1 || cfg->n_experts > kMergeMaxExperts)
+    return mfail(SMAT_ERR_INVALID_ARG, "n_experts %d not in [1, %d]", cfg->n_experts, kMergeMaxExperts);
+  if (!std::isfinite(cfg->gamma)) return mfail(SMAT_ERR_INVALID_ARG, "gamma not finite");
+  if (!(cfg->p_drop >= 0.0f && cfg->p_drop < 1.0f)) return mfail(SMAT_ERR_INVALID_ARG, "p_drop not in [0, 1)");
+  if (!(cfg->retention > 0.0f && cfg->retention <= 1.0f))
+    return mfail(SMAT_ERR_INVALID_ARG, "retention not in (0, 1]");
+  if (cfg->philox_rounds != 0 && cfg->philox_rounds != 7 && cfg->philox_rounds != 10)
+    return mfail(SMAT_ERR_UNSUPPORTED, "philox_rounds %d not supported (7 or 10)", cfg->philox_rounds);
+  if (cfg->flags != 0) return mfail(SMAT_ERR_UNSUPPORTED, "unknown flags 0x%x", cfg->flags);
+  if (n < 0 || (n > 0 && !t)) return mfail(SMAT_ERR_INVALID_ARG, "bad tensor list");
+  std::unordered_set<uint32_t> ids;
+  int64_t nc = 0;
+  for (int32_t k = 0; k < n; ++k) {
+    const smat_merge_tensor& d = t[k];
+    if (d.numel < 0 || d.numel >= (int64_t(1) << 40))
+      return mfail(SMAT_ERR_INVALID_ARG, "tensor %d: numel out of range", k);
+    if (d.elem_offset < 0 || d.elem_offset >= (int64_t(1) << 62) - d.numel)
+      return mfail(SMAT_ERR_INVALID_ARG, "tensor %d: elem_offset out of range", k);
+    if (d.tensor_id >= kGlobalAlphaTensor) return mfail(SMAT_ERR_INVALID_ARG, "tensor %d: tensor_id too large", k);
+    if (!ids.insert(d.tensor_id).second) return mfail(SMAT_ERR_INVALID_ARG, "tensor %d: duplicate tensor_id", k);
+    if (d.dtype != SMAT_F32 && d.dtype != SMAT_BF16)
+      return mfail(SMAT_ERR_UNSUPPORTED, "tensor %d: dtype %d not supported", k, d.dtype);
+    if (d.dtype != t[0].dtype) return mfail(SMAT_ERR_UNSUPPORTED, "tensor %d: one dtype per merge call", k);
+    if (d.numel > 0) {
+      const size_t es = d.dtype == SMAT_BF16 ? 2 : 4, bytes = es * (size_t)d.numel;
+      if (!d.theta0 || !d.out || !d.experts) return mfail(SMAT_ERR_INVALID_ARG, "tensor %d: NULL pointer", k);
+      if ((uintptr_t)d.theta0 % es || (uintptr_t)d.out % es)
+        return mfail(SMAT_ERR_ALIGNMENT, "tensor %d: pointer not aligned to its element size", k);
+      if (d.out != d.theta0 && m_overlaps(d.out, bytes, d.theta0, bytes))
+        return mfail(SMAT_ERR_INVALID_ARG, "tensor %d: out overlaps theta0 without being equal to it", k);
+      for (int e = 0; e < cfg->n_experts; ++e) {
+        const void* x = d.experts[e];
+        if (!x) return mfail(SMAT_ERR_INVALID_ARG, "tensor %d: expert %d is NULL", k, e);
+        if ((uintptr_t)x % es) return mfail(SMAT_ERR_ALIGNMENT, "tensor %d: expert %d misaligned", k, e);
+        if (m_overlaps(d.out, bytes, x, bytes))
+          return mfail(SMAT_ERR_INVALID_ARG, "tensor %d: out overlaps expert %d", k, e);
+      }
+    }
+    nc += (d.numel + kMergeChunk - 1) / kMergeChunk;
+  }
+  if (nc >= (int64_t(1) << 31)) return mfail(SMAT_ERR_INVALID_ARG, "too many chunks");
+  *n_chunks = nc;
+  *dtype_out = n > 0 ? t[0].dtype : SMAT_F32;
+  return SMAT_OK;
+}
+
+template <int R, int DT>
+cudaError_t merge_launch(MArgs m, int64_t slots, bool ties, int sms, cudaStream_t s) {
+  if (ties) {
+    const int64_t items = m.n_chunks * m.K;
+    const int hgrid = (int)(items < 4 * (int64_t)sms ? items : 4 * (int64_t)sms);
+    for (int p = 0; p < kPasses; ++p) {
+      m.shift = kPassShift[p];
+      m.width = kPassWidth[p];
+      m.decided = (m.shift + m.width >= 32) ? 0u : ~((1u << (m.shift + m.width)) - 1u);
+      m.last_pass = p == kPasses - 1;
+      ties_hist_kernel<DT><<<hgrid, kBlock, 0, s>>>(m);
+      ties_select_kernel<<<(int)slots, kBlock, 0, s>>>(m);
+    }
+  }
+  const int grid = (int)(m.n_chunks < 2 * (int64_t)sms ? m.n_chunks : 2 * (int64_t)sms);
+  return merge_method<R, DT>(m, grid, s);
+}
+
+}  // namespace
+}  // namespace smat
+
+using namespace smat;
+
+extern "C" size_t smat_merge_workspace_bytes(const smat_merge_tensor* tensors, int32_t n_tensors,
+                                             const smat_merge_config* cfg) {
+  int64_t nc = 0;
+  int32_t dt = 0;
+  if (merge_check(tensors, n_tensors, cfg, &nc, &dt) != SMAT_OK) return 0;
+  return merge_layout(n_tensors, nc, cfg->n_experts, cfg->method == SMAT_MERGE_TIES).total;
+}
+
+extern "C" smat_status smat_merge(const smat_merge_tensor* tensors, int32_t n_tensors, const smat_merge_config* cfg,
+                                  void* d_workspace, size_t workspace_bytes, smat_stream_t stream) {
+  int64_t nc = 0;
+  int32_t dtype = 0;
+  smat_status st = merge_check(tensors, n_tensors, cfg, &nc, &dtype);
+  if (st != SMAT_OK) return st;
+  const int K = cfg->n_experts;
+  const bool ties = cfg->method == SMAT_MERGE_TIES;
+  const MLayout L = merge_layout(n_tensors, nc, K, ties);
+  if (!d_workspace || (uintptr_t)d_workspace % kMergeAlign)
+    return mfail(SMAT_ERR_WORKSPACE, "workspace NULL or not 256-byte aligned");
+  if (workspace_bytes < L.total) return mfail(SMAT_ERR_WORKSPACE, "workspace %zu < %zu bytes", workspace_bytes, L.total);
+  for (int32_t k = 0; k < n_tensors; ++k) {
+    if (tensors[k].numel <= 0) continue;
+    int ok = gpu_can_access(tensors[k].theta0) == 1 && gpu_can_access(tensors[k].out) == 1;
+    for (int e = 0; ok && e < K; ++e) ok = gpu_can_access(tensors[k].experts[e]) == 1;
+    if (!ok) return mfail(SMAT_ERR_INVALID_ARG, "tensor %d: a pointer is not accessible from the GPU", k);
+  }
+  if (n_tensors == 0 || nc == 0) return SMAT_OK;
+
+  // tables (host), then one upload each
+  const float keep = 1.0f - cfg->p_drop;
+  const uint64_t T = (uint64_t)std::floor((double)keep * 4294967296.0);
+  std::vector<MTensor> ht((size_t)n_tensors);
+  std::vector<Chunk> hc;
+  hc.reserve((size_t)nc);
+  std::vector<const void*> hx((size_t)n_tensors * (size_t)K, nullptr);
+  std::vector<int64_t> hrank((size_t)n_tensors * (size_t)K, 0);
+  for (int32_t k = 0; k < n_tensors; ++k) {
+    const smat_merge_tensor& d = tensors[k];
+    MTensor& M = ht[(size_t)k];
+    std::memset(&M, 0, sizeof(M));
+    M.theta0 = d.theta0;
+    M.out = d.out;
+    M.numel = d.numel;
+    M.elem_offset = d.elem_offset;
+    M.tid = d.tensor_id;
+    M.dtype = d.dtype;
+    bool vec = d.numel > 0 && (uintptr_t)d.theta0 % 32 == 0 && (uintptr_t)d.out % 32 == 0 && d.elem_offset % 16 == 0;
+    for (int e = 0; e < K; ++e) {
+      hx[(size_t)k * K + e] = d.numel > 0 ? d.experts[e] : nullptr;
+      vec = vec && (uintptr_t)d.experts[e] % 32 == 0;
+    }
+    M.flags = vec ? TF_VEC : 0u;
+    if (cfg->method == SMAT_MERGE_DARE_TA && T < (uint64_t(1) << 32)) {
+      M.flags |= TF_MASK;
+      M.t_hi = (uint32_t)(T >> 24);
+      M.t_lo = (uint32_t)(T & 0xFFFFFFu);
+    }
+    if (ties && d.numel > 0) {
+      int64_t r = (int64_t)std::ceil((double)cfg->retention * (double)d.numel);
+      r = r < 1 ? 1 : (r > d.numel ? d.numel : r);
+      for (int e = 0; e < K; ++e) hrank[(size_t)k * K + e] = r;
+    }
+    for (int64_t j = 0; j * kMergeChunk < d.numel; ++j) {
+      Chunk ch;
+      ch.tensor = k;
+      ch.pad = 0;
+      ch.begin = j * kMergeChunk;
+      ch.end = (j + 1) * kMergeChunk < d.numel ? (j + 1) * kMergeChunk : d.numel;
+      hc.push_back(ch);
+    }
+  }
+  char* ws = static_cast<char*>(d_workspace);
+  MArgs m;
+  std::memset(&m, 0, sizeof(m));
+  m.tensors = reinterpret_cast<const MTensor*>(ws + L.tensors);
+  m.chunks = reinterpret_cast<const Chunk*>(ws + L.chunks);
+  m.experts = reinterpret_cast<const void* const*>(ws + L.experts);
+  m.thr = reinterpret_cast<uint32_t*>(ws + L.thr);
+  m.prefix = reinterpret_cast<uint32_t*>(ws + L.prefix);
+  m.rank = reinterpret_cast<int64_t*>(ws + L.rank);
+  m.hist = ties ? reinterpret_cast<unsigned long long*>(ws + L.hist) : nullptr;
+  m.n_chunks = nc;
+  m.key = make_round_keys(cfg->seed);
+  m.K = K;
+  m.method = cfg->method;
+  m.gamma = cfg->gamma;
+  const float inv_keep = (float)(1.0 / (double)keep);
+  m.c = cfg->method == SMAT_MERGE_WA ? (float)(1.0 / (double)K)
+        : cfg->method == SMAT_MERGE_DARE_TA ? cfg->gamma * inv_keep : cfg->gamma;
+  const size_t slots = (size_t)n_tensors * (size_t)K;
+  cudaError_t e = cudaMemcpyAsync(ws + L.tensors, ht.data(), sizeof(MTensor) * ht.size(), cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(ws + L.chunks, hc.data(), sizeof(Chunk) * hc.size(), cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(ws + L.experts, hx.data(), sizeof(void*) * slots, cudaMemcpyHostToDevice, stream);
+  if (e != cudaSuccess) return mfail(SMAT_ERR_CUDA, "merge table upload failed");
+  int dev = 0, sms = 1;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return mfail(SMAT_ERR_CUDA, "device query failed");
+  const int rounds = cfg->philox_rounds == 7 ? 7 : 10;
+  if (ties) {
+    e = cudaMemsetAsync(ws + L.prefix, 0, sizeof(uint32_t) * slots, stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(ws + L.thr, 0, sizeof(uint32_t) * slots, stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(ws + L.hist, 0, sizeof(unsigned long long) * kHistBins * slots, stream);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(ws + L.rank, hrank.data(), sizeof(int64_t) * slots, cudaMemcpyHostToDevice, stream);
+    if (e != cudaSuccess) return mfail(SMAT_ERR_CUDA, "TIES state initialisation failed");
+  }
+  const int64_t slots64 = (int64_t)slots;
+  if (dtype == SMAT_BF16)
+    e = rounds == 7 ? merge_launch<7, DT_BF16>(m, slots64, ties, sms, stream)
+                    : merge_launch<10, DT_BF16>(m, slots64, ties, sms, stream);
+  else
+    e = rounds == 7 ? merge_launch<7, DT_F32>(m, slots64, ties, sms, stream)
+                    : merge_launch<10, DT_F32>(m, slots64, ties, sms, stream);
+  if (e != cudaSuccess) return mfail(SMAT_ERR_CUDA, "merge launch failed");
+  return SMAT_OK;
+}
+
+extern "C" smat_status smat_merge_ties_thresholds(const smat_merge_tensor* tensors, int32_t n_tensors,
+                                                  const smat_merge_config* cfg, const void* d_workspace,
+                                                  uint32_t* d_out, smat_stream_t stream) {
+  int64_t nc = 0;
+  int32_t dtype = 0;
+  smat_status st = merge_check(tensors, n_tensors, cfg, &nc, &dtype);
+  if (st != SMAT_OK) return st;
+  if (cfg->method != SMAT_MERGE_TIES) return mfail(SMAT_ERR_STATE, "not a TIES configuration");
+  if (!d_workspace || !d_out) return mfail(SMAT_ERR_INVALID_ARG, "NULL pointer");
+  const MLayout L = merge_layout(n_tensors, nc, cfg->n_experts, true);
+  const size_t bytes = sizeof(uint32_t) * (size_t)n_tensors * (size_t)cfg->n_experts;
+  if (bytes && cudaMemcpyAsync(d_out, static_cast<const char*>(d_workspace) + L.thr, bytes,
+                               cudaMemcpyDeviceToDevice, stream) != cudaSuccess)
+    return mfail(SMAT_ERR_CUDA, "threshold copy failed");
+  return SMAT_OK;
+}

@@ -26,7 +26,8 @@ EXPORTED = ("smat_workspace_bytes", "smat_init", "smat_simulate_multi", "smat_gr
             "smat_swap", "smat_active", "smat_mask_bits", "smat_tensor_scalars", "smat_destroy",
             "smat_debug_philox", "smat_debug_noise_unit", "smat_debug_fused", "smat_poll_errors",
             "smat_delta_sigma_noalloc", "smat_timing_enable", "smat_timing_read", "smat_status_string",
-            "smat_last_error", "smat_abi_version")
+            "smat_last_error", "smat_abi_version", "smat_refill_theta0", "smat_mark_theta0_resident",
+            "smat_merge_workspace_bytes", "smat_merge", "smat_merge_ties_thresholds")
 
 
 class SmatError(RuntimeError):
@@ -86,6 +87,10 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
     L.smat_tensor_scalars.argtypes = [P, U32, P, P]
     L.smat_destroy.argtypes = [P]
     L.smat_refill_theta0.argtypes = [P, P, P]
+    L.smat_merge_workspace_bytes.argtypes = [P, I32, P]
+    L.smat_merge_workspace_bytes.restype = ctypes.c_size_t
+    L.smat_merge.argtypes = [P, I32, P, P, ctypes.c_size_t, P]
+    L.smat_merge_ties_thresholds.argtypes = [P, I32, P, P, P, P]
     L.smat_mark_theta0_resident.argtypes = [P]
     L.smat_debug_philox.argtypes = [P, I64, U64, I32, P, P, P]
     L.smat_debug_noise_unit.argtypes = [P, I64, I32, P, P]
@@ -103,7 +108,7 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
     for name in ("smat_init", "smat_simulate_multi", "smat_grad_map_multi", "smat_swap", "smat_active",
                  "smat_mask_bits", "smat_tensor_scalars", "smat_destroy", "smat_debug_philox", "smat_debug_noise_unit",
                  "smat_poll_errors", "smat_debug_fused", "smat_timing_enable", "smat_timing_read",
-                 "smat_refill_theta0", "smat_mark_theta0_resident"):
+                 "smat_refill_theta0", "smat_mark_theta0_resident", "smat_merge", "smat_merge_ties_thresholds"):
         getattr(L, name).restype = I32
     _lib = L
     return L
@@ -371,3 +376,69 @@ class SmatParameters:
     def grad_map(self, step: int, accumulate: bool = False):
         gs = [p.grad for p in self.params]
         self.session.grad_map_multi(step, gs, gs, accumulate=accumulate)
+
+
+# ------------------------------------------------------------------ merging ---
+SMAT_MERGE_WA, SMAT_MERGE_TA, SMAT_MERGE_DARE_TA, SMAT_MERGE_TIES = 0, 1, 2, 3
+
+
+class MergeTensor(ctypes.Structure):
+    _fields_ = [("theta0", ctypes.c_void_p), ("experts", ctypes.c_void_p), ("out", ctypes.c_void_p),
+                ("numel", ctypes.c_int64), ("elem_offset", ctypes.c_int64), ("tensor_id", ctypes.c_uint32),
+                ("dtype", ctypes.c_int32)]
+
+
+class MergeConfig(ctypes.Structure):
+    _fields_ = [("method", ctypes.c_int32), ("n_experts", ctypes.c_int32), ("gamma", ctypes.c_float),
+                ("p_drop", ctypes.c_float), ("retention", ctypes.c_float), ("seed", ctypes.c_uint64),
+                ("philox_rounds", ctypes.c_int32), ("flags", ctypes.c_int32)]
+
+
+def merge(theta0s: Sequence[torch.Tensor], experts: Sequence[Sequence[torch.Tensor]], outs: Sequence[torch.Tensor],
+          method: int, gamma: float = 1.0, p_drop: float = 0.0, retention: float = 1.0, seed: int = 0,
+          tensor_ids: Optional[Sequence[int]] = None, elem_offsets: Optional[Sequence[int]] = None,
+          philox_rounds: int = 10, stream: Optional[torch.cuda.Stream] = None, return_thresholds: bool = False):
+    """Merge K experts per tensor into outs (Eq. merged-state; see smat_merge
+    in include/smat.h): experts[k] lists tensor k's K expert tensors. outs[k]
+    may be theta0s[k]. With return_thresholds (TIES), returns the
+    n_tensors x K threshold keys (int32 view of the uint32 bits)."""
+    L = load_library()
+    n = len(theta0s)
+    if len(experts) != n or len(outs) != n:
+        raise ValueError("per-tensor lists differ in length")
+    K = len(experts[0]) if n else 0
+    tensor_ids = tensor_ids if tensor_ids is not None else list(range(n))
+    elem_offsets = elem_offsets if elem_offsets is not None else [0] * n
+    descs = (MergeTensor * max(n, 1))()
+    keep = []
+    for k in range(n):
+        if len(experts[k]) != K:
+            raise ValueError("every tensor needs the same number of experts")
+        for t in [theta0s[k], outs[k], *experts[k]]:
+            if not t.is_contiguous() or t.numel() != theta0s[k].numel() or t.dtype != theta0s[k].dtype:
+                raise ValueError(f"tensor {k}: contiguous tensors of one shape and dtype")
+        ptrs = (ctypes.c_void_p * max(K, 1))(*[x.data_ptr() for x in experts[k]])
+        keep.append(ptrs)
+        d = descs[k]
+        d.theta0, d.out = theta0s[k].data_ptr(), outs[k].data_ptr()
+        d.experts = ctypes.cast(ptrs, ctypes.c_void_p)
+        d.numel = theta0s[k].numel()
+        d.elem_offset = int(elem_offsets[k])
+        d.tensor_id = int(tensor_ids[k])
+        d.dtype = dtype_code(theta0s[k].dtype)
+    cfg = MergeConfig(int(method), K, float(gamma), float(p_drop), float(retention), int(seed) & (2**64 - 1),
+                      int(philox_rounds), 0)
+    nbytes = L.smat_merge_workspace_bytes(ctypes.byref(descs), n, ctypes.byref(cfg))
+    device = outs[0].device if n else torch.device("cuda", torch.cuda.current_device())
+    ws = torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+    check("smat_merge", L.smat_merge(ctypes.byref(descs), n, ctypes.byref(cfg), ctypes.c_void_p(ws.data_ptr()),
+                                     ws.numel(), _stream_handle(stream)))
+    if stream is not None:
+        ws.record_stream(stream)
+    if return_thresholds:
+        thr = torch.empty(max(n * K, 1), dtype=torch.int32, device=device)
+        check("smat_merge_ties_thresholds",
+              L.smat_merge_ties_thresholds(ctypes.byref(descs), n, ctypes.byref(cfg), ctypes.c_void_p(ws.data_ptr()),
+                                           ctypes.c_void_p(thr.data_ptr()), _stream_handle(stream)))
+        return thr[:n * K].view(n, K)
+    return None

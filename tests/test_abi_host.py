@@ -17,7 +17,7 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 def header_functions():
     src = open(os.path.join(ROOT, "include", "smat.h")).read()
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
-    return sorted(set(re.findall(r"\b(smat_[a-z_]+)\s*\(", src)))
+    return sorted(set(re.findall(r"\b(smat_[a-z0-9_]+)\s*\(", src)))
 
 
 @pytest.fixture(scope="module")
@@ -195,3 +195,35 @@ def test_workload_inventory():
     for w in (W.dec_0p5b(), W.llama_7b(), W.vl_7b()):
         for t in w.tensors:
             assert (t.keep_prob < 1.0) == (t.kind == "linear")
+
+
+def test_merge_host_validation(L):
+    """smat_merge_workspace_bytes sizes valid lists (TIES adds the radix
+    histograms) and returns 0 for invalid ones, without a GPU."""
+    K, n = 3, 1 << 20
+    exps = (ctypes.c_void_p * K)(*[0x40000000 + (k + 1) * 0x1000000 for k in range(K)])
+
+    def tens(out=0x30000000, dtype=S.SMAT_F32, numel=n, experts=exps):
+        t = S.MergeTensor()
+        t.theta0, t.out, t.numel, t.dtype, t.tensor_id = 0x20000000, out, numel, dtype, 0
+        t.experts = ctypes.cast(experts, ctypes.c_void_p)
+        return t
+
+    def ws(ts, method=S.SMAT_MERGE_TA, k=K, **kw):
+        arr = (S.MergeTensor * len(ts))(*ts)
+        c = S.MergeConfig(method, k, kw.get("gamma", 1.0), kw.get("p_drop", 0.0), kw.get("retention", 1.0), 0,
+                          kw.get("rounds", 10), kw.get("flags", 0))
+        return L.smat_merge_workspace_bytes(ctypes.byref(arr), len(ts), ctypes.byref(c))
+
+    ta, ties = ws([tens()]), ws([tens()], S.SMAT_MERGE_TIES)
+    assert ta > 0 and ties >= ta + 2048 * 8 * K
+    assert ws([tens(out=0x20000000)]) > 0  # in place into theta0
+    assert ws([tens(out=0x41000000)]) == 0  # out is expert 0
+    assert ws([tens(out=0x20000004)]) == 0  # partial overlap with theta0
+    assert ws([tens()], k=0) == 0 and ws([tens()], k=17) == 0
+    assert ws([tens()], S.SMAT_MERGE_DARE_TA, p_drop=1.0) == 0
+    assert ws([tens()], S.SMAT_MERGE_TIES, retention=0.0) == 0
+    assert ws([tens()], 4) == 0 and ws([tens()], rounds=8) == 0 and ws([tens()], flags=1) == 0
+    b = tens(dtype=S.SMAT_BF16)
+    b.tensor_id = 1
+    assert ws([tens(), b]) == 0  # one dtype per call
