@@ -99,6 +99,26 @@ __device__ __forceinline__ bool dare_kept1(const MArgs& m, const MTensor& T, uin
   return (pick(l, (unsigned)(g & 3)) >> 8) < T.t_lo;
 }
 
+// Expert e's contribution to a 16-element group: acc += c Delta (kept only).
+template <int R, int DT, int METHOD>
+__device__ __forceinline__ void merge_acc16(const MArgs& m, const MTensor& T, int e, uint64_t g0,
+                                            const Raw16<DT>& x, const Raw16<DT>& t0, float2 (&acc)[8]) {
+  uint32_t kw[4] = {0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u};
+  if (METHOD == SMAT_MERGE_DARE_TA && (T.flags & TF_MASK)) dare_keep16<R>(m, T, (uint32_t)e, g0, kw);
+  const float2 c2 = splat(m.c);
+#pragma unroll
+  for (int h = 0; h < 8; ++h) {
+    const float2 b = t0.pair(h);
+    const float2 d = add2_rn(x.pair(h), make_float2(-b.x, -b.y));
+    const float2 f = fma2_rn(c2, d, acc[h]);
+    acc[h] = make_float2(kept_of(kw, 2 * h) ? f.x : acc[h].x, kept_of(kw, 2 * h + 1) ? f.y : acc[h].y);
+  }
+}
+
+// Experts are loaded four at a time (all four loads in flight before the
+// first is used) and accumulated in index order.
+constexpr int kExpertBatch = 4;
+
 // WA / TA / DARE on one 16-element group (vector path).
 template <int R, int DT, int METHOD>
 __device__ __forceinline__ void merge_linear16(const MArgs& m, const MTensor& T, int t, int64_t i) {
@@ -107,22 +127,22 @@ __device__ __forceinline__ void merge_linear16(const MArgs& m, const MTensor& T,
   float2 acc[8];
 #pragma unroll
   for (int h = 0; h < 8; ++h) acc[h] = splat(0.0f);
-  const float2 c2 = splat(m.c);
   const uint64_t g0 = (uint64_t)(T.elem_offset + i);
-  const bool masked = METHOD == SMAT_MERGE_DARE_TA && (T.flags & TF_MASK) != 0u;
+  const void* const* xp = m.experts + t * m.K;
+  int e = 0;
 #pragma unroll 1
-  for (int e = 0; e < m.K; ++e) {
-    Raw16<DT> x;
-    load16<DT>(m.experts[t * m.K + e], i, x);
-    uint32_t kw[4] = {0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u};
-    if (masked) dare_keep16<R>(m, T, (uint32_t)e, g0, kw);
+  for (; e + kExpertBatch <= m.K; e += kExpertBatch) {
+    Raw16<DT> x[kExpertBatch];
 #pragma unroll
-    for (int h = 0; h < 8; ++h) {
-      const float2 b = t0.pair(h);
-      const float2 d = add2_rn(x.pair(h), make_float2(-b.x, -b.y));
-      const float2 f = fma2_rn(c2, d, acc[h]);
-      acc[h] = make_float2(kept_of(kw, 2 * h) ? f.x : acc[h].x, kept_of(kw, 2 * h + 1) ? f.y : acc[h].y);
-    }
+    for (int b = 0; b < kExpertBatch; ++b) load16<DT>(xp[e + b], i, x[b]);
+#pragma unroll
+    for (int b = 0; b < kExpertBatch; ++b) merge_acc16<R, DT, METHOD>(m, T, e + b, g0, x[b], t0, acc);
+  }
+#pragma unroll 1
+  for (; e < m.K; ++e) {
+    Raw16<DT> x;
+    load16<DT>(xp[e], i, x);
+    merge_acc16<R, DT, METHOD>(m, T, e, g0, x, t0, acc);
   }
   float out[16];
 #pragma unroll
@@ -140,29 +160,38 @@ template <int DT>
 __device__ __forceinline__ void merge_ties16(const MArgs& m, const MTensor& T, int t, int64_t i) {
   Raw16<DT> t0;
   load16<DT>(T.theta0, i, t0);
+  const void* const* xp = m.experts + t * m.K;
+  const uint32_t* tp = m.thr + t * m.K;
   float sum[16];
 #pragma unroll
   for (int k = 0; k < 16; ++k) sum[k] = 0.0f;
-#pragma unroll 1
-  for (int e = 0; e < m.K; ++e) {
-    Raw16<DT> x;
-    load16<DT>(m.experts[t * m.K + e], i, x);
-    const uint32_t thr = m.thr[t * m.K + e];
+  auto elect = [&](const Raw16<DT>& x, uint32_t thr) {
 #pragma unroll
     for (int k = 0; k < 16; ++k) {
       const float d = __fsub_rn(x.at(k), t0.at(k));
       if (abs_key(d) >= thr) sum[k] = __fadd_rn(sum[k], d);
     }
+  };
+  int e = 0;
+#pragma unroll 1
+  for (; e + kExpertBatch <= m.K; e += kExpertBatch) {
+    Raw16<DT> x[kExpertBatch];
+#pragma unroll
+    for (int b = 0; b < kExpertBatch; ++b) load16<DT>(xp[e + b], i, x[b]);
+#pragma unroll
+    for (int b = 0; b < kExpertBatch; ++b) elect(x[b], tp[e + b]);
+  }
+#pragma unroll 1
+  for (; e < m.K; ++e) {
+    Raw16<DT> x;
+    load16<DT>(xp[e], i, x);
+    elect(x, tp[e]);
   }
   float part[16];
   uint32_t cnt[4] = {0u, 0u, 0u, 0u};  // four 8-bit counts per word (K <= 16)
 #pragma unroll
   for (int k = 0; k < 16; ++k) part[k] = 0.0f;
-#pragma unroll 1
-  for (int e = 0; e < m.K; ++e) {
-    Raw16<DT> x;
-    load16<DT>(m.experts[t * m.K + e], i, x);
-    const uint32_t thr = m.thr[t * m.K + e];
+  auto gather = [&](const Raw16<DT>& x, uint32_t thr) {
 #pragma unroll
     for (int k = 0; k < 16; ++k) {
       const float d = __fsub_rn(x.at(k), t0.at(k));
@@ -172,6 +201,21 @@ __device__ __forceinline__ void merge_ties16(const MArgs& m, const MTensor& T, i
         cnt[k >> 2] += 1u << (8 * (k & 3));
       }
     }
+  };
+  e = 0;
+#pragma unroll 1
+  for (; e + kExpertBatch <= m.K; e += kExpertBatch) {
+    Raw16<DT> x[kExpertBatch];
+#pragma unroll
+    for (int b = 0; b < kExpertBatch; ++b) load16<DT>(xp[e + b], i, x[b]);
+#pragma unroll
+    for (int b = 0; b < kExpertBatch; ++b) gather(x[b], tp[e + b]);
+  }
+#pragma unroll 1
+  for (; e < m.K; ++e) {
+    Raw16<DT> x;
+    load16<DT>(xp[e], i, x);
+    gather(x, tp[e]);
   }
   float out[16];
 #pragma unroll
