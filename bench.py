@@ -310,10 +310,14 @@ def host_available_bytes():
         return 0
 
 
-def e2e_run(w, sess_factory, steps, warmup, world):
+def e2e_run(w, sess_factory, steps, warmup, world, groups=8):
     """The same step through the public API with host inputs: pinned host
     theta, theta0 and g~ are copied in and theta~ and g copied out every
-    step, inside the timed region."""
+    step, inside the timed region. The list is cut into `groups` groups of
+    consecutive tensors (one session each, same tensor ids, so the results
+    are those of one session) and pipelined over three streams: group k's
+    inputs are copied in while group k - 1 computes and group k - 2's results
+    are copied out; each step ends when all of its results are on the host."""
     dev = torch.device("cuda")
     tdt, gdt = W.torch_dtype(w.dtype), W.torch_dtype(w.gdtype)
     n = w.numel
@@ -335,23 +339,50 @@ def e2e_run(w, sess_factory, steps, warmup, world):
         d_gs.append(g)
         d_sim.append(torch.empty_like(th))
         d_go.append(torch.empty_like(g))
-    sess = sess_factory(d_th, d_t0, d_sim)
     hv = lambda h: [h[int(offs[k]):int(offs[k + 1])] for k in range(len(w.tensors))]  # noqa: E731
     hth, ht0, hgs, hsim, hgo = hv(h_th), hv(h_t0), hv(h_gs), hv(h_sim), hv(h_go)
+    # groups of consecutive tensors with about n / groups elements each
+    cuts, target, acc, start = [], n / max(1, groups), 0, 0
+    for k, t in enumerate(w.tensors):
+        acc += t.numel
+        if acc >= target * (len(cuts) + 1) or k == len(w.tensors) - 1:
+            cuts.append(list(range(start, k + 1)))
+            start = k + 1
+    sessions = [sess_factory([d_th[k] for k in ks], [d_t0[k] for k in ks], [d_sim[k] for k in ks], ks)
+                for ks in cuts]
+    s_in, s_cmp, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    done = [None] * len(cuts)    # compute of the group finished (its inputs are free)
+    copied = [None] * len(cuts)  # results of the group copied out (its outputs are free)
 
     def one(step):
-        for k in range(len(w.tensors)):
-            d_th[k].copy_(hth[k], non_blocking=True)
-            d_t0[k].copy_(ht0[k], non_blocking=True)
-            d_gs[k].copy_(hgs[k], non_blocking=True)
-        sess.simulate_multi(step)
-        sess.swap()
-        sess.grad_map_multi(step, d_gs, d_go)
-        sess.swap()
-        for k in range(len(w.tensors)):
-            hsim[k].copy_(d_sim[k], non_blocking=True)
-            hgo[k].copy_(d_go[k], non_blocking=True)
-        torch.cuda.current_stream().synchronize()
+        for gi, ks in enumerate(cuts):
+            ev_in = torch.cuda.Event()
+            with torch.cuda.stream(s_in):
+                if done[gi] is not None:
+                    s_in.wait_event(done[gi])
+                for k in ks:
+                    d_th[k].copy_(hth[k], non_blocking=True)
+                    d_t0[k].copy_(ht0[k], non_blocking=True)
+                    d_gs[k].copy_(hgs[k], non_blocking=True)
+                ev_in.record(s_in)
+            sess = sessions[gi]
+            s_cmp.wait_event(ev_in)
+            if copied[gi] is not None:
+                s_cmp.wait_event(copied[gi])
+            sess.simulate_multi(step, stream=s_cmp)
+            sess.swap()
+            sess.grad_map_multi(step, [d_gs[k] for k in ks], [d_go[k] for k in ks], stream=s_cmp)
+            sess.swap()
+            done[gi] = torch.cuda.Event()
+            done[gi].record(s_cmp)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(done[gi])
+                for k in ks:
+                    hsim[k].copy_(d_sim[k], non_blocking=True)
+                    hgo[k].copy_(d_go[k], non_blocking=True)
+                copied[gi] = torch.cuda.Event()
+                copied[gi].record(s_out)
+        s_out.synchronize()
 
     for s in range(warmup):
         one(s)
@@ -365,9 +396,11 @@ def e2e_run(w, sess_factory, steps, warmup, world):
     bytes_step = sum(step_bytes(w).values())
     h2d = 2 * h_th.element_size() * n + h_gs.element_size() * n
     d2h = h_sim.element_size() * n + h_go.element_size() * n
-    sess.close()
+    for sess in sessions:
+        sess.close()
     return {"value": world * bytes_step * steps / el / 1e9, "unit": UNIT, "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h, "ms_per_step": 1e3 * el / steps, "workload": w.name}
+            "d2h_bytes_per_step": d2h, "ms_per_step": 1e3 * el / steps, "workload": w.name,
+            "pipeline": f"{len(cuts)} tensor groups over copy-in / compute / copy-out streams"}
 
 
 def run_smat(args):
@@ -377,9 +410,12 @@ def run_smat(args):
     dev = torch.device("cuda", local)
     w = rank_workload(workload(args), rank)
 
-    def make_session(th, t0, sim):
-        return S.SmatSession(th, t0, sim, [t.keep_prob for t in w.tensors], [t.sigma for t in w.tensors],
-                             [t.sigma_rel for t in w.tensors], seed=w.seed, alpha_min=w.alpha_min,
+    def make_session(th, t0, sim, idx=None):
+        # idx: the tensors' positions in the list (their ids; all tensors by default)
+        idx = list(range(len(w.tensors))) if idx is None else list(idx)
+        ts = [w.tensors[i] for i in idx]
+        return S.SmatSession(th, t0, sim, [t.keep_prob for t in ts], [t.sigma for t in ts],
+                             [t.sigma_rel for t in ts], tensor_ids=idx, seed=w.seed, alpha_min=w.alpha_min,
                              alpha_max=w.alpha_max, alpha_mode=w.alpha_mode, noise=w.noise,
                              philox_rounds=args.philox_rounds)
 
