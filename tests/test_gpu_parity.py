@@ -198,6 +198,43 @@ def test_shard_invariance_on_gpu():
     assert torch.equal(torch.cat([a, b]).view(torch.int16), full.view(torch.int16))
 
 
+def test_tensor_order_and_grouping_invariance():
+    """Results depend on each tensor's id, not on its position in the list or
+    on which other tensors share the launch: the list in reverse order, and
+    split into two contexts, give the same bits (forward, with sigma_rel
+    statistics fused, and gradient map)."""
+    dev = torch.device("cuda")
+    sizes = [70_001, 262_144 + 7, 17, 300_000, 4096]
+    th = [(torch.randn(n, device=dev) * 0.02).to(torch.bfloat16) for n in sizes]
+    t0 = [(x.float() + torch.randn(x.numel(), device=dev) * 1e-3).to(torch.bfloat16) for x in th]
+    gs = [torch.randn(n, device=dev).to(torch.bfloat16) for n in sizes]
+    keeps = [0.7, 0.5, 1.0, 0.3, 0.9]
+    sig = [1e-3, 0.0, 2e-3, 0.0, 1e-3]
+    rel = [0.0, 0.1, 0.0, 0.1, 0.0]
+    kw = dict(seed=21, alpha_min=0.3, alpha_mode=S.SMAT_ALPHA_PER_TENSOR, noise=S.SMAT_NOISE_GAUSSIAN)
+
+    def run(order_groups):
+        sims = [torch.empty_like(x) for x in th]
+        gos = [torch.empty_like(g) for g in gs]
+        for idx in order_groups:
+            s = S.SmatSession([th[i] for i in idx], [t0[i] for i in idx], [sims[i] for i in idx],
+                              [keeps[i] for i in idx], [sig[i] for i in idx], [rel[i] for i in idx],
+                              tensor_ids=[100 + i for i in idx], **kw)
+            s.simulate_multi(3)
+            s.swap()
+            s.grad_map_multi(3, [gs[i] for i in idx], [gos[i] for i in idx])
+            s.swap()
+            assert s.poll_errors() == 0
+        torch.cuda.synchronize()
+        return sims, gos
+
+    ref = run([[0, 1, 2, 3, 4]])
+    for groups in ([[4, 3, 2, 1, 0]], [[3, 0], [4, 2, 1]]):
+        got = run(groups)
+        for a, b in zip(ref[0] + ref[1], got[0] + got[1]):
+            assert torch.equal(a.view(torch.int16), b.view(torch.int16)), groups
+
+
 def test_inplace_gradient_map():
     dev = torch.device("cuda")
     n = 100_003
