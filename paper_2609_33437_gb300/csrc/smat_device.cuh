@@ -423,16 +423,21 @@ struct TieList {
   }
 };
 
-// Keep decision of one element (any alignment).
+// Keep decision of one element (any alignment) of the Mask stream at `step`.
 template <int R>
-__device__ __forceinline__ bool elem_kept(const KArgs& a, uint32_t tid, uint32_t t_hi,
-                                          uint32_t t_lo, uint64_t gidx) {
-  const uint4 w = stream_block<R>(a, S_MASK, tid, gidx >> 4);
+__device__ __forceinline__ bool elem_kept_at(const RoundKeys& key, uint32_t step, uint32_t tid, uint32_t t_hi,
+                                             uint32_t t_lo, uint64_t gidx) {
+  const uint4 w = stream_block_at<R>(key, step, S_MASK, tid, gidx >> 4);
   const uint32_t hi = (pick(w, (unsigned)((gidx >> 2) & 3)) >> (8u * (unsigned)(gidx & 3))) & 0xFFu;
   if (hi != t_hi) return hi < t_hi;
   if (t_lo == 0u) return false;
-  const uint4 l = stream_block<R>(a, S_MASK_LO, tid, gidx >> 2);
+  const uint4 l = stream_block_at<R>(key, step, S_MASK_LO, tid, gidx >> 2);
   return (pick(l, (unsigned)(gidx & 3)) >> 8) < t_lo;
+}
+template <int R>
+__device__ __forceinline__ bool elem_kept(const KArgs& a, uint32_t tid, uint32_t t_hi,
+                                          uint32_t t_lo, uint64_t gidx) {
+  return elem_kept_at<R>(a.key, a.step, tid, t_hi, t_lo, gidx);
 }
 
 // ------------------------------------------------------------ memory I/O ---

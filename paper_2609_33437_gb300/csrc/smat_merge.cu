@@ -89,15 +89,6 @@ __device__ __forceinline__ void dare_keep16(const MArgs& m, const MTensor& T, ui
   }
 }
 
-template <int R>
-__device__ __forceinline__ bool dare_kept1(const MArgs& m, const MTensor& T, uint32_t e, uint64_t g) {
-  const uint4 w = stream_block_at<R>(m.key, e, S_MASK, T.tid, g >> 4);
-  const uint32_t hi = (pick(w, (unsigned)((g >> 2) & 3)) >> (8u * (unsigned)(g & 3))) & 0xFFu;
-  if (hi != T.t_hi) return hi < T.t_hi;
-  if (T.t_lo == 0u) return false;
-  const uint4 l = stream_block_at<R>(m.key, e, S_MASK_LO, T.tid, g >> 2);
-  return (pick(l, (unsigned)(g & 3)) >> 8) < T.t_lo;
-}
 
 // Expert e's contribution to a 16-element group: acc += c Delta (kept only).
 template <int R, int DT, int METHOD>
@@ -251,7 +242,8 @@ __device__ __forceinline__ void merge_elem(const MArgs& m, const MTensor& T, int
   } else {
     for (int e = 0; e < m.K; ++e) {
       const float d = __fsub_rn(load1<DT>(m.experts[t * m.K + e], i), t0);
-      const bool kept = METHOD != SMAT_MERGE_DARE_TA || !(T.flags & TF_MASK) || dare_kept1<R>(m, T, (uint32_t)e, g);
+      const bool kept = METHOD != SMAT_MERGE_DARE_TA || !(T.flags & TF_MASK) ||
+                        elem_kept_at<R>(m.key, (uint32_t)e, T.tid, T.t_hi, T.t_lo, g);
       if (kept) acc = __fmaf_rn(m.c, d, acc);
     }
   }
