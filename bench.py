@@ -310,6 +310,27 @@ def host_available_bytes():
         return 0
 
 
+def gpu_local_cpus(device_index: int):
+    """CPUs of the NUMA node the GPU's PCI function reports (sysfs), or None."""
+    try:
+        p = torch.cuda.get_device_properties(device_index)
+        dev = "%04x:%02x:%02x.0" % (p.pci_domain_id, p.pci_bus_id, p.pci_device_id)
+        with open(f"/sys/bus/pci/devices/{dev}/numa_node") as f:
+            node = int(f.read().strip())
+        if node < 0:
+            return None
+        with open(f"/sys/devices/system/node/node{node}/cpulist") as f:
+            spec = f.read().strip()
+        cpus = set()
+        for part in spec.split(","):
+            if part:
+                a, _, b = part.partition("-")
+                cpus.update(range(int(a), int(b or a) + 1))
+        return (node, cpus) if cpus else None
+    except Exception:
+        return None
+
+
 def e2e_run(w, sess_factory, steps, warmup, world, groups=8):
     """The same step through the public API with host inputs: pinned host
     theta, theta0 and g~ are copied in and theta~ and g copied out every
@@ -321,6 +342,11 @@ def e2e_run(w, sess_factory, steps, warmup, world, groups=8):
     dev = torch.device("cuda")
     tdt, gdt = W.torch_dtype(w.dtype), W.torch_dtype(w.gdtype)
     n = w.numel
+    # host buffers and copies on the CPUs next to the GPU (first-touch placement)
+    local = gpu_local_cpus(torch.cuda.current_device())
+    saved = os.sched_getaffinity(0) if local else None
+    if local:
+        os.sched_setaffinity(0, local[1])
     h_th = torch.empty(n, dtype=tdt, pin_memory=True)
     h_t0 = torch.empty(n, dtype=tdt, pin_memory=True)
     h_gs = torch.empty(n, dtype=gdt, pin_memory=True)
@@ -398,9 +424,12 @@ def e2e_run(w, sess_factory, steps, warmup, world, groups=8):
     d2h = h_sim.element_size() * n + h_go.element_size() * n
     for sess in sessions:
         sess.close()
+    if saved:
+        os.sched_setaffinity(0, saved)
     return {"value": world * bytes_step * steps / el / 1e9, "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": 1e3 * el / steps, "workload": w.name,
-            "pipeline": f"{len(cuts)} tensor groups over copy-in / compute / copy-out streams"}
+            "pipeline": f"{len(cuts)} tensor groups over copy-in / compute / copy-out streams",
+            "host_numa_node": local[0] if local else None}
 
 
 def run_smat(args):
