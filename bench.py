@@ -331,7 +331,7 @@ def gpu_local_cpus(device_index: int):
         return None
 
 
-def e2e_run(w, sess_factory, steps, warmup, world, groups=8):
+def e2e_run(w, sess_factory, steps, warmup, world, groups=8, keep_outputs=False):
     """The same step through the public API with host inputs: pinned host
     theta, theta0 and g~ are copied in and theta~ and g copied out every
     step, inside the timed region. The list is cut into `groups` groups of
@@ -426,6 +426,8 @@ def e2e_run(w, sess_factory, steps, warmup, world, groups=8):
         sess.close()
     if saved:
         os.sched_setaffinity(0, saved)
+    if keep_outputs:  # the last step's theta~ and g on the host (tests)
+        return hsim, hgo
     return {"value": world * bytes_step * steps / el / 1e9, "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": 1e3 * el / steps, "workload": w.name,
             "pipeline": f"{len(cuts)} tensor groups over copy-in / compute / copy-out streams",

@@ -124,3 +124,15 @@ def test_merge_argument_errors():
     with pytest.raises(S.SmatError):
         S.merge(t0s + [t0s[0].to(torch.bfloat16)], exs + [[x.to(torch.bfloat16) for x in exs[0]]],
                 out + [torch.empty(1000, device="cuda", dtype=torch.bfloat16)], S.SMAT_MERGE_TA)  # two dtypes
+
+
+def test_merge_dare_seven_rounds():
+    """DARE masks with the 7-round stream option equal the oracle's."""
+    t0s, exs = _experts([70_001, 4096], 3, O.BF16, seed=17)
+    outs = [torch.empty_like(t) for t in t0s]
+    S.merge(t0s, exs, outs, S.SMAT_MERGE_DARE_TA, gamma=0.5, p_drop=0.3, seed=8, philox_rounds=7)
+    torch.cuda.synchronize()
+    for k, (t0, ex, out) in enumerate(zip(t0s, exs, outs)):
+        ref, _ = O.merge(O.MERGE_DARE_TA, to_host(t0), [to_host(x) for x in ex], dtype=O.BF16, gamma=0.5,
+                         p_drop=0.3, seed=8, tensor_id=k, rounds=7)
+        assert np.array_equal(to_host(out).view(np.uint16), ref.view(np.uint16)), k
