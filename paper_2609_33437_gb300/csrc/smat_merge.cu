@@ -71,70 +71,24 @@ struct MArgs {
 
 __device__ __forceinline__ uint32_t abs_key(float x) { return __float_as_uint(x) & 0x7FFFFFFFu; }
 
-// DARE keep flags of the 16-element group at g0 for expert e: the Mask
-// stream at step e; the rare byte ties are decided at once.
-template <int R>
-__device__ __forceinline__ void dare_keep16(const MArgs& m, const MTensor& T, uint32_t e, uint64_t g0,
-                                            uint32_t (&kw)[4]) {
-  const uint4 w = stream_block_at<R>(m.key, e, S_MASK, T.tid, g0 >> 4);
-  if (keep_bytes16(w, T.t_hi, kw) && T.t_lo != 0u) {
-    uint32_t tb = tie_bits16(w, T.t_hi);
-    while (tb) {
-      const int k = __ffs(tb) - 1;
-      tb &= tb - 1u;
-      const uint64_t g = g0 + (uint64_t)k;
-      const uint4 l = stream_block_at<R>(m.key, e, S_MASK_LO, T.tid, g >> 2);
-      if ((pick(l, (unsigned)(g & 3)) >> 8) < T.t_lo) set_kept(kw, k);
-    }
-  }
-}
-
-
-// Expert e's contribution to a 16-element group: acc += c Delta (kept only).
-template <int R, int DT, int METHOD>
-__device__ __forceinline__ void merge_acc16(const MArgs& m, const MTensor& T, int e, uint64_t g0,
-                                            const Raw16<DT>& x, const Raw16<DT>& t0, float2 (&acc)[8]) {
-  uint32_t kw[4] = {0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u};
-  if (METHOD == SMAT_MERGE_DARE_TA && (T.flags & TF_MASK)) dare_keep16<R>(m, T, (uint32_t)e, g0, kw);
-  const float2 c2 = splat(m.c);
+// Expert e's contribution to a 16-element group: acc += c Delta on the
+// elements whose bit is set in keep (bit k: element k).
+template <int DT>
+__device__ __forceinline__ void merge_acc16(float c, uint32_t keep, const Raw16<DT>& x, const Raw16<DT>& t0,
+                                            float2 (&acc)[8]) {
+  const float2 c2 = splat(c);
 #pragma unroll
   for (int h = 0; h < 8; ++h) {
     const float2 b = t0.pair(h);
     const float2 d = add2_rn(x.pair(h), make_float2(-b.x, -b.y));
     const float2 f = fma2_rn(c2, d, acc[h]);
-    acc[h] = make_float2(kept_of(kw, 2 * h) ? f.x : acc[h].x, kept_of(kw, 2 * h + 1) ? f.y : acc[h].y);
+    acc[h] = make_float2(((keep >> (2 * h)) & 1u) ? f.x : acc[h].x, ((keep >> (2 * h + 1)) & 1u) ? f.y : acc[h].y);
   }
 }
 
-// Experts are loaded four at a time (all four loads in flight before the
-// first is used) and accumulated in index order.
-constexpr int kExpertBatch = 4;
-
-// WA / TA / DARE on one 16-element group (vector path).
-template <int R, int DT, int METHOD>
-__device__ __forceinline__ void merge_linear16(const MArgs& m, const MTensor& T, int t, int64_t i) {
-  Raw16<DT> t0;
-  load16<DT>(T.theta0, i, t0);
-  float2 acc[8];
-#pragma unroll
-  for (int h = 0; h < 8; ++h) acc[h] = splat(0.0f);
-  const uint64_t g0 = (uint64_t)(T.elem_offset + i);
-  const void* const* xp = m.experts + t * m.K;
-  int e = 0;
-#pragma unroll 1
-  for (; e + kExpertBatch <= m.K; e += kExpertBatch) {
-    Raw16<DT> x[kExpertBatch];
-#pragma unroll
-    for (int b = 0; b < kExpertBatch; ++b) load16<DT>(xp[e + b], i, x[b]);
-#pragma unroll
-    for (int b = 0; b < kExpertBatch; ++b) merge_acc16<R, DT, METHOD>(m, T, e + b, g0, x[b], t0, acc);
-  }
-#pragma unroll 1
-  for (; e < m.K; ++e) {
-    Raw16<DT> x;
-    load16<DT>(xp[e], i, x);
-    merge_acc16<R, DT, METHOD>(m, T, e, g0, x, t0, acc);
-  }
+template <int DT>
+__device__ __forceinline__ void store_merged16(const MTensor& T, int64_t i, const Raw16<DT>& t0,
+                                               const float2 (&acc)[8]) {
   float out[16];
 #pragma unroll
   for (int h = 0; h < 8; ++h) {
@@ -143,6 +97,153 @@ __device__ __forceinline__ void merge_linear16(const MArgs& m, const MTensor& T,
     out[2 * h + 1] = o.y;
   }
   store16<DT>(T.out, i, out);
+}
+
+// Experts are loaded four at a time (all four loads in flight before the
+// first is used) and accumulated in index order.
+constexpr int kExpertBatch = 4;
+
+// WA / TA on one 16-element group (vector path).
+template <int DT>
+__device__ __forceinline__ void merge_linear16(const MArgs& m, const MTensor& T, int t, int64_t i) {
+  Raw16<DT> t0;
+  load16<DT>(T.theta0, i, t0);
+  float2 acc[8];
+#pragma unroll
+  for (int h = 0; h < 8; ++h) acc[h] = splat(0.0f);
+  const void* const* xp = m.experts + t * m.K;
+  int e = 0;
+#pragma unroll 1
+  for (; e + kExpertBatch <= m.K; e += kExpertBatch) {
+    Raw16<DT> x[kExpertBatch];
+#pragma unroll
+    for (int b = 0; b < kExpertBatch; ++b) load16<DT>(xp[e + b], i, x[b]);
+#pragma unroll
+    for (int b = 0; b < kExpertBatch; ++b) merge_acc16<DT>(m.c, 0xFFFFu, x[b], t0, acc);
+  }
+#pragma unroll 1
+  for (; e < m.K; ++e) {
+    Raw16<DT> x;
+    load16<DT>(xp[e], i, x);
+    merge_acc16<DT>(m.c, 0xFFFFu, x, t0, acc);
+  }
+  store_merged16<DT>(T, i, t0, acc);
+}
+
+// DARE keep masks. A warp first draws the masks of its 32 groups for all K
+// experts (expert e's mask is the Mask stream at step e) into shared memory,
+// two experts per word (bit 16 (e & 1) + k: element k of expert e). An
+// element whose mask byte equals the threshold's high byte (probability
+// 1/256 per element and expert) is decided by its low 24 bits (MASK_LO
+// stream): these ties are queued per warp across all experts and then drawn
+// by the whole warp, one MASK_LO block per lane, so a warp spends about one
+// Philox pass per group on them instead of one mostly idle pass per expert.
+// A queue that fills up (about K/16 ties per thread are expected, the
+// capacity is 4 per thread) makes the owner draw the rest itself.
+constexpr int kDareQueue = 128;
+struct DareShared {
+  uint32_t keep[kMergeMaxExperts / 2][kBlock];
+  uint16_t q[kBlock / 32][kDareQueue];  // (lane << 8) | (expert << 4) | element
+  int n[kBlock / 32];
+};
+
+// kw's flag bits 8b + 7 of word q -> bit 4q + b.
+__device__ __forceinline__ uint32_t compress_keep16(const uint32_t (&kw)[4]) {
+  uint32_t r = 0u;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) r |= ((((kw[q] >> 7) * 0x00204081u) >> 21) & 0xFu) << (4 * q);
+  return r;
+}
+
+// Keep bits of expert e from its Mask block w (bit k: element k); ties go to
+// the warp's queue, or are drawn here once the queue is full.
+template <int R>
+__device__ __forceinline__ uint32_t dare_keep_bits(const MArgs& m, const MTensor& T, const uint4& w, int e,
+                                                   uint64_t g0, DareShared& s) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t kw[4];
+  if (keep_bytes16(w, T.t_hi, kw) && T.t_lo != 0u) {
+    uint32_t tb = tie_bits16(w, T.t_hi);
+    int slot = atomicAdd(&s.n[warp], __popc(tb));
+    while (tb) {
+      const int k = __ffs(tb) - 1;
+      tb &= tb - 1u;
+      if (slot < kDareQueue) {
+        s.q[warp][slot] = (uint16_t)((lane << 8) | (e << 4) | k);
+      } else {
+        const uint64_t g = g0 + (uint64_t)k;
+        const uint4 l = stream_block_at<R>(m.key, (uint32_t)e, S_MASK_LO, T.tid, g >> 2);
+        if ((pick(l, (unsigned)(g & 3)) >> 8) < T.t_lo) set_kept(kw, k);
+      }
+      ++slot;
+    }
+  }
+  return compress_keep16(kw);
+}
+
+// Called by all 32 lanes of the warp (full: this lane has a vector group at
+// element index g0; gw0: lane 0's group). Two experts' Mask blocks are drawn
+// together (two independent Philox chains per thread). On return the lane's
+// keep words are complete.
+template <int R>
+__device__ __forceinline__ void dare_masks(const MArgs& m, const MTensor& T, bool full, uint64_t g0, uint64_t gw0,
+                                           DareShared& s) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (lane == 0) s.n[warp] = 0;
+  __syncwarp();
+  if (full) {
+#pragma unroll 1
+    for (int e = 0; e < m.K; e += 2) {
+      const uint4 w0 = stream_block_at<R>(m.key, (uint32_t)e, S_MASK, T.tid, g0 >> 4);
+      const uint4 w1 = stream_block_at<R>(m.key, (uint32_t)e + 1u, S_MASK, T.tid, g0 >> 4);
+      uint32_t pair = dare_keep_bits<R>(m, T, w0, e, g0, s);
+      if (e + 1 < m.K) pair |= dare_keep_bits<R>(m, T, w1, e + 1, g0, s) << 16;
+      s.keep[e >> 1][threadIdx.x] = pair;
+    }
+  }
+  __syncwarp();
+  const int n = min(s.n[warp], kDareQueue);
+  for (int j = lane; j < n; j += 32) {
+    const uint32_t it = s.q[warp][j];
+    const int owner = (int)(it >> 8), e = (int)((it >> 4) & 15u), k = (int)(it & 15u);
+    const uint64_t g = gw0 + 16 * (uint64_t)owner + (uint64_t)k;
+    const uint4 l = stream_block_at<R>(m.key, (uint32_t)e, S_MASK_LO, T.tid, g >> 2);
+    if ((pick(l, (unsigned)(g & 3)) >> 8) < T.t_lo)
+      atomicOr(&s.keep[e >> 1][(warp << 5) + owner], 1u << (16 * (e & 1) + k));
+  }
+  __syncwarp();
+}
+
+// Experts loaded before the keep masks are drawn (fp32 groups are twice the
+// registers: two, so that nothing spills).
+template <int DT>
+constexpr int kDarePrefetch = DT == DT_BF16 ? kExpertBatch : 2;
+
+// DARE + TA on one 16-element group whose t0 and first kDarePrefetch experts
+// are already loaded; keep masks from shared memory (masked) or all kept.
+template <int DT>
+__device__ __forceinline__ void dare_linear16(const MArgs& m, const MTensor& T, int t, int64_t i, bool masked,
+                                              const Raw16<DT>& t0, Raw16<DT> (&x)[kExpertBatch],
+                                              const DareShared& s) {
+  float2 acc[8];
+#pragma unroll
+  for (int h = 0; h < 8; ++h) acc[h] = splat(0.0f);
+  const void* const* xp = m.experts + t * m.K;
+#pragma unroll 1
+  for (int e = 0; e < m.K; e += kExpertBatch) {
+#pragma unroll
+    for (int b = 0; b < kExpertBatch; ++b)
+      if ((e > 0 || b >= kDarePrefetch<DT>) && e + b < m.K) load16<DT>(xp[e + b], i, x[b]);
+#pragma unroll
+    for (int b = 0; b < kExpertBatch; ++b) {
+      if (e + b < m.K) {
+        const int ee = e + b;
+        const uint32_t keep = masked ? (s.keep[ee >> 1][threadIdx.x] >> (16 * (ee & 1))) & 0xFFFFu : 0xFFFFu;
+        merge_acc16<DT>(m.c, keep, x[b], t0, acc);
+      }
+    }
+  }
+  store_merged16<DT>(T, i, t0, acc);
 }
 
 // TIES on one 16-element group: elect, then the disjoint mean (the experts
@@ -261,10 +362,47 @@ __global__ void __launch_bounds__(kBlock, 2) merge_kernel(const __grid_constant_
         if (METHOD == SMAT_MERGE_TIES)
           merge_ties16<DT>(m, T, ch.tensor, i);
         else
-          merge_linear16<R, DT, METHOD>(m, T, ch.tensor, i);
+          merge_linear16<DT>(m, T, ch.tensor, i);
       } else {
         const int64_t e_end = (i + 16 < ch.end) ? i + 16 : ch.end;
         for (int64_t e = i; e < e_end; ++e) merge_elem<R, DT, METHOD>(m, T, ch.tensor, e);
+      }
+    }
+  }
+}
+
+// DARE + TA. The loop runs the same number of iterations on every lane of
+// the CTA (the keep masks are drawn warp-cooperatively); t0 and the first
+// experts are loaded before the masks are drawn, so the loads are in flight
+// during the Philox work.
+template <int R, int DT>
+__global__ void __launch_bounds__(kBlock, 2) dare_kernel(const __grid_constant__ MArgs m) {
+  __shared__ DareShared s;
+  const int warp = threadIdx.x >> 5;
+  for (int64_t ci = blockIdx.x; ci < m.n_chunks; ci += gridDim.x) {
+    const Chunk ch = m.chunks[ci];
+    const MTensor& T = m.tensors[ch.tensor];
+    const bool vec = (T.flags & TF_VEC) != 0u;
+    const bool masked = (T.flags & TF_MASK) != 0u;
+    const void* const* xp = m.experts + ch.tensor * m.K;
+    for (int64_t base = ch.begin; base < ch.end; base += 16 * (int64_t)kBlock) {
+      const int64_t i = base + 16 * (int64_t)threadIdx.x;
+      const bool full = vec && i + 16 <= ch.end;
+      Raw16<DT> t0, x[kExpertBatch];
+      if (full) {
+        load16<DT>(T.theta0, i, t0);
+#pragma unroll
+        for (int b = 0; b < kDarePrefetch<DT>; ++b)
+          if (b < m.K) load16<DT>(xp[b], i, x[b]);
+      }
+      if (masked)
+        dare_masks<R>(m, T, full, (uint64_t)(T.elem_offset + i),
+                      (uint64_t)(T.elem_offset + base + 16 * 32 * (int64_t)warp), s);
+      if (full) {
+        dare_linear16<DT>(m, T, ch.tensor, i, masked, t0, x, s);
+      } else if (i < ch.end) {
+        const int64_t e_end = (i + 16 < ch.end) ? i + 16 : ch.end;
+        for (int64_t e = i; e < e_end; ++e) merge_elem<R, DT, SMAT_MERGE_DARE_TA>(m, T, ch.tensor, e);
       }
     }
   }
@@ -371,7 +509,7 @@ cudaError_t merge_method(const MArgs& m, int grid, cudaStream_t s) {
   switch (m.method) {
     case SMAT_MERGE_WA: merge_kernel<R, DT, SMAT_MERGE_WA><<<grid, kBlock, 0, s>>>(m); break;
     case SMAT_MERGE_TA: merge_kernel<R, DT, SMAT_MERGE_TA><<<grid, kBlock, 0, s>>>(m); break;
-    case SMAT_MERGE_DARE_TA: merge_kernel<R, DT, SMAT_MERGE_DARE_TA><<<grid, kBlock, 0, s>>>(m); break;
+    case SMAT_MERGE_DARE_TA: dare_kernel<R, DT><<<grid, kBlock, 0, s>>>(m); break;
     default: merge_kernel<R, DT, SMAT_MERGE_TIES><<<grid, kBlock, 0, s>>>(m); break;
   }
   return cudaGetLastError();
