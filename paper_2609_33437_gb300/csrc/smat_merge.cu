@@ -408,45 +408,67 @@ __global__ void __launch_bounds__(kBlock, 2) dare_kernel(const __grid_constant__
   }
 }
 
-// One radix pass of the TIES threshold selection: work items are (chunk,
-// expert) pairs.
+// One radix pass of the TIES threshold selection. A work item is a chunk
+// and up to kHistExperts of its experts: theta0 is read once for them, and
+// each thread has theta0's and every expert's 32-byte load in flight at once;
+// one shared-memory histogram per expert, flushed into the 64-bit global bins.
+constexpr int kHistExperts = 4;
+
 template <int DT>
 __global__ void __launch_bounds__(kBlock) ties_hist_kernel(const __grid_constant__ MArgs m) {
-  __shared__ uint32_t h[kHistBins];
-  const int64_t items = m.n_chunks * m.K;
+  __shared__ uint32_t h[kHistExperts * kHistBins];
+  const int nbat = (m.K + kHistExperts - 1) / kHistExperts;
+  const int64_t items = m.n_chunks * nbat;
   const uint32_t digit = (1u << m.width) - 1u;
   for (int64_t w = blockIdx.x; w < items; w += gridDim.x) {
-    const int64_t ci = w / m.K;
-    const int e = (int)(w % m.K);
+    const int64_t ci = w / nbat;
+    const int e0 = (int)(w % nbat) * kHistExperts;
+    const int ne = m.K - e0 < kHistExperts ? m.K - e0 : kHistExperts;
     const Chunk ch = m.chunks[ci];
     const MTensor& T = m.tensors[ch.tensor];
-    const int slot = ch.tensor * m.K + e;
-    for (int b = threadIdx.x; b < kHistBins; b += kBlock) h[b] = 0u;
+    const int slot0 = ch.tensor * m.K + e0;
+    for (int b = threadIdx.x; b < kHistExperts * kHistBins; b += kBlock) h[b] = 0u;
     __syncthreads();
-    const uint32_t P = m.prefix[slot];
-    const void* xp = m.experts[slot];
+    uint32_t P[kHistExperts];
+    const void* xp[kHistExperts];
+#pragma unroll
+    for (int b = 0; b < kHistExperts; ++b) {
+      P[b] = b < ne ? m.prefix[slot0 + b] : 0u;
+      xp[b] = b < ne ? m.experts[slot0 + b] : nullptr;
+    }
     const bool vec = (T.flags & TF_VEC) != 0u;
     for (int64_t i = ch.begin + 16 * (int64_t)threadIdx.x; i < ch.end; i += 16 * (int64_t)kBlock) {
       if (vec && i + 16 <= ch.end) {
-        Raw16<DT> t0, x;
+        Raw16<DT> t0, x[kHistExperts];
         load16<DT>(T.theta0, i, t0);
-        load16<DT>(xp, i, x);
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
-          const uint32_t key = abs_key(__fsub_rn(x.at(k), t0.at(k)));
-          if ((key & m.decided) == P) atomicAdd(&h[(key >> m.shift) & digit], 1u);
+        for (int b = 0; b < kHistExperts; ++b)
+          if (b < ne) load16<DT>(xp[b], i, x[b]);
+#pragma unroll
+        for (int b = 0; b < kHistExperts; ++b) {
+          if (b < ne) {
+#pragma unroll
+            for (int k = 0; k < 16; ++k) {
+              const uint32_t key = abs_key(__fsub_rn(x[b].at(k), t0.at(k)));
+              if ((key & m.decided) == P[b]) atomicAdd(&h[b * kHistBins + ((key >> m.shift) & digit)], 1u);
+            }
+          }
         }
       } else {
         const int64_t e_end = (i + 16 < ch.end) ? i + 16 : ch.end;
         for (int64_t k = i; k < e_end; ++k) {
-          const uint32_t key = abs_key(__fsub_rn(load1<DT>(xp, k), load1<DT>(T.theta0, k)));
-          if ((key & m.decided) == P) atomicAdd(&h[(key >> m.shift) & digit], 1u);
+          const float t0 = load1<DT>(T.theta0, k);
+          for (int b = 0; b < ne; ++b) {
+            const uint32_t key = abs_key(__fsub_rn(load1<DT>(xp[b], k), t0));
+            if ((key & m.decided) == P[b]) atomicAdd(&h[b * kHistBins + ((key >> m.shift) & digit)], 1u);
+          }
         }
       }
     }
     __syncthreads();
-    unsigned long long* gh = m.hist + (size_t)slot * kHistBins;
-    for (int b = threadIdx.x; b < kHistBins; b += kBlock)
+    // the ne histograms are consecutive slots' bins in the global array
+    unsigned long long* gh = m.hist + (size_t)slot0 * kHistBins;
+    for (int b = threadIdx.x; b < ne * kHistBins; b += kBlock)
       if (h[b]) atomicAdd(gh + b, (unsigned long long)h[b]);
     __syncthreads();
   }
@@ -607,8 +629,12 @@ smat_status merge_check(const smat_merge_tensor* t, int32_t n, const smat_merge_
 template <int R, int DT>
 cudaError_t merge_launch(MArgs m, int64_t slots, bool ties, int sms, cudaStream_t s) {
   if (ties) {
-    const int64_t items = m.n_chunks * m.K;
-    const int hgrid = (int)(items < 4 * (int64_t)sms ? items : 4 * (int64_t)sms);
+    const int64_t items = m.n_chunks * ((m.K + kHistExperts - 1) / kHistExperts);
+    int occ = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, ties_hist_kernel<DT>, kBlock, 0) != cudaSuccess || occ < 1)
+      occ = 1;
+    const int64_t resident = (int64_t)occ * sms;
+    const int hgrid = (int)(items < resident ? items : resident);
     for (int p = 0; p < kPasses; ++p) {
       m.shift = kPassShift[p];
       m.width = kPassWidth[p];
