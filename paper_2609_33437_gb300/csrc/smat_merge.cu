@@ -247,7 +247,11 @@ __device__ __forceinline__ void dare_linear16(const MArgs& m, const MTensor& T, 
 }
 
 // TIES on one 16-element group: elect, then the disjoint mean (the experts
-// are read twice; the second read is served by the L2).
+// are read twice; the second read is served by the L2). The oracle's
+// agreement test, abs(Delta) >= thr and (sum > 0 and Delta > 0 or sum < 0 and
+// Delta < 0), is taken as: key in [max(thr, 1), key(+inf)] (Delta nonzero,
+// not NaN) and equal sign bits of Delta and sum; elements whose sum is 0 or
+// NaN, where the oracle finds no agreeing expert, are set to 0 at the end.
 template <int DT>
 __device__ __forceinline__ void merge_ties16(const MArgs& m, const MTensor& T, int t, int64_t i) {
   Raw16<DT> t0;
@@ -259,9 +263,11 @@ __device__ __forceinline__ void merge_ties16(const MArgs& m, const MTensor& T, i
   for (int k = 0; k < 16; ++k) sum[k] = 0.0f;
   auto elect = [&](const Raw16<DT>& x, uint32_t thr) {
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
-      const float d = __fsub_rn(x.at(k), t0.at(k));
-      if (abs_key(d) >= thr) sum[k] = __fadd_rn(sum[k], d);
+    for (int h = 0; h < 8; ++h) {
+      const float2 b = t0.pair(h);
+      const float2 d = add2_rn(x.pair(h), make_float2(-b.x, -b.y));
+      if (abs_key(d.x) >= thr) sum[2 * h] = __fadd_rn(sum[2 * h], d.x);
+      if (abs_key(d.y) >= thr) sum[2 * h + 1] = __fadd_rn(sum[2 * h + 1], d.y);
     }
   };
   int e = 0;
@@ -283,14 +289,24 @@ __device__ __forceinline__ void merge_ties16(const MArgs& m, const MTensor& T, i
   uint32_t cnt[4] = {0u, 0u, 0u, 0u};  // four 8-bit counts per word (K <= 16)
 #pragma unroll
   for (int k = 0; k < 16; ++k) part[k] = 0.0f;
+  constexpr uint32_t kInfKey = 0x7F800000u;
+  auto agree = [&](float d, uint32_t lo, int k) {
+    const uint32_t key = abs_key(d);
+    return key >= lo && key <= kInfKey && ((__float_as_uint(d) ^ __float_as_uint(sum[k])) & 0x80000000u) == 0u;
+  };
   auto gather = [&](const Raw16<DT>& x, uint32_t thr) {
+    const uint32_t lo = thr > 1u ? thr : 1u;
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
-      const float d = __fsub_rn(x.at(k), t0.at(k));
-      const bool agree = abs_key(d) >= thr && ((sum[k] > 0.0f && d > 0.0f) || (sum[k] < 0.0f && d < 0.0f));
-      if (agree) {
-        part[k] = __fadd_rn(part[k], d);
-        cnt[k >> 2] += 1u << (8 * (k & 3));
+    for (int h = 0; h < 8; ++h) {
+      const float2 b = t0.pair(h);
+      const float2 d = add2_rn(x.pair(h), make_float2(-b.x, -b.y));
+      if (agree(d.x, lo, 2 * h)) {
+        part[2 * h] = __fadd_rn(part[2 * h], d.x);
+        cnt[h >> 1] += 1u << (16 * (h & 1));
+      }
+      if (agree(d.y, lo, 2 * h + 1)) {
+        part[2 * h + 1] = __fadd_rn(part[2 * h + 1], d.y);
+        cnt[h >> 1] += 1u << (16 * (h & 1) + 8);
       }
     }
   };
@@ -313,7 +329,8 @@ __device__ __forceinline__ void merge_ties16(const MArgs& m, const MTensor& T, i
 #pragma unroll
   for (int k = 0; k < 16; ++k) {
     const uint32_t n = (cnt[k >> 2] >> (8 * (k & 3))) & 0xFFu;
-    const float merged = n ? __fdiv_rn(part[k], (float)n) : 0.0f;
+    const bool elected = sum[k] > 0.0f || sum[k] < 0.0f;
+    const float merged = (n && elected) ? __fdiv_rn(part[k], (float)n) : 0.0f;
     out[k] = __fadd_rn(t0.at(k), __fmul_rn(m.gamma, merged));
   }
   store16<DT>(T.out, i, out);

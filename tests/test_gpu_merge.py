@@ -10,7 +10,7 @@ import torch
 import oracle as O
 from paper_2609_33437_gb300 import smat as S
 
-from _parity import to_host
+from _parity import f32_of, to_host
 
 pytestmark = pytest.mark.gpu
 
@@ -136,3 +136,37 @@ def test_merge_dare_seven_rounds():
         ref, _ = O.merge(O.MERGE_DARE_TA, to_host(t0), [to_host(x) for x in ex], dtype=O.BF16, gamma=0.5,
                          p_drop=0.3, seed=8, tensor_id=k, rounds=7)
         assert np.array_equal(to_host(out).view(np.uint16), ref.view(np.uint16)), k
+
+
+@pytest.mark.parametrize("method", list(METHODS))
+@pytest.mark.parametrize("dtype", [O.F32, O.BF16])
+def test_merge_special_values(method, dtype):
+    """Signed zeros, infinities, NaN, subnormals and experts equal to theta0
+    sprinkled into theta0 and the experts: every result equals the oracle's
+    bit for bit, NaN matching any NaN (payloads differ between host and GPU).
+    Retention keeps the TIES thresholds among the finite keys."""
+    n, K = 20_000 + 7, 5
+    g = torch.Generator().manual_seed(23)
+    t0 = torch.randn(n, generator=g) * 0.02
+    ex = [t0 + torch.randn(n, generator=g) * 1e-3 for _ in range(K)]
+    specials = torch.tensor([0.0, -0.0, float("inf"), float("-inf"), float("nan"), 1e-40, -1e-40, 3e-39])
+    for arr in [t0] + ex:
+        pos = torch.randint(0, n, (n // 50,), generator=g)
+        arr[pos] = specials[torch.randint(0, len(specials), (len(pos),), generator=g)]
+    for e in range(K):  # Delta exactly 0 on a few coordinates
+        pos = torch.randint(0, n, (n // 100,), generator=g)
+        ex[e][pos] = t0[pos]
+    tdt = torch.bfloat16 if dtype == O.BF16 else torch.float32
+    t0d = t0.to(tdt).cuda()
+    exd = [x.to(tdt).cuda() for x in ex]
+    out = torch.empty_like(t0d)
+    kw = dict(gamma=0.7, p_drop=0.3, retention=0.3, seed=4)
+    S.merge([t0d], [exd], [out], method, **kw)
+    torch.cuda.synchronize()
+    ref, _ = O.merge(METHODS[method], to_host(t0d), [to_host(x) for x in exd], dtype=dtype, tensor_id=0, **kw)
+    got = to_host(out)
+    gf, rf = f32_of(got), f32_of(ref)
+    view = np.uint16 if dtype == O.BF16 else np.uint32
+    nan_g, nan_r = np.isnan(gf), np.isnan(rf)
+    assert np.array_equal(nan_g, nan_r)
+    assert np.array_equal(got.view(view)[~nan_g], ref.view(view)[~nan_r])
