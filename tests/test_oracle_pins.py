@@ -700,3 +700,32 @@ def test_merge_ties_threshold_is_the_rth_largest_magnitude():
             d = np.abs(ex[j] - t0)
             ref = np.sort(d)[::-1][min(n, max(1, math.ceil(k * n))) - 1]
             assert thr.view(np.float32)[j] == ref
+
+
+def test_merge_ties_degenerate_cases():
+    """TIES reduces to simpler merges in degenerate cases. One expert with no
+    trimming is TA with that expert: its own sign is elected and the mean of
+    one value is that value. Four identical experts give the same, exactly,
+    since 4 Delta and 4 Delta / 4 are exact in fp32. Two opposite experts
+    cancel: the sum is 0, no sign is elected and theta0 is kept. A NaN Delta
+    makes the elected sum NaN, so theta0 is kept. A +inf among positive
+    Deltas elects + and the mean is +inf."""
+    r = rng(33)
+    n = 513
+    t0 = _dyadic(r, n)
+    x = _dyadic(r, n)
+    ta, _ = O.merge(O.MERGE_TA, t0, [x], gamma=0.5)
+    one, _ = O.merge(O.MERGE_TIES, t0, [x], gamma=0.5, retention=1.0)
+    assert np.array_equal(one.view(np.uint32), ta.view(np.uint32))
+    four, _ = O.merge(O.MERGE_TIES, t0, [x] * 4, gamma=0.5, retention=1.0)
+    assert np.array_equal(four.view(np.uint32), ta.view(np.uint32))
+    z = np.zeros(n, np.float32)
+    cancel, _ = O.merge(O.MERGE_TIES, z, [x, -x], gamma=0.5, retention=1.0)
+    assert np.array_equal(cancel.view(np.uint32), z.view(np.uint32))
+    z4 = np.zeros(4, np.float32)
+    nan = np.array([np.nan, 1, 1, 1], np.float32)
+    out, _ = O.merge(O.MERGE_TIES, z4, [nan, np.ones(4, np.float32)], gamma=0.5, retention=1.0)
+    assert np.array_equal(out, np.array([0, 0.5, 0.5, 0.5], np.float32))
+    inf = np.array([np.inf, 2, 2, 2], np.float32)
+    out, _ = O.merge(O.MERGE_TIES, z4, [inf, np.ones(4, np.float32)], gamma=0.5, retention=1.0)
+    assert np.array_equal(out, np.array([np.inf, 0.75, 0.75, 0.75], np.float32))
