@@ -227,3 +227,53 @@ def test_merge_host_validation(L):
     b = tens(dtype=S.SMAT_BF16)
     b.tensor_id = 1
     assert ws([tens(), b]) == 0  # one dtype per call
+
+
+def test_binding_matches_header_layout(tmp_path):
+    """The ctypes binding agrees with include/smat.h as a C compiler reads it:
+    the size and every field offset of each struct, the value of each constant
+    the binding defines, and the parameter count of each function it
+    declares."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no host C compiler")
+    structs = {"smat_tensor_desc": S.TensorDesc, "smat_config": S.Config,
+               "smat_merge_tensor": S.MergeTensor, "smat_merge_config": S.MergeConfig}
+    consts = ["SMAT_F32", "SMAT_BF16", "SMAT_NOISE_UNIFORM", "SMAT_NOISE_GAUSSIAN", "SMAT_NOISE_LAPLACE",
+              "SMAT_ALPHA_GLOBAL", "SMAT_ALPHA_PER_TENSOR", "SMAT_ALPHA_PER_ELEMENT", "SMAT_FLAG_UNFUSED_STATS",
+              "SMAT_MERGE_WA", "SMAT_MERGE_TA", "SMAT_MERGE_DARE_TA", "SMAT_MERGE_TIES"]
+    src = ["#include <stddef.h>", "#include <stdio.h>", '#include "smat.h"', "int main(void) {"]
+    for cname, py in structs.items():
+        src.append(f'printf("{cname} . %zu\\n", sizeof({cname}));')
+        src += [f'printf("{cname} {f} %zu\\n", offsetof({cname}, {f}));' for f, _ in py._fields_]
+    src += [f'printf("const {c} %lld\\n", (long long)({c}));' for c in consts]
+    src += [f'printf("const SMAT_FLAG_CHUNK_LOG2({k}) %lld\\n", (long long)SMAT_FLAG_CHUNK_LOG2({k}));'
+            for k in (12, 18)]
+    src.append("return 0; }")
+    c_file, exe = tmp_path / "layout.c", tmp_path / "layout"
+    c_file.write_text("\n".join(src) + "\n")
+    subprocess.run([cc, "-std=c11", "-Wall", "-Werror", "-I", os.path.join(ROOT, "include"), str(c_file), "-o",
+                    str(exe)], check=True, capture_output=True)
+    seen = {}
+    for line in subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.splitlines():
+        a, b, v = line.split(" ")
+        seen[(a, b)] = int(v)
+    for cname, py in structs.items():
+        assert ctypes.sizeof(py) == seen[(cname, ".")], cname
+        for f, _ in py._fields_:
+            assert getattr(py, f).offset == seen[(cname, f)], (cname, f)
+    for c in consts:
+        assert getattr(S, c) == seen[("const", c)], c
+    for k in (12, 18):
+        assert S.SMAT_FLAG_CHUNK_LOG2(k) == seen[("const", f"SMAT_FLAG_CHUNK_LOG2({k})")]
+    # parameter counts of the declarations against the binding's argtypes
+    hdr = re.sub(r"/\*.*?\*/", "", open(os.path.join(ROOT, "include", "smat.h")).read(), flags=re.S)
+    lib = S.load_library()
+    for name, params in re.findall(r"\b(smat_[a-z0-9_]+)\s*\(([^()]*)\)\s*;", hdr):
+        argtypes = getattr(lib, name).argtypes
+        if argtypes is None:
+            continue
+        n = 0 if params.strip() in ("", "void") else params.count(",") + 1
+        assert len(argtypes) == n, name
