@@ -80,6 +80,8 @@ def parse():
     ap.add_argument("--merge", choices=["wa", "ta", "dare", "ties"], default=None,
                     help="time merging K experts of the chosen list (Eq. merged-state) instead of the SMAT step")
     ap.add_argument("--experts", type=int, default=8)
+    ap.add_argument("--ref-sample", type=int, default=0,
+                    help="elements per step of the oracle sample in --impl reference (0: sized for about 150 s)")
     ap.add_argument("--schedule", action="store_true",
                     help="training-loop overhead of periodic SMAT (Sec. 4.3) over plain fine-tuning, synthetic model")
     return ap.parse_args()
@@ -278,6 +280,8 @@ def run_reference(args):
     # about 150 s in all: the oracle takes about 1 us per element (forward +
     # gradient map on one Grace core) plus the sample's input generation
     per_step = int(min(8_000_000, max(200_000, 150.0 / max(1, args.steps + args.warmup) / 1.1e-6)))
+    if args.ref_sample > 0:
+        per_step = args.ref_sample
     for _ in range(args.warmup):
         oracle_run(w, per_step)
     tot_s, tot_b, tot_n = 0.0, 0, 0
