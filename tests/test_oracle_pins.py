@@ -292,6 +292,71 @@ def test_alpha_uniform_per_tensor_and_global():
     assert len(pa) == 20
 
 
+def _alpha_per_element(cfg, tid, n, elem_offset=0):
+    """Per-element alpha of n coordinates, read through the gradient map: with
+    p_keep = 1 every coordinate is kept and rescaled by 1, so g~ = 1 maps to
+    alpha_i itself (Eq. smat-gradient)."""
+    t = O.tensor(tid, n, keep_prob=1.0, elem_offset=elem_offset)
+    return O.gradmap(cfg, t, np.ones(n, np.float32)).astype(np.float64)
+
+
+@pytest.mark.parametrize("amin,amax", [(0.0, 1.0), (0.3, 0.8)])
+def test_alpha_per_element_law(amin, amax):
+    """Scale per coordinate (Sec. 4.1, reading R4): alpha_i ~ U[alpha_min,
+    alpha_max), independent across coordinates (lags inside and across the
+    4-coordinate draw blocks) and independent of the same coordinate's Mask and
+    Perturb draws."""
+    n = 1 << 18
+    cfg = O.config(seed=31, step=3, alpha_mode=O.ALPHA_PER_ELEMENT, alpha_min=amin, alpha_max=amax,
+                   noise=O.NOISE_GAUSSIAN)
+    a = _alpha_per_element(cfg, 40, n)
+    assert a.min() >= amin and a.max() < amax
+    assert stats.kstest((a - amin) / (amax - amin), "uniform").pvalue > 1e-4
+    assert abs(a.mean() - (amin + amax) / 2) < 5 * (amax - amin) / math.sqrt(12 * n)
+    se = 1 / math.sqrt(n)
+    for lag in (1, 2, 3, 4, 5, 8, 16):
+        assert abs(np.corrcoef(a[:-lag], a[lag:])[0, 1]) < 5 * se, lag
+    # Mask of the same coordinates at p_keep = 1/2
+    kept = O.unpack_bits(O.mask_bits(cfg, O.tensor(40, n, keep_prob=0.5)), n).astype(np.float64)
+    assert abs(np.corrcoef(a, kept)[0, 1]) < 5 * se
+    # Perturb of the same coordinates
+    z = O.noise_z(cfg, O.tensor(40, n, keep_prob=1.0, sigma=1.0), np.arange(n))
+    assert abs(np.corrcoef(a, z)[0, 1]) < 5 * se
+    assert abs(np.corrcoef(a, np.abs(z))[0, 1]) < 5 * se
+    # and the kept rescaled coordinates carry alpha_i / p_keep
+    g = O.gradmap(cfg, O.tensor(40, n, keep_prob=0.5), np.ones(n, np.float32)).astype(np.float64)
+    on = kept.astype(bool)
+    assert np.array_equal(g[on], (a[on].astype(np.float32) * np.float32(2.0)).astype(np.float64))
+    assert np.all(g[~on] == 0.0)
+
+
+def test_alpha_per_element_stream_layout_matches_triton_library():
+    """Coordinate gidx's alpha comes from word gidx mod 4 of the ALPHA_E
+    (stream 2) block gidx div 4: (alpha_i - alpha_min) / (alpha_max - alpha_min)
+    equals the top 24 bits of that word of Triton's Philox block, scaled by
+    2^-24, to within the fp32 rounding of the affine map. Covers element
+    offsets and draw-block indices at and above 2^32 (counter word 1)."""
+    seed, step, tid, amin, amax = 0x0DDB1A5E5BADDEC0, 6, 0x0ABCDEF, 0.25, 0.875
+    cfg = O.config(seed=seed, step=step, alpha_mode=O.ALPHA_PER_ELEMENT, alpha_min=amin, alpha_max=amax)
+    cases = [(0, 40), (13, 19), ((1 << 34) - 6, 12), (5 << 34, 8)]
+    ctrs, gidx, alphas = [], [], []
+    for off, n in cases:
+        a = _alpha_per_element(cfg, tid, n, elem_offset=off)
+        for i in range(n):
+            g = off + i
+            gidx.append(g)
+            alphas.append(a[i])
+            j = g >> 2
+            ctrs.append([j & 0xFFFFFFFF, j >> 32, (2 << 28) | tid, step])
+    words = _triton_philox(ctrs, [seed] * len(ctrs), 10)
+    u = np.array([(int(words[k][g & 3]) >> 8) * 2.0**-24 for k, g in enumerate(gidx)])
+    back = (np.array(alphas) - amin) / (amax - amin)
+    assert np.all(np.abs(back - u) <= 2.0**-22), np.max(np.abs(back - u))
+    # a neighbouring word would be another, unrelated uniform
+    wrong = np.array([(int(words[k][(g + 1) & 3]) >> 8) * 2.0**-24 for k, g in enumerate(gidx)])
+    assert np.mean(np.abs(back - wrong) <= 2.0**-22) < 0.1
+
+
 def test_uniform_noise_law():
     """Perturb: eps ~ U[-sqrt3 sigma, sqrt3 sigma] (Sec. 4.1): with theta0 = 0 and
     every coordinate dropped, theta~ = eps exactly; mean 0, variance sigma^2,
@@ -436,6 +501,44 @@ def test_state_moments_proposition():
         assert abs(prod.mean() - ref) < 5 * prod.std() / math.sqrt(steps), (k, l)
 
 
+def test_state_moments_proposition_per_element_alpha():
+    """Prop. moments (App. C) with alpha drawn per coordinate (reading R4):
+    the mean is still theta0 + abar Delta and each coordinate's variance is
+    v_a Delta^2 + s_a Delta^2 p/(1-p) + sigma^2, but coordinates no longer
+    share a scale, so every off-diagonal covariance is 0 (the shared-alpha
+    term v_a Delta_k Delta_l of the global mode vanishes)."""
+    r = rng(32)
+    n, steps = 24, 6000
+    amin, pk, sigma = 0.2, 0.6, 0.05
+    t0 = r.standard_normal(n).astype(np.float32)
+    delta = (r.standard_normal(n) * 0.5 + np.sign(r.standard_normal(n))).astype(np.float32)
+    th = (t0 + delta).astype(np.float32)
+    D = (th - t0).astype(np.float64)
+    X = np.zeros((steps, n))
+    for s in range(steps):
+        cfg = O.config(seed=13, step=s, alpha_mode=O.ALPHA_PER_ELEMENT, alpha_min=amin, alpha_max=1.0)
+        X[s] = O.simulate(cfg, O.tensor(3, n, keep_prob=pk, sigma=sigma), th, t0)
+    abar = (1 + amin) / 2
+    va = (1 - amin) ** 2 / 12
+    sa = abar**2 + va
+    p_drop = 1 - pk
+    mean_ref = t0 + abar * D
+    var_ref = va * D**2 + sa * D**2 * p_drop / (1 - p_drop) + sigma**2
+    mean = X.mean(0)
+    assert np.all(np.abs(mean - mean_ref) < 5 * np.sqrt(var_ref / steps))
+    var = X.var(0)
+    m4 = ((X - mean) ** 4).mean(0)
+    assert np.all(np.abs(var - var_ref) < 5 * np.sqrt((m4 - var**2) / steps) + 1e-12)
+    Xc = X - mean
+    for (k, l) in ((0, 1), (2, 3), (4, 7), (5, 19), (10, 11), (15, 16)):
+        prod = Xc[:, k] * Xc[:, l]
+        assert abs(prod.mean()) < 5 * prod.std() / math.sqrt(steps), (k, l)
+    # the shared-alpha covariance of the global mode is far outside that band
+    big = max(((k, l) for k in range(n) for l in range(k + 1, n)), key=lambda kl: abs(D[kl[0]] * D[kl[1]]))
+    prod = Xc[:, big[0]] * Xc[:, big[1]]
+    assert abs(va * D[big[0]] * D[big[1]]) > 5 * prod.std() / math.sqrt(steps)
+
+
 # ---------------------------------------------- gradient (Eq. smat-gradient) ---
 
 @pytest.mark.parametrize("mode", [O.ALPHA_PER_TENSOR, O.ALPHA_PER_ELEMENT])
@@ -554,6 +657,39 @@ def test_simulate_at_matches_full_tensor():
     idx = r.choice(n, 300, replace=False)
     bits, _ = O.simulate_at(cfg, t, sig, idx, O.bf16_to_f32(th[idx]), O.bf16_to_f32(t0[idx]))
     assert np.array_equal(bits.astype(np.uint16), full[idx])
+
+
+@pytest.mark.parametrize("dtype", [O.F32, O.BF16])
+@pytest.mark.parametrize("mode", [O.ALPHA_GLOBAL, O.ALPHA_PER_TENSOR, O.ALPHA_PER_ELEMENT])
+@pytest.mark.parametrize("noise", [O.NOISE_UNIFORM, O.NOISE_GAUSSIAN, O.NOISE_LAPLACE])
+def test_at_index_evaluation_matches_full_tensor(dtype, mode, noise):
+    """The sampled evaluations (simulate_at, gradmap_at: what the full-size GPU
+    checks compare against) give the bits of the whole-tensor forward and
+    gradient map at every sampled index, with an element offset, mask ties in
+    range, and with and without accumulation."""
+    r = rng(41 + 3 * mode + noise)
+    n, off = 3001, (1 << 33) + 7
+    th = r.standard_normal(n).astype(np.float32) * np.float32(0.02)
+    t0 = r.standard_normal(n).astype(np.float32) * np.float32(0.02)
+    gs = r.standard_normal(n).astype(np.float32)
+    go = r.standard_normal(n).astype(np.float32)
+    if dtype == O.BF16:
+        th, t0, gs, go = O.f32_to_bf16(th), O.f32_to_bf16(t0), O.f32_to_bf16(gs), O.f32_to_bf16(go)
+    f = (lambda x: O.bf16_to_f32(x)) if dtype == O.BF16 else (lambda x: x)
+    cfg = O.config(seed=77, step=9, alpha_mode=mode, noise=noise, alpha_min=0.1, alpha_max=0.9)
+    t = O.tensor(31, n, dtype=dtype, keep_prob=0.5 + 2.0**-10, sigma=3e-3, elem_offset=off)
+    idx = np.sort(r.choice(n, 700, replace=False))
+    bits_t = np.uint16 if dtype == O.BF16 else np.uint32
+    full = O.simulate(cfg, t, th, t0).view(bits_t)
+    bits, kept = O.simulate_at(cfg, t, 3e-3, idx, f(th)[idx], f(t0)[idx])
+    assert np.array_equal(bits.astype(bits_t), full[idx])
+    mb = O.unpack_bits(O.mask_bits(cfg, t), n)
+    assert np.array_equal(kept, mb[idx])
+    for acc in (False, True):
+        gfull = O.gradmap(cfg, t, gs, gdtype=dtype, accumulate=acc, g_old=go if acc else None).view(bits_t)
+        gat = O.gradmap_at(cfg, t, idx, f(gs)[idx], gdtype=dtype, accumulate=acc,
+                           gold_vals=f(go)[idx] if acc else None)
+        assert np.array_equal(gat.astype(bits_t), gfull[idx]), acc
 
 
 def test_delta_stats_match_numpy():
