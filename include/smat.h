@@ -131,10 +131,15 @@ size_t smat_workspace_bytes(const smat_tensor_desc* tensors, int32_t n_tensors,
                             const smat_config* cfg);
 
 /* Validate the list, build the tables and upload them into d_workspace on
- * `stream`. d_workspace: caller-owned device memory of at least
- * smat_workspace_bytes(...) bytes, 256-byte aligned, untouched by the caller
- * until smat_destroy. On success *out receives a new context, initially with
- * the original storage (theta) active. */
+ * `stream`. The list is the set of trainable tensors SMAT simulates (Sec. 4.1:
+ * Perturb acts on every trainable coordinate; the Mask set, p_keep < 1, is the
+ * attention and MLP linear weights), each with its own Mask rate (Eq.
+ * smat-mask) and Perturb RMS; the configuration holds the Scale range and
+ * granularity (Sec. 4.1, App. A) and the Philox key. d_workspace: caller-owned
+ * device memory of at least smat_workspace_bytes(...) bytes, 256-byte aligned,
+ * untouched by the caller until smat_destroy. On success *out receives a new
+ * context, initially with the original storage (theta) active (Sec. 4.3) and
+ * no forward run yet. */
 smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n_tensors,
                       const smat_config* cfg, void* d_workspace, size_t workspace_bytes,
                       smat_stream_t stream);
@@ -160,7 +165,11 @@ smat_status smat_simulate_multi(smat_ctx* ctx, uint32_t step, smat_stream_t stre
  * same order as the descriptors; an entry may be NULL only if numel == 0).
  * g_out[k] may equal g_sim[k] (in place). The pointer table is uploaded only
  * when it differs from the previous call's. The mask is regenerated from the
- * stream, never stored. */
+ * stream, never stored (App. D, implementation details), so it must be the
+ * mask of the forward that produced the theta~ the gradient was taken at:
+ * `step` must be the step of the last smat_simulate_multi on this context
+ * (SMAT_ERR_STATE otherwise, including when no forward has run). Any number of
+ * gradient maps may follow one forward (gradient accumulation). */
 smat_status smat_grad_map_multi(smat_ctx* ctx, uint32_t step, const void* const* g_sim,
                                 void* const* g_out, int32_t gdtype, int32_t accumulate,
                                 smat_stream_t stream);
@@ -188,16 +197,21 @@ smat_status smat_mark_theta0_resident(smat_ctx* ctx);
 /* Which storage is active (0 = theta, 1 = sim). */
 smat_status smat_active(const smat_ctx* ctx, int32_t* active_out);
 
-/* Test hook: packed keep bits of tensor `tensor_index` at `step` into the
- * device buffer d_bits of ceil(numel / 32) uint32 words; bit (i mod 32) of
- * word i / 32 is 1 iff local element i is kept (LSB first; high bits of the
- * last word 0). */
+/* Test hook: the Mask of Eq. smat-mask (m_i != 0, i.e. coordinate i kept
+ * with probability p_keep = 1 - p) of tensor `tensor_index` at `step`, as
+ * packed bits into the device buffer d_bits of ceil(numel / 32) uint32 words;
+ * bit (i mod 32) of word i / 32 is 1 iff local element i is kept (LSB first;
+ * high bits of the last word 0). Any step may be asked for: the bits are
+ * regenerated from the stream, as the gradient map does (App. D). */
 smat_status smat_mask_bits(smat_ctx* ctx, uint32_t step, int32_t tensor_index, uint32_t* d_bits,
                            smat_stream_t stream);
 
 /* Test hook: per-call scalars at `step` into the device buffer d_out of
  * 4 * n_tensors floats: {alpha_t, c_t = alpha_t / p_keep, sigma_t,
- * noise scale} per tensor (alpha_t and c_t are 0 in per-element mode).
+ * noise scale} per tensor (alpha_t and c_t are 0 in per-element mode):
+ * alpha_t is the Scale draw (Sec. 4.1, alpha ~ U[alpha_min, alpha_max)), c_t
+ * its product with the Mask rescale 1 / (1 - p) of Eq. smat-mask, sigma_t the
+ * Perturb RMS (Sec. 4.1) and the noise scale the law's factor at that RMS.
  * Computes the delta statistics first for sigma_rel tensors (which, for
  * in-place sigma_rel tensors, needs theta0 resident: SMAT_ERR_STATE
  * otherwise). */

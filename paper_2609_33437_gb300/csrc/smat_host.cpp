@@ -237,6 +237,7 @@ struct smat_ctx {
   int64_t chunk_elems = kMaxChunkElems;  // work-chunk size of this list
   int32_t active = 0;
   int64_t scalars_step = -1;  // step whose scalars the table holds
+  int64_t sim_step = -1;      // step of the last forward: the only step whose mask a gradient map may regenerate
   bool scalars_sigma = false; // the table's sigma_t are current
   std::vector<GradPtr> h_grads;
   bool grads_uploaded = false;
@@ -517,6 +518,7 @@ smat_status smat_simulate_multi(smat_ctx* c, uint32_t step, smat_stream_t stream
   if (c->any_inplace && !c->theta0_resident)
     return fail(SMAT_ERR_STATE, "in-place tensors: theta0 has not been refilled since the last forward");
   c->theta0_resident = false;  // the forward below overwrites it
+  c->sim_step = -1;            // set again once every launch of this forward is enqueued
   if (c->fused) {
     // a1 (alpha, c; sigma of fixed-sigma tensors; counter reset), then a3 (with a2
     // for sigma_rel tensors) in one work-list launch
@@ -539,6 +541,7 @@ smat_status smat_simulate_multi(smat_ctx* c, uint32_t step, smat_stream_t stream
       t.done();
       if (e != cudaSuccess) return cuda_fail(e, "fused statistics + forward launch");
     }
+    c->sim_step = step;
     return SMAT_OK;
   }
   smat_status st = run_scalars(c, step, true, stream);
@@ -555,6 +558,7 @@ smat_status smat_simulate_multi(smat_ctx* c, uint32_t step, smat_stream_t stream
     t.done();
     if (e != cudaSuccess) return cuda_fail(e, "simulate launch");
   }
+  c->sim_step = step;
   return SMAT_OK;
 }
 
@@ -563,6 +567,14 @@ smat_status smat_grad_map_multi(smat_ctx* c, uint32_t step, const void* const* g
   if (!c) return fail(SMAT_ERR_INVALID_ARG, "ctx is NULL");
   if (gdtype != SMAT_F32 && gdtype != SMAT_BF16)
     return fail(SMAT_ERR_UNSUPPORTED, "gradient dtype %d not supported", gdtype);
+  // Eq. smat-gradient maps g~ through the mask of the forward that produced
+  // theta~ (regenerated, App. D): only the step of the last forward qualifies.
+  if (c->sim_step != (int64_t)step) {
+    if (c->sim_step < 0)
+      return fail(SMAT_ERR_STATE, "gradient map for step %u, but no forward has run on this context", step);
+    return fail(SMAT_ERR_STATE, "gradient map for step %u, but the last forward on this context was step %lld", step,
+                (long long)c->sim_step);
+  }
   const int32_t n = (int32_t)c->desc.size();
   if (n > 0 && (!g_sim || !g_out)) return fail(SMAT_ERR_INVALID_ARG, "gradient pointer arrays are NULL");
   const size_t es = elem_size(gdtype);
@@ -717,6 +729,7 @@ smat_status smat_debug_fused(smat_ctx* c, uint32_t step, const int32_t* d_items,
                                  c->cfg.noise, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT, c->rounds, stream);
   if (e != cudaSuccess) return cuda_fail(e, "fused launch");
   c->scalars_step = -1;  // sigma_t of this call may be incomplete
+  c->sim_step = -1;      // and its forward too
   return SMAT_OK;
 }
 

@@ -92,13 +92,26 @@ def test_philox_7_rounds_and_accumulate_and_f32_grads_on_bf16_params():
     run_and_check_full(w, steps=(1,), rounds=7, accumulate=True, gdtype=O.F32)
 
 
-def test_sweep_points_small_sizes():
-    """Flat-tensor sweep points at 2^16 and 2^18 (both dtypes, several keep
-    probabilities, both alpha modes, sigma 0 and 1e-4)."""
-    for log2n in (16, 18):
-        for dt in (O.F32, O.BF16):
-            for p, am, sig in ((0.1, 1, 0.0), (0.5, 2, 1e-4), (0.9, 1, 1e-4), (0.3, 2, 0.0)):
-                run_and_check_full(W.flat_sweep(log2n, dt, p, am, sig), steps=(0,))
+@pytest.mark.parametrize("sig", [0.0, 1e-4])
+@pytest.mark.parametrize("am", [O.ALPHA_PER_TENSOR, O.ALPHA_PER_ELEMENT])
+@pytest.mark.parametrize("dt", [O.F32, O.BF16])
+def test_sweep_grid_at_2_16(dt, am, sig):
+    """Every setting of the flat-tensor sweep (2 dtypes x 5 keep probabilities
+    x alpha per tensor or per element, U[0, 1) x sigma 0 or 1e-4, Gaussian) on
+    a 2^16-element tensor, element by element."""
+    for p in (0.1, 0.3, 0.5, 0.7, 0.9):
+        run_and_check_full(W.flat_sweep(16, dt, p, am, sig), steps=(0,))
+
+
+def test_sweep_points_2_18_and_2_20_small_chunks():
+    """Larger sweep points: 2^18 in both dtypes; 2^20 fp32 with per-element
+    alpha and noise on 2^12-element work chunks (256 chunks, each its own
+    rare-element queue)."""
+    for dt in (O.F32, O.BF16):
+        for p, am, sig in ((0.1, 1, 0.0), (0.5, 2, 1e-4), (0.9, 1, 1e-4), (0.3, 2, 0.0)):
+            run_and_check_full(W.flat_sweep(18, dt, p, am, sig), steps=(0,))
+    run_and_check_full(W.flat_sweep(20, O.F32, 0.7, O.ALPHA_PER_ELEMENT, 1e-4), steps=(0, 1),
+                       flags=S.SMAT_FLAG_CHUNK_LOG2(12))
 
 
 # ------------------------------------------------------------------ edges ---
@@ -241,11 +254,45 @@ def test_inplace_gradient_map():
     sess, th, t0, sim, _ = _one(n, keep=0.7)
     g = torch.randn(n, device=dev).to(torch.bfloat16)
     g0 = to_host(g)
+    sess.simulate_multi(4)
     sess.grad_map_multi(4, [g], [g])
     torch.cuda.synchronize()
     cfg = O.config(seed=9, step=4, alpha_mode=O.ALPHA_PER_TENSOR, noise=O.NOISE_UNIFORM, alpha_min=0.2)
     ref = O.gradmap(cfg, O.tensor(0, n, O.BF16, keep_prob=0.7, sigma=1e-3), g0, gdtype=O.BF16)
     assert np.array_equal(to_host(g), ref)
+
+
+def test_gradient_map_needs_the_forward_of_its_step():
+    """The gradient map regenerates the mask of the forward that produced
+    theta~ (Eq. smat-gradient; App. D): a map for a step that no forward on
+    this context ran, or for an earlier forward's step, is refused with
+    SMAT_ERR_STATE before any device work, and g_out stays untouched."""
+    n = 5000
+    sess, th, t0, sim, _ = _one(n, keep=0.7)
+    dev = torch.device("cuda")
+    g = torch.randn(n, device=dev).to(torch.bfloat16)
+    go = torch.full((n,), 7.0, dtype=torch.bfloat16, device=dev)
+    for bad in (0, 3):
+        with pytest.raises(S.SmatError) as e:
+            sess.grad_map_multi(bad, [g], [go])  # no forward yet
+        assert e.value.status == "SMAT_ERR_STATE"
+    sess.simulate_multi(3)
+    with pytest.raises(S.SmatError) as e:
+        sess.grad_map_multi(2, [g], [go])
+    assert e.value.status == "SMAT_ERR_STATE" and "step 3" in e.value.detail
+    torch.cuda.synchronize()
+    assert torch.all(go == 7.0)
+    sess.grad_map_multi(3, [g], [go])
+    sess.grad_map_multi(3, [g], [go], accumulate=True)  # accumulation over one forward
+    sess.simulate_multi(4)
+    with pytest.raises(S.SmatError):
+        sess.grad_map_multi(3, [g], [go])
+    sess.grad_map_multi(4, [g], [go])
+    torch.cuda.synchronize()
+    cfg = O.config(seed=9, step=4, alpha_mode=O.ALPHA_PER_TENSOR, noise=O.NOISE_UNIFORM, alpha_min=0.2)
+    ref = O.gradmap(cfg, O.tensor(0, n, O.BF16, keep_prob=0.7, sigma=1e-3), to_host(g), gdtype=O.BF16)
+    assert np.array_equal(to_host(go), ref)
+    assert sess.poll_errors() == 0
 
 
 def test_swap_state_and_errors():
