@@ -341,12 +341,19 @@ def delta_sigma_noalloc(theta: torch.Tensor, theta0: torch.Tensor, sigma_rel: fl
     L = load_library()
     if theta.dtype != theta0.dtype or theta.numel() != theta0.numel():
         raise ValueError("theta and theta0 differ in dtype or numel")
+    if not (theta.is_cuda and theta0.is_cuda and theta.device == theta0.device):
+        raise ValueError("theta and theta0 must be CUDA tensors on one device")
+    if not (theta.is_contiguous() and theta0.is_contiguous()):
+        raise ValueError("theta and theta0 must be contiguous")
     if out is None:
         out = torch.empty(1, dtype=torch.float32, device=theta.device)
-    check("smat_delta_sigma_noalloc",
-          L.smat_delta_sigma_noalloc(ctypes.c_void_p(theta.data_ptr()), ctypes.c_void_p(theta0.data_ptr()),
-                                     theta.numel(), dtype_code(theta.dtype), float(sigma_rel),
-                                     ctypes.c_void_p(out.data_ptr()), _stream_handle(stream)))
+    if not (out.is_cuda and out.device == theta.device and out.dtype == torch.float32 and out.numel() >= 1):
+        raise ValueError("out must be a float32 CUDA tensor of at least one element on theta's device")
+    with torch.cuda.device(theta.device):
+        check("smat_delta_sigma_noalloc",
+              L.smat_delta_sigma_noalloc(ctypes.c_void_p(theta.data_ptr()), ctypes.c_void_p(theta0.data_ptr()),
+                                         theta.numel(), dtype_code(theta.dtype), float(sigma_rel),
+                                         ctypes.c_void_p(out.data_ptr()), _stream_handle(stream)))
     return out
 
 

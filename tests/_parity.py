@@ -5,8 +5,11 @@ sampled elements (full-size lists).
 Tolerances (written out in compare()):
   masks, gradient map, uniform-noise forward: bit-exact;
   Gaussian-noise forward, fp32: |gpu - cpu| <= 1e-6 max(|cpu|, |theta|, |theta0|, 2^-126);
-  Gaussian-noise forward, bf16: at most 1 bf16 ulp apart, or, where the sum
-    cancels, |gpu - cpu| <= 1e-6 max(|theta|, |theta0|) (the fp32 bound).
+  Gaussian-noise forward, bf16: at most 1 bf16 ulp apart, or, only where the
+    sum cancels (|cpu| <= 2^-8 max(|theta|, |theta0|): the result is at least
+    256 times smaller than its inputs), |gpu - cpu| <= 1e-6 max(|theta|,
+    |theta0|) (the fp32 bound on the input scale); at most CANCEL_MAX elements
+    per comparison may use that escape, and the count is printed.
 """
 
 import numpy as np
@@ -18,6 +21,8 @@ from paper_2609_33437_gb300 import workloads as W
 
 FP32_RTOL = 1e-6
 BF16_ULPS = 1
+CANCEL_RATIO = 2.0**-8
+CANCEL_MAX = 8
 
 
 def to_host(x: torch.Tensor) -> np.ndarray:
@@ -92,12 +97,19 @@ def compare(got_bits, ref_bits, dtype, noise, th=None, t0=None, what=""):
         far = d > BF16_ULPS
         if far.any() and th is not None:
             # Where theta0 + ... + eps cancels, a bf16 ulp of the result is far
-            # below the fp32 rounding of the inputs: such elements take the
-            # fp32 bound on the input scale instead.
+            # below the fp32 rounding of the inputs: such elements (and only
+            # those) take the fp32 bound on the input scale instead.
             scale = np.maximum(np.abs(np.asarray(th, np.float64)[ok]), np.abs(np.asarray(t0, np.float64)[ok]))
+            rr = np.abs(r[ok].astype(np.float64))
             err = np.abs(g[ok].astype(np.float64) - r[ok].astype(np.float64))
-            far &= err > FP32_RTOL * np.maximum(scale, 2.0**-126)
-        assert not far.any(), f"{what}: {int(far.sum())} elements beyond {BF16_ULPS} ulp and the fp32 input-scale bound"
+            cancels = rr <= CANCEL_RATIO * scale
+            escaped = far & cancels & (err <= FP32_RTOL * np.maximum(scale, 2.0**-126))
+            n_esc = int(escaped.sum())
+            if n_esc:
+                print(f"{what}: {n_esc} cancelling element(s) compared on the fp32 input-scale bound")
+            assert n_esc <= CANCEL_MAX, f"{what}: {n_esc} elements needed the cancellation escape (at most {CANCEL_MAX})"
+            far &= ~escaped
+        assert not far.any(), f"{what}: {int(far.sum())} elements beyond {BF16_ULPS} ulp and the cancellation bound"
         return
     scale = np.abs(r[ok]).astype(np.float64)
     if th is not None:
