@@ -335,6 +335,46 @@ def gpu_local_cpus(device_index: int):
         return None
 
 
+def link_roof(h_in, h_out, nbytes=4 << 30, reps=3):
+    """Host-link copy roof on this machine: one pinned-host-to-device and one
+    device-to-pinned-host cudaMemcpyAsync of `nbytes` each (torch copy_,
+    non_blocking), alone and both at once on two streams; best of `reps`,
+    timed with CUDA events. h_in / h_out: pinned host tensors of at least
+    nbytes."""
+    hi = h_in.view(-1).view(torch.uint8)[:nbytes]
+    ho = h_out.view(-1).view(torch.uint8)[:nbytes]
+    nbytes = min(hi.numel(), ho.numel())
+    hi, ho = hi[:nbytes], ho[:nbytes]
+    d1 = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    d2 = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
+
+    def timed(which):
+        best = float("inf")
+        for _ in range(reps):
+            torch.cuda.synchronize()
+            e0, ea, eb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True), \
+                torch.cuda.Event(enable_timing=True)
+            e0.record(sa)
+            sb.wait_event(e0)
+            if which in ("h2d", "both"):
+                with torch.cuda.stream(sa):
+                    d1.copy_(hi, non_blocking=True)
+            if which in ("d2h", "both"):
+                with torch.cuda.stream(sb):
+                    ho.copy_(d2, non_blocking=True)
+            ea.record(sa)
+            eb.record(sb)
+            torch.cuda.synchronize()
+            best = min(best, max(e0.elapsed_time(ea), e0.elapsed_time(eb)) / 1e3)
+        return best
+
+    out = {"h2d": nbytes / timed("h2d") / 1e9, "d2h": nbytes / timed("d2h") / 1e9,
+           "bidirectional": 2 * nbytes / timed("both") / 1e9, "bytes_per_copy": nbytes}
+    del d1, d2
+    return out
+
+
 def e2e_run(w, sess_factory, steps, warmup, world, groups=8, keep_outputs=False):
     """The same step through the public API with host inputs: pinned host
     theta, theta0 and g~ are copied in and theta~ and g copied out every
@@ -428,14 +468,20 @@ def e2e_run(w, sess_factory, steps, warmup, world, groups=8, keep_outputs=False)
     d2h = h_sim.element_size() * n + h_go.element_size() * n
     for sess in sessions:
         sess.close()
+    if keep_outputs:  # the last step's theta~ and g on the host (tests)
+        if saved:
+            os.sched_setaffinity(0, saved)
+        return hsim, hgo
+    roof = link_roof(h_th, h_sim)
     if saved:
         os.sched_setaffinity(0, saved)
-    if keep_outputs:  # the last step's theta~ and g on the host (tests)
-        return hsim, hgo
+    host_gbs = (h2d + d2h) * steps / el / 1e9
     return {"value": world * bytes_step * steps / el / 1e9, "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": 1e3 * el / steps, "workload": w.name,
             "pipeline": f"{len(cuts)} tensor groups over copy-in / compute / copy-out streams",
-            "host_numa_node": local[0] if local else None}
+            "host_numa_node": local[0] if local else None,
+            "host_link_gbs": host_gbs, "link_roof_gbs": roof,
+            "frac_of_link_roof": host_gbs / roof["bidirectional"] if roof["bidirectional"] > 0 else None}
 
 
 def run_smat(args):

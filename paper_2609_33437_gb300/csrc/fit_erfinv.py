@@ -1,5 +1,5 @@
 """Fit the polynomial coefficients of the device erfinv used by the Gaussian
-Perturb transform (smat_kernels.cu, erfinv_poly).
+Perturb transform (smat_device.cuh: erfinv_poly, erfinv_poly2, erfinv_central2).
 
 Method (structure of M. Giles, "Approximating the erfinv function", GPU
 Computing Gems Jade Edition, 2011; coefficients fitted here): for

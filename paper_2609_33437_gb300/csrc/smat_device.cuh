@@ -10,12 +10,16 @@
 //   a5 gradmap_kernel      g = alpha m (.) g~ (Eq. smat-gradient), mask regenerated
 //   a6 mask_bits_kernel    packed keep bits (test hook)
 //
-// All of them are multi-tensor launches over a chunk table: each CTA walks
-// chunks of 2^16 elements of one tensor in grid-stride order; each thread
-// owns 16 consecutive elements at a time (one 256-bit load per bf16 input,
-// two per fp32 input), which is exactly one Philox block of the mask stream
-// (16 high bytes) and four blocks of the noise stream. The random words stay
-// in registers; masks and noise are never written to memory.
+// All of them are multi-tensor launches over a chunk table (chunks of one
+// tensor, 2^12 to 2^18 elements, the size chosen per list). The forward, with
+// the statistics fused for sigma_rel tensors, is a persistent launch whose
+// CTAs take whole chunks from an ordered work list; the unfused statistics,
+// the grid-stride forward and the gradient map walk the table in grid-stride
+// order. Each thread owns 16 consecutive elements at a time (one 256-bit load
+// per bf16 input, two per fp32 input), which is exactly one Philox block of
+// the mask stream (16 high bytes) and three blocks of the noise stream (24
+// bits per element). The random words stay in registers; masks and noise are
+// never written to memory.
 //
 // The path is elementwise and bound by HBM bandwidth or by the integer
 // pipeline (Philox): there is no contraction, so no tensor-core work.
