@@ -30,11 +30,14 @@
 //     hi = byte (gidx & 3) of W(MASK, tid, gidx >> 4)[(gidx >> 2) & 3]
 //     lo = W(MASK_LO, tid, gidx >> 2)[gidx & 3] >> 8
 //     U  = hi * 2^24 + lo ;  kept  <=>  U < T,  T = floor(p_keep * 2^32)
-//   Noise field u (24 bits) of element gidx, k = gidx & 15, q = k >> 2, r = k & 3:
-//     S[0..11] = the 12 words of W(NOISE, tid, 3 (gidx >> 4) + b), b = 0, 1, 2
+//   Packed 24-bit field F(stream, tid, gidx) of element gidx, k = gidx & 15,
+//   q = k >> 2, r = k & 3:
+//     S[0..11] = the 12 words of W(stream, tid, 3 (gidx >> 4) + b), b = 0, 1, 2
 //     (S[4b + w] = word w of block b); the quad q uses A = S[3q], B = S[3q+1],
-//     C = S[3q+2]: u = A >> 8, B >> 8, C >> 8 for r = 0, 1, 2, and for r = 3
-//     u = (A & 255) | (B & 255) << 8 | (C & 255) << 16.
+//     C = S[3q+2]: F = A >> 8, B >> 8, C >> 8 for r = 0, 1, 2, and for r = 3
+//     F = (A & 255) | (B & 255) << 8 | (C & 255) << 16 (three words serve four
+//     elements).
+//   Noise field u = F(NOISE, tid, gidx);
 //     sym24(u) = (2u + 1 - 2^24) 2^-24
 //     uniform   eps = fl(sqrt3 sigma) * sym24(u)
 //     Gaussian  eps = fl(sqrt2 sigma) * fl(erfinv(sym24(u)))  (inverse-CDF transform:
@@ -45,7 +48,7 @@
 //               RMS sigma, the matched-RMS comparison of Sec. 4.1 "Perturb")
 //   Alpha:  per tensor  alpha = fma(amax - amin, u01(W(ALPHA_T, t_a, 0)[0]), amin)
 //           t_a = 0x0FFFFFFF (one alpha for all tensors) or the tensor id;
-//           per element alpha = fma(amax - amin, u01(W(ALPHA_E, tid, gidx >> 2)[gidx & 3]), amin)
+//           per element alpha = fma(amax - amin, F(ALPHA_E, tid, gidx) 2^-24, amin)
 //
 // Merging (the evaluation side, Eq. merged-state): theta_merge = theta0 +
 // sum_j alpha_j (.) m_j (.) Delta_j over K experts, Delta_j = theta_j - theta0
@@ -263,11 +266,28 @@ bool is_kept(const OrcConfig& cfg, const OrcTensor& t, const Scalars& s, uint64_
   return U < s.T;
 }
 
+// 24-bit field of element gidx in a packed stream: the 12 words of blocks
+// 3 (gidx >> 4) .. 3 (gidx >> 4) + 2 serve the group's 16 elements, three words
+// per quad of four elements (the top 24 bits of each word for the quad's first
+// three elements, the three low bytes for the fourth).
+uint32_t field24(const OrcConfig& cfg, uint32_t stream, uint32_t tid, uint64_t gidx) {
+  const unsigned k = (unsigned)(gidx & 15), q = k >> 2, r = k & 3;
+  uint32_t quad[3];
+  for (unsigned m = 0; m < 3; ++m) {
+    const unsigned s_idx = 3 * q + m;  // index into the 12 words of the 3 blocks
+    quad[m] = stream_word(cfg, stream, tid, 3 * (gidx >> 4) + s_idx / 4, s_idx % 4);
+  }
+  if (r < 3) return quad[r] >> 8;
+  return (quad[0] & 0xFFu) | ((quad[1] & 0xFFu) << 8) | ((quad[2] & 0xFFu) << 16);
+}
+
+// Scale per coordinate: alpha ~ U[alpha_min, alpha_max) from the element's
+// 24-bit ALPHA_E field, then c = alpha / p_keep (Eq. smat-mask rescale).
 float element_c(const OrcConfig& cfg, const OrcTensor& t, const Scalars& s, uint64_t gidx) {
   if (cfg.alpha_mode != ALPHA_PER_ELEMENT) return s.c;
   const float width = cfg.alpha_max - cfg.alpha_min;
-  const uint32_t u = stream_word(cfg, S_ALPHA_E, t.tensor_id, gidx >> 2, (unsigned)(gidx & 3));
-  const float alpha = std::fma(width, u01(u), cfg.alpha_min);
+  const uint32_t u = field24(cfg, S_ALPHA_E, t.tensor_id, gidx);
+  const float alpha = std::fma(width, (float)u * kTwoPow24Inv, cfg.alpha_min);
   return alpha * s.inv_keep;
 }
 
@@ -298,14 +318,7 @@ double erfinv_d(double v) {
 
 // 24-bit noise field of element gidx (three noise words serve four elements).
 uint32_t noise_field(const OrcConfig& cfg, const OrcTensor& t, uint64_t gidx) {
-  const unsigned k = (unsigned)(gidx & 15), q = k >> 2, r = k & 3;
-  uint32_t quad[3];
-  for (unsigned m = 0; m < 3; ++m) {
-    const unsigned s_idx = 3 * q + m;  // index into the 12 words of the 3 blocks
-    quad[m] = stream_word(cfg, S_NOISE, t.tensor_id, 3 * (gidx >> 4) + s_idx / 4, s_idx % 4);
-  }
-  if (r < 3) return quad[r] >> 8;
-  return (quad[0] & 0xFFu) | ((quad[1] & 0xFFu) << 8) | ((quad[2] & 0xFFu) << 16);
+  return field24(cfg, S_NOISE, t.tensor_id, gidx);
 }
 
 float sym24(uint32_t u24) { return (float)(2 * (int32_t)u24 + 1 - (1 << 24)) * kTwoPow24Inv; }

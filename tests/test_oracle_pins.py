@@ -330,30 +330,50 @@ def test_alpha_per_element_law(amin, amax):
     assert np.all(g[~on] == 0.0)
 
 
+def _packed_field24(words12, k):
+    """The 24-bit field of element k (0..15) of a 16-element group from the
+    group's twelve words: quad q = k // 4 reads words 3q, 3q + 1, 3q + 2; its
+    first three elements take their top 24 bits, the fourth their low bytes."""
+    q, r = k >> 2, k & 3
+    A, B, C = (int(words12[3 * q + m]) for m in range(3))
+    if r < 3:
+        return (A, B, C)[r] >> 8
+    return (A & 255) | ((B & 255) << 8) | ((C & 255) << 16)
+
+
 def test_alpha_per_element_stream_layout_matches_triton_library():
-    """Coordinate gidx's alpha comes from word gidx mod 4 of the ALPHA_E
-    (stream 2) block gidx div 4: (alpha_i - alpha_min) / (alpha_max - alpha_min)
-    equals the top 24 bits of that word of Triton's Philox block, scaled by
-    2^-24, to within the fp32 rounding of the affine map. Covers element
-    offsets and draw-block indices at and above 2^32 (counter word 1)."""
+    """Coordinate gidx's alpha comes from the 24-bit field of gidx in the
+    ALPHA_E stream (stream 2): the twelve words of blocks 3 (gidx div 16) + b,
+    b = 0, 1, 2, of Triton's Philox serve the group's sixteen coordinates,
+    three words per quad of four (reading R22). (alpha_i - alpha_min) /
+    (alpha_max - alpha_min) equals that field times 2^-24 to within the fp32
+    rounding of the affine map. Covers element offsets and draw-block indices
+    at and above 2^32 (counter word 1); the noise field has the same packing
+    (R18) and shares the oracle's routine."""
     seed, step, tid, amin, amax = 0x0DDB1A5E5BADDEC0, 6, 0x0ABCDEF, 0.25, 0.875
     cfg = O.config(seed=seed, step=step, alpha_mode=O.ALPHA_PER_ELEMENT, alpha_min=amin, alpha_max=amax)
-    cases = [(0, 40), (13, 19), ((1 << 34) - 6, 12), (5 << 34, 8)]
-    ctrs, gidx, alphas = [], [], []
+    cases = [(0, 40), (13, 19), ((1 << 36) - 6, 12), (3 << 36, 8)]
+    groups = sorted({(off + i) >> 4 for off, n in cases for i in range(n)})
+    ctrs = []
+    for g in groups:
+        for b in range(3):
+            j = 3 * g + b
+            ctrs.append([j & 0xFFFFFFFF, j >> 32, (2 << 28) | tid, step])
+    assert any((3 * g) >> 32 for g in groups)
+    words = _triton_philox(ctrs, [seed] * len(ctrs), 10)
+    w12 = {g: np.concatenate([words[3 * n + b] for b in range(3)]) for n, g in enumerate(groups)}
+    back, exp, wrong = [], [], []
     for off, n in cases:
         a = _alpha_per_element(cfg, tid, n, elem_offset=off)
         for i in range(n):
-            g = off + i
-            gidx.append(g)
-            alphas.append(a[i])
-            j = g >> 2
-            ctrs.append([j & 0xFFFFFFFF, j >> 32, (2 << 28) | tid, step])
-    words = _triton_philox(ctrs, [seed] * len(ctrs), 10)
-    u = np.array([(int(words[k][g & 3]) >> 8) * 2.0**-24 for k, g in enumerate(gidx)])
-    back = (np.array(alphas) - amin) / (amax - amin)
-    assert np.all(np.abs(back - u) <= 2.0**-22), np.max(np.abs(back - u))
-    # a neighbouring word would be another, unrelated uniform
-    wrong = np.array([(int(words[k][(g + 1) & 3]) >> 8) * 2.0**-24 for k, g in enumerate(gidx)])
+            gidx = off + i
+            k = gidx & 15
+            back.append((a[i] - amin) / (amax - amin))
+            exp.append(_packed_field24(w12[gidx >> 4], k) * 2.0**-24)
+            wrong.append(_packed_field24(w12[gidx >> 4], (k & 12) | ((k + 1) & 3)) * 2.0**-24)
+    back, exp, wrong = np.array(back), np.array(exp), np.array(wrong)
+    assert np.all(np.abs(back - exp) <= 2.0**-22), np.max(np.abs(back - exp))
+    # another coordinate's field is an unrelated uniform
     assert np.mean(np.abs(back - wrong) <= 2.0**-22) < 0.1
 
 
