@@ -77,6 +77,7 @@ def parse():
     ap.add_argument("--sweep", metavar="PATH", default=None,
                     help="run the flat-tensor sweep, one JSON line per point to PATH")
     ap.add_argument("--sweep-max-log2n", type=int, default=32)
+    ap.add_argument("--sweep-min-log2n", type=int, default=16)
     ap.add_argument("--merge", choices=["wa", "ta", "dare", "ties"], default=None,
                     help="time merging K experts of the chosen list (Eq. merged-state) instead of the SMAT step")
     ap.add_argument("--experts", type=int, default=8)
@@ -655,7 +656,7 @@ def run_sweep(args):
         clocks.mark()
     n_points, fracs = 0, []
     with open(args.sweep, "w") as out:
-        for log2n in [x for x in SWEEP_LOG2N if x <= args.sweep_max_log2n]:
+        for log2n in [x for x in SWEEP_LOG2N if args.sweep_min_log2n <= x <= args.sweep_max_log2n]:
             for dt in (W.F32, W.BF16):
                 w0 = W.flat_sweep(log2n, dt, 0.5, 1, 0.0)
                 th, t0, sim, gs, go = W.generate(w0, device=dev)

@@ -295,15 +295,16 @@ __device__ __forceinline__ float noise_of(uint32_t u24, float scale) {
   return 0.0f;
 }
 
-// The 24-bit noise field of one element (any alignment): its quad's three
-// words come from one or two of the group's three noise blocks.
+// The packed 24-bit field of one element (any alignment) in the NOISE or
+// ALPHA_E stream: its quad's three words come from one or two of the group's
+// three blocks.
 template <int R>
-__device__ __forceinline__ uint32_t noise_field1(const KArgs& a, uint32_t tid, uint64_t gidx) {
+__device__ __forceinline__ uint32_t field1(const KArgs& a, uint32_t stream, uint32_t tid, uint64_t gidx) {
   const unsigned k = (unsigned)(gidx & 15), q = k >> 2, r = k & 3;
   const uint64_t j0 = 3 * (gidx >> 4);
   const unsigned s0 = 3 * q;  // first of the quad's words among the group's 12
-  const uint4 lo = stream_block<R>(a, S_NOISE, tid, j0 + s0 / 4);
-  const uint4 hi = (s0 / 4 == (s0 + 2) / 4) ? lo : stream_block<R>(a, S_NOISE, tid, j0 + (s0 + 2) / 4);
+  const uint4 lo = stream_block<R>(a, stream, tid, j0 + s0 / 4);
+  const uint4 hi = (s0 / 4 == (s0 + 2) / 4) ? lo : stream_block<R>(a, stream, tid, j0 + (s0 + 2) / 4);
   const uint32_t w8[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
   // words s0, s0 + 1, s0 + 2 relative to block s0 / 4
   const unsigned b = s0 % 4;
@@ -526,8 +527,14 @@ __device__ __forceinline__ void store1(void* base, int64_t i, float v) {
   }
 }
 
+// Scale from a raw 32-bit word (per tensor, global): its top 24 bits.
 __device__ __forceinline__ float alpha_elem(const KArgs& a, uint32_t u) {
   return __fmaf_rn(a.alpha_width, u01(u), a.alpha_min);
+}
+
+// Scale per element from its packed 24-bit ALPHA_E field: u 2^-24 is exact.
+__device__ __forceinline__ float alpha_of24(const KArgs& a, uint32_t u24) {
+  return __fmaf_rn(a.alpha_width, __fmul_rn(__uint2float_rn(u24), 5.9604644775390625e-08f), a.alpha_min);
 }
 
 // Per-chunk view of one tensor's constants.

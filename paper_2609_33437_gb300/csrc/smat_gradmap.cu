@@ -18,14 +18,27 @@ __device__ __forceinline__ void grad_compute16(const KArgs& a, const TView& v, u
     if (v.t_lo != 0u && tie && (ACC || !defer || !tl.push(off >> 4)))
       resolve_group_ties<R, J0>(a, v.tid, v.t_hi, v.t_lo, g0, kw);
   }
+  // per-element alpha: three ALPHA_E blocks per group, three words per quad
+  uint4 ab0 = make_uint4(0u, 0u, 0u, 0u), ab1 = ab0, ab2 = ab0;
+  if (PE) {
+    const uint64_t jn = 3 * (g0 >> 4);
+    ab0 = stream_block<R, J0>(a, S_ALPHA_E, v.tid, jn);
+    ab1 = stream_block<R, J0>(a, S_ALPHA_E, v.tid, jn + 1);
+    ab2 = stream_block<R, J0>(a, S_ALPHA_E, v.tid, jn + 2);
+  }
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
-    uint4 aw = make_uint4(0u, 0u, 0u, 0u);
-    if (PE) aw = stream_block<R, J0>(a, S_ALPHA_E, v.tid, (g0 >> 2) + q);
+    uint32_t ua[4] = {0u, 0u, 0u, 0u};
+    if (PE) {
+      if (q == 0) quad_fields(ab0.x, ab0.y, ab0.z, ua);
+      if (q == 1) quad_fields(ab0.w, ab1.x, ab1.y, ua);
+      if (q == 2) quad_fields(ab1.z, ab1.w, ab2.x, ua);
+      if (q == 3) quad_fields(ab2.y, ab2.z, ab2.w, ua);
+    }
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
       const int e = 4 * q + k;
-      const float c = PE ? __fmul_rn(alpha_elem(a, pick(aw, k)), v.inv_keep) : v.c;
+      const float c = PE ? __fmul_rn(alpha_of24(a, ua[k]), v.inv_keep) : v.c;
       float g = kept_of(kw, e) ? __fmul_rn(c, gs.at(e)) : 0.0f;
       if (ACC) g = __fadd_rn(go.at(e), g);
       out[e] = g;
@@ -38,10 +51,7 @@ __device__ __forceinline__ void grad_elem_as(const KArgs& a, const TView& v, con
                                              bool kept) {
   const uint64_t g = (uint64_t)(v.off + e);
   float c = v.c;
-  if (PE) {
-    const uint4 w = stream_block<R>(a, S_ALPHA_E, v.tid, g >> 2);
-    c = __fmul_rn(alpha_elem(a, pick(w, (unsigned)(g & 3))), v.inv_keep);
-  }
+  if (PE) c = __fmul_rn(alpha_of24(a, field1<R>(a, S_ALPHA_E, v.tid, g)), v.inv_keep);
   float r = kept ? __fmul_rn(c, load1<GDT>(G.g_sim, e)) : 0.0f;
   if (ACC) r = __fadd_rn(load1<GDT>(G.g_out, e), r);
   store1<GDT>(G.g_out, e, r);

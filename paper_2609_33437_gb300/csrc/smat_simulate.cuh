@@ -36,13 +36,20 @@ __device__ __forceinline__ uint32_t sim_group16(const KArgs& a, const TView& v, 
   float minL = 0.0f;
   const float2 c2 = splat(v.c);
   const float2 scale2 = splat(v.noise_scale);
-  // noise: three blocks per group, three words per quad (see quad_fields)
+  // noise and per-element alpha: three blocks per group each, three words per
+  // quad (see quad_fields)
   uint4 nb0 = make_uint4(0u, 0u, 0u, 0u), nb1 = nb0, nb2 = nb0;
+  uint4 ab0 = nb0, ab1 = nb0, ab2 = nb0;
   const uint64_t jn = 3 * (g0 >> 4);
   if (NOISE != NOISE_NONE) {
     nb0 = stream_block<R, J0>(a, S_NOISE, v.tid, jn);
     nb1 = stream_block<R, J0>(a, S_NOISE, v.tid, jn + 1);
     nb2 = stream_block<R, J0>(a, S_NOISE, v.tid, jn + 2);
+  }
+  if (PE) {
+    ab0 = stream_block<R, J0>(a, S_ALPHA_E, v.tid, jn);
+    ab1 = stream_block<R, J0>(a, S_ALPHA_E, v.tid, jn + 1);
+    ab2 = stream_block<R, J0>(a, S_ALPHA_E, v.tid, jn + 2);
   }
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
@@ -53,16 +60,21 @@ __device__ __forceinline__ uint32_t sim_group16(const KArgs& a, const TView& v, 
       if (q == 2) quad_fields(nb1.z, nb1.w, nb2.x, u);
       if (q == 3) quad_fields(nb2.y, nb2.z, nb2.w, u);
     }
-    uint4 aw = make_uint4(0u, 0u, 0u, 0u);
-    if (PE) aw = stream_block<R, J0>(a, S_ALPHA_E, v.tid, (g0 >> 2) + q);
+    uint32_t ua[4] = {0u, 0u, 0u, 0u};
+    if (PE) {
+      if (q == 0) quad_fields(ab0.x, ab0.y, ab0.z, ua);
+      if (q == 1) quad_fields(ab0.w, ab1.x, ab1.y, ua);
+      if (q == 2) quad_fields(ab1.z, ab1.w, ab2.x, ua);
+      if (q == 3) quad_fields(ab2.y, ab2.z, ab2.w, ua);
+    }
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       const int e0 = 4 * q + 2 * h;  // elements e0, e0 + 1
       const float2 th2 = th.pair(e0 >> 1), t02 = t0.pair(e0 >> 1);
       float2 kv;
       if (PE) {
-        const float2 cc = make_float2(__fmul_rn(alpha_elem(a, pick(aw, 2 * h)), v.inv_keep),
-                                      __fmul_rn(alpha_elem(a, pick(aw, 2 * h + 1)), v.inv_keep));
+        const float2 cc = make_float2(__fmul_rn(alpha_of24(a, ua[2 * h]), v.inv_keep),
+                                      __fmul_rn(alpha_of24(a, ua[2 * h + 1]), v.inv_keep));
         const float2 f = fma2_rn(cc, add2_rn(th2, make_float2(-t02.x, -t02.y)), t02);
         kv = make_float2(cc.x == 1.0f ? th2.x : f.x, cc.y == 1.0f ? th2.y : f.y);
       } else if (IDENT) {
@@ -118,14 +130,11 @@ __device__ __forceinline__ void sim_elem_as(const KArgs& a, const TView& v, cons
                                             const void* t0_p, void* sim_p, int64_t e, bool kept) {
   const uint64_t g = (uint64_t)(v.off + e);
   float c = v.c;
-  if (PE) {
-    const uint4 w = stream_block<R>(a, S_ALPHA_E, v.tid, g >> 2);
-    c = __fmul_rn(alpha_elem(a, pick(w, (unsigned)(g & 3))), v.inv_keep);
-  }
+  if (PE) c = __fmul_rn(alpha_of24(a, field1<R>(a, S_ALPHA_E, v.tid, g)), v.inv_keep);
   const float x_th = load1<DT>(th_p, e), x_t0 = load1<DT>(t0_p, e);
   float x = x_t0;
   if (kept) x = (c == 1.0f) ? x_th : __fmaf_rn(c, __fsub_rn(x_th, x_t0), x_t0);
-  if (NOISE != NOISE_NONE) x = __fadd_rn(x, noise_of<NOISE>(noise_field1<R>(a, v.tid, g), v.noise_scale));
+  if (NOISE != NOISE_NONE) x = __fadd_rn(x, noise_of<NOISE>(field1<R>(a, S_NOISE, v.tid, g), v.noise_scale));
   store1<DT>(sim_p, e, x);
 }
 
