@@ -336,57 +336,73 @@ def gpu_local_cpus(device_index: int):
         return None
 
 
-def link_roof(h_in, h_out, nbytes=4 << 30, reps=3):
-    """Host-link copy roof on this machine: one pinned-host-to-device and one
-    device-to-pinned-host cudaMemcpyAsync of `nbytes` each (torch copy_,
-    non_blocking), alone and both at once on two streams; best of `reps`,
+def link_roof(h_in, h_out, nbytes=4 << 30, reps=3, max_streams=4):
+    """Host-link copy roof on this machine: pinned-host-to-device and
+    device-to-pinned-host cudaMemcpyAsync (torch copy_, non_blocking) of
+    `nbytes` in each direction, split over 1, 2 or 4 streams at once (several
+    copy engines), alone and both directions together; best of `reps` for each,
     timed with CUDA events. h_in / h_out: pinned host tensors of at least
-    nbytes."""
-    hi = h_in.view(-1).view(torch.uint8)[:nbytes]
-    ho = h_out.view(-1).view(torch.uint8)[:nbytes]
-    nbytes = min(hi.numel(), ho.numel())
+    nbytes. Returns the best rate of each kind and the rates per stream count."""
+    hi = h_in.view(-1).view(torch.uint8)
+    ho = h_out.view(-1).view(torch.uint8)
+    nbytes = min(nbytes, hi.numel(), ho.numel())
     hi, ho = hi[:nbytes], ho[:nbytes]
     d1 = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
     d2 = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
-    sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
+    streams = [torch.cuda.Stream() for _ in range(2 * max_streams)]
 
-    def timed(which):
+    def timed(which, k):
         best = float("inf")
+        parts = [(p * nbytes // k, (p + 1) * nbytes // k) for p in range(k)]
         for _ in range(reps):
             torch.cuda.synchronize()
-            e0, ea, eb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True), \
-                torch.cuda.Event(enable_timing=True)
-            e0.record(sa)
-            sb.wait_event(e0)
-            if which in ("h2d", "both"):
-                with torch.cuda.stream(sa):
-                    d1.copy_(hi, non_blocking=True)
-            if which in ("d2h", "both"):
-                with torch.cuda.stream(sb):
-                    ho.copy_(d2, non_blocking=True)
-            ea.record(sa)
-            eb.record(sb)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e0.record(streams[0])
+            ends = []
+            for p, (a, b) in enumerate(parts):
+                for d, (src, dst) in enumerate(((hi, d1), (d2, ho))):
+                    if (which == "h2d" and d == 1) or (which == "d2h" and d == 0):
+                        continue
+                    st = streams[2 * p + d]
+                    st.wait_event(e0)
+                    with torch.cuda.stream(st):
+                        dst[a:b].copy_(src[a:b], non_blocking=True)
+                    e = torch.cuda.Event(enable_timing=True)
+                    e.record(st)
+                    ends.append(e)
             torch.cuda.synchronize()
-            best = min(best, max(e0.elapsed_time(ea), e0.elapsed_time(eb)) / 1e3)
+            best = min(best, max(e0.elapsed_time(e) for e in ends) / 1e3)
         return best
 
-    out = {"h2d": nbytes / timed("h2d") / 1e9, "d2h": nbytes / timed("d2h") / 1e9,
-           "bidirectional": 2 * nbytes / timed("both") / 1e9, "bytes_per_copy": nbytes}
+    out = {"bytes_per_direction": nbytes, "per_streams": {}}
+    for k in (1, 2, max_streams):
+        r = {"h2d": nbytes / timed("h2d", k) / 1e9, "d2h": nbytes / timed("d2h", k) / 1e9,
+             "bidirectional": 2 * nbytes / timed("both", k) / 1e9}
+        out["per_streams"][k] = r
+    for kind in ("h2d", "d2h", "bidirectional"):
+        out[kind] = max(r[kind] for r in out["per_streams"].values())
     del d1, d2
     return out
 
 
-def e2e_run(w, sess_factory, steps, warmup, world, groups=8, keep_outputs=False):
+def e2e_run(w, sess_factory, steps, warmup, world, groups=8, keep_outputs=False, copy_streams=2):
     """The same step through the public API with host inputs: pinned host
     theta, theta0 and g~ are copied in and theta~ and g copied out every
     step, inside the timed region. The list is cut into `groups` groups of
     consecutive tensors (one session each, same tensor ids, so the results
-    are those of one session) and pipelined over three streams: group k's
-    inputs are copied in while group k - 1 computes and group k - 2's results
-    are copied out; each step ends when all of its results are on the host."""
+    are those of one session). A group's tensors are views of one device
+    buffer per array, laid out as on the host (a tensor whose size is not a
+    multiple of 16 elements pads the next one's start to keep 32-byte
+    alignment), so a group moves with a few large copies, each split over
+    `copy_streams` streams per direction so several copy engines work at once.
+    Groups and steps are pipelined: group k's inputs of step s + 1 are copied
+    in as soon as its compute of step s has read them, its results copied out
+    while later groups compute; the timed region ends when the results of the
+    last step are on the host."""
     dev = torch.device("cuda")
     tdt, gdt = W.torch_dtype(w.dtype), W.torch_dtype(w.gdtype)
     n = w.numel
+    nt = len(w.tensors)
     # host buffers and copies on the CPUs next to the GPU (first-touch placement)
     local = gpu_local_cpus(torch.cuda.current_device())
     saved = os.sched_getaffinity(0) if local else None
@@ -398,65 +414,103 @@ def e2e_run(w, sess_factory, steps, warmup, world, groups=8, keep_outputs=False)
     h_sim = torch.empty(n, dtype=tdt, pin_memory=True)
     h_go = torch.empty(n, dtype=gdt, pin_memory=True)
     offs = np.cumsum([0] + [t.numel for t in w.tensors])
-    d_th, d_t0, d_sim, d_gs, d_go = [], [], [], [], []
-    for k in range(len(w.tensors)):
+    # groups of consecutive tensors with about n / groups elements each
+    cuts, target, acc, start = [], n / max(1, groups), 0, 0
+    for k, t in enumerate(w.tensors):
+        acc += t.numel
+        if acc >= target * (len(cuts) + 1) or k == nt - 1:
+            cuts.append(list(range(start, k + 1)))
+            start = k + 1
+    # per group: device offsets of its tensors (16-element aligned) and the
+    # runs of tensors whose device layout equals the host layout
+    bufs, views, runs = [], [None] * nt, []
+    for ks in cuts:
+        doff, d = {}, 0
+        for k in ks:
+            d = (d + 15) // 16 * 16
+            doff[k] = d
+            d += w.tensors[k].numel
+        gb = {name: torch.empty(max(d, 1), dtype=(gdt if name in ("gs", "go") else tdt), device=dev)
+              for name in ("th", "t0", "gs", "sim", "go")}
+        bufs.append(gb)
+        for k in ks:
+            a, b = doff[k], doff[k] + w.tensors[k].numel
+            views[k] = {name: buf[a:b] for name, buf in gb.items()}
+        r = []
+        for k in ks:
+            if r and doff[k] - int(offs[k]) == r[-1][2]:
+                r[-1][1] = int(offs[k + 1])
+            else:
+                r.append([int(offs[k]), int(offs[k + 1]), doff[k] - int(offs[k])])
+        runs.append(r)
+    for k in range(nt):
         th, t0, g = W.generate_tensor(w, k, dev)
         a, b = int(offs[k]), int(offs[k + 1])
         h_th[a:b].copy_(th)
         h_t0[a:b].copy_(t0)
         h_gs[a:b].copy_(g)
-        d_th.append(th)
-        d_t0.append(t0)
-        d_gs.append(g)
-        d_sim.append(torch.empty_like(th))
-        d_go.append(torch.empty_like(g))
-    hv = lambda h: [h[int(offs[k]):int(offs[k + 1])] for k in range(len(w.tensors))]  # noqa: E731
-    hth, ht0, hgs, hsim, hgo = hv(h_th), hv(h_t0), hv(h_gs), hv(h_sim), hv(h_go)
-    # groups of consecutive tensors with about n / groups elements each
-    cuts, target, acc, start = [], n / max(1, groups), 0, 0
-    for k, t in enumerate(w.tensors):
-        acc += t.numel
-        if acc >= target * (len(cuts) + 1) or k == len(w.tensors) - 1:
-            cuts.append(list(range(start, k + 1)))
-            start = k + 1
-    sessions = [sess_factory([d_th[k] for k in ks], [d_t0[k] for k in ks], [d_sim[k] for k in ks], ks)
-                for ks in cuts]
-    s_in, s_cmp, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+        views[k]["th"].copy_(th)
+        views[k]["t0"].copy_(t0)
+        views[k]["gs"].copy_(g)
+        del th, t0, g
+    sessions = [sess_factory([views[k]["th"] for k in ks], [views[k]["t0"] for k in ks],
+                             [views[k]["sim"] for k in ks], ks) for ks in cuts]
+    s_in = [torch.cuda.Stream() for _ in range(copy_streams)]
+    s_out = [torch.cuda.Stream() for _ in range(copy_streams)]
+    s_cmp = torch.cuda.Stream()
     done = [None] * len(cuts)    # compute of the group finished (its inputs are free)
     copied = [None] * len(cuts)  # results of the group copied out (its outputs are free)
 
+    def pieces(a, b):
+        # split [a, b) into copy_streams parts when it is large enough to gain from it
+        if b - a < (32 << 20):
+            return [(0, a, b)]
+        return [(p, a + p * (b - a) // copy_streams, a + (p + 1) * (b - a) // copy_streams)
+                for p in range(copy_streams)]
+
     def one(step):
         for gi, ks in enumerate(cuts):
-            ev_in = torch.cuda.Event()
-            with torch.cuda.stream(s_in):
+            gb = bufs[gi]
+            ev_in = []
+            for p, st in enumerate(s_in):
                 if done[gi] is not None:
-                    s_in.wait_event(done[gi])
-                for k in ks:
-                    d_th[k].copy_(hth[k], non_blocking=True)
-                    d_t0[k].copy_(ht0[k], non_blocking=True)
-                    d_gs[k].copy_(hgs[k], non_blocking=True)
-                ev_in.record(s_in)
-            sess = sessions[gi]
-            s_cmp.wait_event(ev_in)
+                    st.wait_event(done[gi])
+            for a0, b0, shift in runs[gi]:
+                for p, a, b in pieces(a0, b0):
+                    with torch.cuda.stream(s_in[p]):
+                        gb["th"][a + shift:b + shift].copy_(h_th[a:b], non_blocking=True)
+                        gb["t0"][a + shift:b + shift].copy_(h_t0[a:b], non_blocking=True)
+                        gb["gs"][a + shift:b + shift].copy_(h_gs[a:b], non_blocking=True)
+            for st in s_in:
+                e = torch.cuda.Event()
+                e.record(st)
+                s_cmp.wait_event(e)
             if copied[gi] is not None:
-                s_cmp.wait_event(copied[gi])
+                for e in copied[gi]:
+                    s_cmp.wait_event(e)
+            sess = sessions[gi]
             sess.simulate_multi(step, stream=s_cmp)
             sess.swap()
-            sess.grad_map_multi(step, [d_gs[k] for k in ks], [d_go[k] for k in ks], stream=s_cmp)
+            sess.grad_map_multi(step, [views[k]["gs"] for k in ks], [views[k]["go"] for k in ks], stream=s_cmp)
             sess.swap()
             done[gi] = torch.cuda.Event()
             done[gi].record(s_cmp)
-            with torch.cuda.stream(s_out):
-                s_out.wait_event(done[gi])
-                for k in ks:
-                    hsim[k].copy_(d_sim[k], non_blocking=True)
-                    hgo[k].copy_(d_go[k], non_blocking=True)
-                copied[gi] = torch.cuda.Event()
-                copied[gi].record(s_out)
-        s_out.synchronize()
+            for st in s_out:
+                st.wait_event(done[gi])
+            for a0, b0, shift in runs[gi]:
+                for p, a, b in pieces(a0, b0):
+                    with torch.cuda.stream(s_out[p]):
+                        h_sim[a:b].copy_(gb["sim"][a + shift:b + shift], non_blocking=True)
+                        h_go[a:b].copy_(gb["go"][a + shift:b + shift], non_blocking=True)
+            copied[gi] = []
+            for st in s_out:
+                e = torch.cuda.Event()
+                e.record(st)
+                copied[gi].append(e)
 
     for s in range(warmup):
         one(s)
+    torch.cuda.synchronize()
     barrier(world)
     torch.cuda.synchronize()
     a = time.perf_counter()
@@ -472,14 +526,18 @@ def e2e_run(w, sess_factory, steps, warmup, world, groups=8, keep_outputs=False)
     if keep_outputs:  # the last step's theta~ and g on the host (tests)
         if saved:
             os.sched_setaffinity(0, saved)
-        return hsim, hgo
+        hv = lambda h: [h[int(offs[k]):int(offs[k + 1])] for k in range(nt)]  # noqa: E731
+        return hv(h_sim), hv(h_go)
+    del bufs, views
+    torch.cuda.empty_cache()
     roof = link_roof(h_th, h_sim)
     if saved:
         os.sched_setaffinity(0, saved)
     host_gbs = (h2d + d2h) * steps / el / 1e9
     return {"value": world * bytes_step * steps / el / 1e9, "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": 1e3 * el / steps, "workload": w.name,
-            "pipeline": f"{len(cuts)} tensor groups over copy-in / compute / copy-out streams",
+            "pipeline": f"{len(cuts)} tensor groups, steps and groups pipelined over {copy_streams} copy-in, "
+                        f"one compute and {copy_streams} copy-out streams",
             "host_numa_node": local[0] if local else None,
             "host_link_gbs": host_gbs, "link_roof_gbs": roof,
             "frac_of_link_roof": host_gbs / roof["bidirectional"] if roof["bidirectional"] > 0 else None}
@@ -620,7 +678,7 @@ def run_smat(args):
             ew = W.scaled(w, int(0.5 * avail / 10))
         del th, t0, sim, gs, go
         torch.cuda.empty_cache()
-        e2e = e2e_run(ew, make_session, steps=max(1, min(args.steps, 3)), warmup=1, world=world)
+        e2e = e2e_run(ew, make_session, steps=max(2, min(args.steps, 5)), warmup=1, world=world)
         if out is not None:
             out["e2e"] = e2e
     if out is not None and not args.no_cpu_baseline and world == 1:
