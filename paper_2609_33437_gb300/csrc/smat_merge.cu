@@ -132,44 +132,44 @@ __device__ __forceinline__ void merge_linear16(const MArgs& m, const MTensor& T,
 
 // DARE keep masks. A warp first draws the masks of its 32 groups for all K
 // experts (expert e's mask is the Mask stream at step e) into shared memory,
-// two experts per word (bit 16 (e & 1) + k: element k of expert e). An
-// element whose mask byte equals the threshold's high byte (probability
-// 1/256 per element and expert) is decided by its low 24 bits (MASK_LO
-// stream): these ties are queued per warp across all experts and then drawn
-// by the whole warp, one MASK_LO block per lane, so a warp spends about one
-// Philox pass per group on them instead of one mostly idle pass per expert.
-// A queue that fills up (about K/16 ties per thread are expected, the
-// capacity is 4 per thread) makes the owner draw the rest itself.
+// as byte masks: byte b of word q of (expert e, thread t) is 0xFF iff element
+// 4q + b of t's group is kept. An element whose mask byte equals the
+// threshold's high byte (probability 1/256 per element and expert) is decided
+// by its low 24 bits (MASK_LO stream): these ties are queued per warp across
+// all experts and then drawn by the whole warp, one MASK_LO block per lane, so
+// a warp spends about one Philox pass per group on them instead of one mostly
+// idle pass per expert. A queue that fills up (about K/16 ties per thread are
+// expected, the capacity is 4 per thread) makes the owner draw the rest itself.
 constexpr int kDareQueue = 128;
-struct DareShared {
-  uint32_t keep[kMergeMaxExperts / 2][kBlock];
+struct DareQueue {
   uint16_t q[kBlock / 32][kDareQueue];  // (lane << 8) | (expert << 4) | element
   int n[kBlock / 32];
 };
+// Dynamic shared memory of the DARE kernel: the queue, then uint4 keep masks
+// [K][kBlock] (16 bytes per expert and thread).
+constexpr size_t kDareQueueBytes = (sizeof(DareQueue) + 15) / 16 * 16;
+size_t dare_smem_bytes(int K) { return kDareQueueBytes + (size_t)K * kBlock * sizeof(uint4); }
 
-// kw's flag bits 8b + 7 of word q -> bit 4q + b.
-__device__ __forceinline__ uint32_t compress_keep16(const uint32_t (&kw)[4]) {
-  uint32_t r = 0u;
-#pragma unroll
-  for (int q = 0; q < 4; ++q) r |= ((((kw[q] >> 7) * 0x00204081u) >> 21) & 0xFu) << (4 * q);
-  return r;
-}
+struct DareShared {
+  DareQueue* qs;
+  uint4* keep;  // keep[e * kBlock + thread]
+};
 
-// Keep bits of expert e from its Mask block w (bit k: element k); ties go to
-// the warp's queue, or are drawn here once the queue is full.
+// Byte masks of expert e from its Mask block w; ties go to the warp's queue,
+// or are drawn here once the queue is full.
 template <int R>
-__device__ __forceinline__ uint32_t dare_keep_bits(const MArgs& m, const MTensor& T, const uint4& w, int e,
-                                                   uint64_t g0, DareShared& s) {
+__device__ __forceinline__ uint4 dare_keep_masks(const MArgs& m, const MTensor& T, const uint4& w, int e,
+                                                 uint64_t g0, DareShared& s) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   uint32_t kw[4];
   if (keep_bytes16(w, T.t_hi, kw) && T.t_lo != 0u) {
     uint32_t tb = tie_bits16(w, T.t_hi);
-    int slot = atomicAdd(&s.n[warp], __popc(tb));
+    int slot = atomicAdd(&s.qs->n[warp], __popc(tb));
     while (tb) {
       const int k = __ffs(tb) - 1;
       tb &= tb - 1u;
       if (slot < kDareQueue) {
-        s.q[warp][slot] = (uint16_t)((lane << 8) | (e << 4) | k);
+        s.qs->q[warp][slot] = (uint16_t)((lane << 8) | (e << 4) | k);
       } else {
         const uint64_t g = g0 + (uint64_t)k;
         const uint4 l = stream_block_at<R>(m.key, (uint32_t)e, S_MASK_LO, T.tid, g >> 2);
@@ -178,40 +178,89 @@ __device__ __forceinline__ uint32_t dare_keep_bits(const MArgs& m, const MTensor
       ++slot;
     }
   }
-  return compress_keep16(kw);
+  // flag bit 7 of each byte -> 0x00 / 0xFF
+  return make_uint4((kw[0] >> 7) * 0xFFu, (kw[1] >> 7) * 0xFFu, (kw[2] >> 7) * 0xFFu, (kw[3] >> 7) * 0xFFu);
 }
 
 // Called by all 32 lanes of the warp (full: this lane has a vector group at
 // element index g0; gw0: lane 0's group). Two experts' Mask blocks are drawn
 // together (two independent Philox chains per thread). On return the lane's
-// keep words are complete.
+// keep masks are complete.
 template <int R>
 __device__ __forceinline__ void dare_masks(const MArgs& m, const MTensor& T, bool full, uint64_t g0, uint64_t gw0,
                                            DareShared& s) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (lane == 0) s.n[warp] = 0;
+  if (lane == 0) s.qs->n[warp] = 0;
   __syncwarp();
   if (full) {
 #pragma unroll 1
     for (int e = 0; e < m.K; e += 2) {
       const uint4 w0 = stream_block_at<R>(m.key, (uint32_t)e, S_MASK, T.tid, g0 >> 4);
       const uint4 w1 = stream_block_at<R>(m.key, (uint32_t)e + 1u, S_MASK, T.tid, g0 >> 4);
-      uint32_t pair = dare_keep_bits<R>(m, T, w0, e, g0, s);
-      if (e + 1 < m.K) pair |= dare_keep_bits<R>(m, T, w1, e + 1, g0, s) << 16;
-      s.keep[e >> 1][threadIdx.x] = pair;
+      s.keep[e * kBlock + threadIdx.x] = dare_keep_masks<R>(m, T, w0, e, g0, s);
+      if (e + 1 < m.K) s.keep[(e + 1) * kBlock + threadIdx.x] = dare_keep_masks<R>(m, T, w1, e + 1, g0, s);
     }
   }
   __syncwarp();
-  const int n = min(s.n[warp], kDareQueue);
+  const int n = min(s.qs->n[warp], kDareQueue);
   for (int j = lane; j < n; j += 32) {
-    const uint32_t it = s.q[warp][j];
+    const uint32_t it = s.qs->q[warp][j];
     const int owner = (int)(it >> 8), e = (int)((it >> 4) & 15u), k = (int)(it & 15u);
     const uint64_t g = gw0 + 16 * (uint64_t)owner + (uint64_t)k;
     const uint4 l = stream_block_at<R>(m.key, (uint32_t)e, S_MASK_LO, T.tid, g >> 2);
-    if ((pick(l, (unsigned)(g & 3)) >> 8) < T.t_lo)
-      atomicOr(&s.keep[e >> 1][(warp << 5) + owner], 1u << (16 * (e & 1) + k));
+    if ((pick(l, (unsigned)(g & 3)) >> 8) < T.t_lo) {
+      uint32_t* kwp = reinterpret_cast<uint32_t*>(&s.keep[e * kBlock + (warp << 5) + owner]);
+      atomicOr(kwp + (k >> 2), 0xFFu << (8 * (k & 3)));
+    }
   }
   __syncwarp();
+}
+
+// Expert e's DARE contribution to a bf16 group: the expert's bf16 words are
+// blended with theta0's by the keep masks (a dropped element takes theta0's
+// bits), so a dropped element's Delta is fl(theta0 - theta0) = +0 and its
+// multiply-add leaves acc unchanged (acc is never -0: it starts at +0 and a
+// sum rounds to -0 only from two -0). This is exact while theta0 is finite;
+// the caller takes the select path below for a group with an infinite or NaN
+// theta0 (whose Delta would be NaN instead of unused).
+__device__ __forceinline__ void dare_acc16_blend(float c, const uint4& km, const Raw16<DT_BF16>& x,
+                                                 const Raw16<DT_BF16>& t0, float2 (&acc)[8]) {
+  const float2 c2 = splat(c);
+  const uint32_t kmw[4] = {km.x, km.y, km.z, km.w};
+#pragma unroll
+  for (int h = 0; h < 8; ++h) {
+    // 16-bit lanes of the word's two elements: bytes 0, 1 (even h) or 2, 3 (odd h) of mask word h / 2
+    const uint32_t lm = __byte_perm(kmw[h >> 1], 0u, (h & 1) ? 0x3322u : 0x1100u);
+    const uint32_t xw = (x.r[h] & lm) | (t0.r[h] & ~lm);
+    const float2 b = t0.pair(h);
+    const float2 d = add2_rn(make_float2(__uint_as_float(xw << 16), __uint_as_float(xw & 0xFFFF0000u)),
+                             make_float2(-b.x, -b.y));
+    acc[h] = fma2_rn(c2, d, acc[h]);
+  }
+}
+
+// The same with a select per element after the multiply-add (fp32 groups, and
+// bf16 groups whose theta0 is not finite).
+template <int DT>
+__device__ __forceinline__ void dare_acc16_select(float c, const uint4& km, const Raw16<DT>& x, const Raw16<DT>& t0,
+                                                  float2 (&acc)[8]) {
+  const float2 c2 = splat(c);
+  const uint32_t kw[4] = {km.x, km.y, km.z, km.w};
+#pragma unroll
+  for (int h = 0; h < 8; ++h) {
+    const float2 b = t0.pair(h);
+    const float2 d = add2_rn(x.pair(h), make_float2(-b.x, -b.y));
+    const float2 f = fma2_rn(c2, d, acc[h]);
+    acc[h] = make_float2(kept_of(kw, 2 * h) ? f.x : acc[h].x, kept_of(kw, 2 * h + 1) ? f.y : acc[h].y);
+  }
+}
+
+// Some element of a bf16 group is infinite or NaN (exponent all ones).
+__device__ __forceinline__ bool nonfinite16(const Raw16<DT_BF16>& v) {
+  uint32_t nf = 0u;
+#pragma unroll
+  for (int h = 0; h < 8; ++h) nf |= (v.r[h] & 0x7F807F80u) + 0x00800080u;  // 0x8000 in a half iff its exponent is 0xFF
+  return (nf & 0x80008000u) != 0u;
 }
 
 // Experts loaded before the keep masks are drawn (fp32 groups are twice the
@@ -229,6 +278,8 @@ __device__ __forceinline__ void dare_linear16(const MArgs& m, const MTensor& T, 
 #pragma unroll
   for (int h = 0; h < 8; ++h) acc[h] = splat(0.0f);
   const void* const* xp = m.experts + t * m.K;
+  bool blend = false;
+  if (DT == DT_BF16) blend = !nonfinite16(*reinterpret_cast<const Raw16<DT_BF16>*>(&t0));
 #pragma unroll 1
   for (int e = 0; e < m.K; e += kExpertBatch) {
 #pragma unroll
@@ -237,9 +288,13 @@ __device__ __forceinline__ void dare_linear16(const MArgs& m, const MTensor& T, 
 #pragma unroll
     for (int b = 0; b < kExpertBatch; ++b) {
       if (e + b < m.K) {
-        const int ee = e + b;
-        const uint32_t keep = masked ? (s.keep[ee >> 1][threadIdx.x] >> (16 * (ee & 1))) & 0xFFFFu : 0xFFFFu;
-        merge_acc16<DT>(m.c, keep, x[b], t0, acc);
+        const uint4 km = masked ? s.keep[(e + b) * kBlock + threadIdx.x]
+                                : make_uint4(0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu);
+        if (DT == DT_BF16 && blend)
+          dare_acc16_blend(m.c, km, *reinterpret_cast<const Raw16<DT_BF16>*>(&x[b]),
+                           *reinterpret_cast<const Raw16<DT_BF16>*>(&t0), acc);
+        else
+          dare_acc16_select<DT>(m.c, km, x[b], t0, acc);
       }
     }
   }
@@ -394,7 +449,10 @@ __global__ void __launch_bounds__(kBlock, 2) merge_kernel(const __grid_constant_
 // during the Philox work.
 template <int R, int DT>
 __global__ void __launch_bounds__(kBlock, 2) dare_kernel(const __grid_constant__ MArgs m) {
-  __shared__ DareShared s;
+  extern __shared__ __align__(16) unsigned char dare_smem[];
+  DareShared s;
+  s.qs = reinterpret_cast<DareQueue*>(dare_smem);
+  s.keep = reinterpret_cast<uint4*>(dare_smem + kDareQueueBytes);
   const int warp = threadIdx.x >> 5;
   for (int64_t ci = blockIdx.x; ci < m.n_chunks; ci += gridDim.x) {
     const Chunk ch = m.chunks[ci];
@@ -548,7 +606,16 @@ cudaError_t merge_method(const MArgs& m, int grid, cudaStream_t s) {
   switch (m.method) {
     case SMAT_MERGE_WA: merge_kernel<R, DT, SMAT_MERGE_WA><<<grid, kBlock, 0, s>>>(m); break;
     case SMAT_MERGE_TA: merge_kernel<R, DT, SMAT_MERGE_TA><<<grid, kBlock, 0, s>>>(m); break;
-    case SMAT_MERGE_DARE_TA: dare_kernel<R, DT><<<grid, kBlock, 0, s>>>(m); break;
+    case SMAT_MERGE_DARE_TA: {
+      const size_t smem = dare_smem_bytes(m.K);
+      if (smem > 48 * 1024) {
+        const cudaError_t e = cudaFuncSetAttribute(dare_kernel<R, DT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                   (int)smem);
+        if (e != cudaSuccess) return e;
+      }
+      dare_kernel<R, DT><<<grid, kBlock, smem, s>>>(m);
+      break;
+    }
     default: merge_kernel<R, DT, SMAT_MERGE_TIES><<<grid, kBlock, 0, s>>>(m); break;
   }
   return cudaGetLastError();
