@@ -545,6 +545,33 @@ struct TView {
   bool has_noise;
 };
 
+// Flags published by one CTA and waited for by another (work-list launches):
+// a release store after the data, an acquire load before reading it. Every
+// such wait gives up after kWaitLimit polls of 256 ns (about a second).
+constexpr uint32_t kWaitLimit = 1u << 22;
+
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_release(uint32_t* p, uint32_t v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Wait until *p == v; false (and bit 0 of *error set) once the limit is reached.
+__device__ __forceinline__ bool wait_value(const uint32_t* p, uint32_t v, int32_t* error) {
+  for (uint32_t n = 0;; ++n) {
+    if (ld_acquire(p) == v) return true;
+    if (n >= kWaitLimit) {
+      atomicOr(error, 1);
+      return false;
+    }
+    __nanosleep(256);
+  }
+}
+
 __device__ __forceinline__ double warp_sum(double x) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);

@@ -244,28 +244,7 @@ __device__ __forceinline__ void sim_chunk_noise(const KArgs& a, const TView& v, 
 // running CTA. The wait is bounded all the same: after kWaitLimit polls
 // (about one second) it sets bit 0 of *a.error, skips the item and returns to
 // the queue.
-constexpr uint32_t kWaitLimit = 1u << 22;
-
-__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
-  uint32_t v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-
-__device__ __forceinline__ void st_release(uint32_t* p, uint32_t v) {
-  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
-
-__device__ __forceinline__ bool wait_ready(const KArgs& a, int t) {
-  for (uint32_t n = 0;; ++n) {
-    if (ld_acquire(a.ready + t) == a.epoch) return true;
-    if (n >= kWaitLimit) {
-      atomicOr(a.error, 1);
-      return false;
-    }
-    __nanosleep(256);
-  }
-}
+__device__ __forceinline__ bool wait_ready(const KArgs& a, int t) { return wait_value(a.ready + t, a.epoch, a.error); }
 
 // All threads of the CTA call this for the same chunk (it has a barrier).
 template <int R, int DT, int NOISE, bool PE, bool IP>
