@@ -143,14 +143,14 @@ cudaError_t launch_simulate(const KArgs& a, int grid, int dtype, int noise, bool
 }
 
 cudaError_t launch_stats_simulate(const KArgs& a, int grid, int dtype, int noise, bool per_elem_alpha,
-                                  int rounds, bool inplace, cudaStream_t s) {
+                                  int rounds, bool inplace, bool wide, cudaStream_t s) {
   if (noise == NOISE_LAPLACE)
     return dtype == DT_BF16 ? launch_laplace_bf16(a, grid, true, per_elem_alpha, inplace, s)
                             : launch_laplace_f32(a, grid, true, per_elem_alpha, inplace, s);
   if (inplace)
     return dtype == DT_BF16 ? launch_stats_simulate_inplace_bf16(a, grid, noise, per_elem_alpha, rounds, s)
                             : launch_stats_simulate_inplace_f32(a, grid, noise, per_elem_alpha, rounds, s);
-  return dtype == DT_BF16 ? launch_stats_simulate_bf16(a, grid, noise, per_elem_alpha, rounds, s)
+  return dtype == DT_BF16 ? launch_stats_simulate_bf16(a, grid, noise, per_elem_alpha, rounds, wide, s)
                           : launch_stats_simulate_f32(a, grid, noise, per_elem_alpha, rounds, s);
 }
 

@@ -243,6 +243,7 @@ struct smat_ctx {
   bool grads_uploaded = false;
   // work-list forward launch (with the statistics of sigma_rel tensors)
   bool fused = false;
+  bool wide = false;  // the bf16 fused launch carries statistics items: its four-CTA build
   std::vector<int32_t> h_items;
   int32_t item_begin[kMaxRanges] = {0, 0};
   int32_t item_count[kMaxRanges] = {0, 0};
@@ -491,11 +492,13 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
     e = cudaMemcpyAsync(c->d_chunks, c->h_chunks.data(), sizeof(Chunk) * (size_t)nc,
                         cudaMemcpyHostToDevice, stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(c->d_sync, 0, sizeof(int32_t) * sync_words(n_tensors), stream);
+  c->wide = rel && cfg->alpha_mode != SMAT_ALPHA_PER_ELEMENT && cfg->noise != SMAT_NOISE_LAPLACE && !c->any_inplace;
   if (e == cudaSuccess && c->fused) {
     // lead of about two grid widths of the bf16 forward
     const int64_t lead = 2 * (int64_t)c->sm_count *
-                         streaming_ctas_per_sm(SMAT_BF16, cfg->noise, cfg->alpha_mode == SMAT_ALPHA_PER_ELEMENT,
-                                               c->rounds);
+                         (c->wide ? fused_wide_ctas_per_sm(cfg->noise, c->rounds)
+                                  : streaming_ctas_per_sm(SMAT_BF16, cfg->noise,
+                                                          cfg->alpha_mode == SMAT_ALPHA_PER_ELEMENT, c->rounds));
     for (int dt = 0; dt < 2; ++dt) build_items(c, dt, lead);
     if (!c->h_items.empty())
       e = cudaMemcpyAsync(c->d_items, c->h_items.data(), sizeof(int32_t) * c->h_items.size(),
@@ -534,10 +537,16 @@ smat_status smat_simulate_multi(smat_ctx* c, uint32_t step, smat_stream_t stream
       a.items = c->d_items + c->item_begin[dt];
       a.n_items = c->item_count[dt];
       a.work_counter = c->d_sync + dt;
-      const int grid = grid_for(c, c->range_end[dt] - c->range_begin[dt], dt);
+      const bool wide = c->wide && dt == SMAT_BF16;
+      int grid = grid_for(c, c->range_end[dt] - c->range_begin[dt], dt);
+      if (wide) {
+        const int64_t chunks = c->range_end[dt] - c->range_begin[dt];
+        const int64_t resident = (int64_t)c->sm_count * fused_wide_ctas_per_sm(c->cfg.noise, c->rounds);
+        grid = (int)(chunks < resident ? chunks : resident);
+      }
       Timed t(c, 2, stream);
       const cudaError_t e = launch_stats_simulate(a, grid, dt, c->cfg.noise, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT,
-                                                  c->rounds, c->any_inplace, stream);
+                                                  c->rounds, c->any_inplace, wide, stream);
       t.done();
       if (e != cudaSuccess) return cuda_fail(e, "fused statistics + forward launch");
     }
@@ -726,7 +735,7 @@ smat_status smat_debug_fused(smat_ctx* c, uint32_t step, const int32_t* d_items,
   a.n_items = n_items;
   a.work_counter = c->d_sync + SMAT_BF16;
   e = launch_stats_simulate_bf16(a, grid_for(c, c->range_end[SMAT_BF16] - c->range_begin[SMAT_BF16], SMAT_BF16),
-                                 c->cfg.noise, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT, c->rounds, stream);
+                                 c->cfg.noise, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT, c->rounds, false, stream);
   if (e != cudaSuccess) return cuda_fail(e, "fused launch");
   c->scalars_step = -1;  // sigma_t of this call may be incomplete
   c->sim_step = -1;      // and its forward too

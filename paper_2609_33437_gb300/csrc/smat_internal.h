@@ -123,8 +123,10 @@ cudaError_t launch_delta_stats(const KArgs& a, int grid, int dtype, cudaStream_t
 cudaError_t launch_scalars(const KArgs& a, int noise, int rounds, cudaStream_t s);
 cudaError_t launch_simulate(const KArgs& a, int grid, int dtype, int noise, bool per_elem_alpha,
                             int rounds, bool inplace, cudaStream_t s);
+// wide: the list has statistics items (bf16 without per-element alpha, not
+// in place, uniform or Gaussian noise: the four-CTA-per-SM build).
 cudaError_t launch_stats_simulate(const KArgs& a, int grid, int dtype, int noise, bool per_elem_alpha,
-                                  int rounds, bool inplace, cudaStream_t s);
+                                  int rounds, bool inplace, bool wide, cudaStream_t s);
 cudaError_t launch_gradmap(const KArgs& a, int grid, int gdtype, bool per_elem_alpha, bool accumulate,
                            int rounds, cudaStream_t s);
 cudaError_t launch_simulate_f32(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
@@ -136,7 +138,9 @@ int simulate_ctas_per_sm_bf16(int noise, bool per_elem_alpha, int rounds);
 cudaError_t launch_stats_simulate_f32(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
                                       cudaStream_t s);
 cudaError_t launch_stats_simulate_bf16(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
-                                       cudaStream_t s);
+                                       bool wide, cudaStream_t s);
+// Resident CTAs per SM of the four-CTA build (bf16, uniform or Gaussian).
+int fused_wide_ctas_per_sm(int noise, int rounds);
 // Laplace noise (10 rounds; smat_laplace_*.cu): the work-list launch when
 // `fused`, else the grid-stride one; in-place instantiations when `inplace`.
 cudaError_t launch_laplace_f32(const KArgs& a, int grid, bool fused, bool per_elem_alpha, bool inplace, cudaStream_t s);

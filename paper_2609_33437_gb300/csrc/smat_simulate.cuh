@@ -260,8 +260,12 @@ __device__ __forceinline__ void forward_chunk(const KArgs& a, const TView& v, co
   }
 }
 
-template <int R, int DT, int NOISE, bool PE, bool IP>
-__global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 3 : 2)
+// MINB: CTAs per SM the launch is built for. Lists with statistics items run
+// the bf16 launch at four CTAs per SM (64 registers): the extra warps hide
+// the statistics' memory latency (7B list: 11.98 -> 11.73 ms); forward-only
+// lists keep three (80 registers, no spills in the group path).
+template <int R, int DT, int NOISE, bool PE, bool IP, int MINB = ((DT == DT_BF16 && !PE) ? 3 : 2)>
+__global__ void __launch_bounds__(kBlock, MINB)
     stats_simulate_kernel(const __grid_constant__ KArgs a) {
   __shared__ double sh_s[kBlock / 32];
   __shared__ double sh_q[kBlock / 32];
@@ -358,26 +362,50 @@ __global__ void __launch_bounds__(kBlock, (DT == DT_BF16 && !PE) ? 3 : 2) simula
 }
 
 
-template <int R, int DT, int NOISE, bool PE, bool IP>
-struct FusedVariant {
-  static cudaError_t run(const KArgs& a, int grid, cudaStream_t s) {
-    stats_simulate_kernel<R, DT, NOISE, PE, IP><<<grid, kBlock, 0, s>>>(a);
-    return cudaGetLastError();
-  }
-};
-
-template <int R, int DT, bool IP>
-cudaError_t fused_run(const KArgs& a, int grid, int noise, bool pe, cudaStream_t s) {
-  if (noise == NOISE_GAUSSIAN)
-    return pe ? FusedVariant<R, DT, NOISE_GAUSSIAN, true, IP>::run(a, grid, s) : FusedVariant<R, DT, NOISE_GAUSSIAN, false, IP>::run(a, grid, s);
-  return pe ? FusedVariant<R, DT, NOISE_UNIFORM, true, IP>::run(a, grid, s) : FusedVariant<R, DT, NOISE_UNIFORM, false, IP>::run(a, grid, s);
-}
-
 template <typename Kernel>
 int occupancy_of(Kernel k) {
   int v = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, k, kBlock, 0) != cudaSuccess || v < 1) v = 1;
   return v;
+}
+
+template <int R, int DT, int NOISE, bool PE, bool IP, int MINB = ((DT == DT_BF16 && !PE) ? 3 : 2)>
+struct FusedVariant {
+  static int occ() {
+    static int v = occupancy_of(stats_simulate_kernel<R, DT, NOISE, PE, IP, MINB>);
+    return v;
+  }
+  static cudaError_t run(const KArgs& a, int grid, cudaStream_t s) {
+    stats_simulate_kernel<R, DT, NOISE, PE, IP, MINB><<<grid, kBlock, 0, s>>>(a);
+    return cudaGetLastError();
+  }
+};
+
+// wide: the list has statistics items (the four-CTA build for bf16 without
+// per-element alpha and not in place; the other cases have one build).
+template <int R, int DT, bool IP>
+cudaError_t fused_run(const KArgs& a, int grid, int noise, bool pe, bool wide, cudaStream_t s) {
+  if constexpr (DT == DT_BF16 && !IP) {
+    if (wide && !pe)
+      return noise == NOISE_GAUSSIAN ? FusedVariant<R, DT, NOISE_GAUSSIAN, false, IP, 4>::run(a, grid, s)
+                                     : FusedVariant<R, DT, NOISE_UNIFORM, false, IP, 4>::run(a, grid, s);
+  }
+  if (noise == NOISE_GAUSSIAN)
+    return pe ? FusedVariant<R, DT, NOISE_GAUSSIAN, true, IP>::run(a, grid, s) : FusedVariant<R, DT, NOISE_GAUSSIAN, false, IP>::run(a, grid, s);
+  return pe ? FusedVariant<R, DT, NOISE_UNIFORM, true, IP>::run(a, grid, s) : FusedVariant<R, DT, NOISE_UNIFORM, false, IP>::run(a, grid, s);
+}
+
+// Resident CTAs per SM of the launch fused_run makes.
+template <int R, int DT, bool IP>
+int fused_occ(int noise, bool pe, bool wide) {
+  if constexpr (DT == DT_BF16 && !IP) {
+    if (wide && !pe)
+      return noise == NOISE_GAUSSIAN ? FusedVariant<R, DT, NOISE_GAUSSIAN, false, IP, 4>::occ()
+                                     : FusedVariant<R, DT, NOISE_UNIFORM, false, IP, 4>::occ();
+  }
+  if (noise == NOISE_GAUSSIAN)
+    return pe ? FusedVariant<R, DT, NOISE_GAUSSIAN, true, IP>::occ() : FusedVariant<R, DT, NOISE_GAUSSIAN, false, IP>::occ();
+  return pe ? FusedVariant<R, DT, NOISE_UNIFORM, true, IP>::occ() : FusedVariant<R, DT, NOISE_UNIFORM, false, IP>::occ();
 }
 
 template <int R, int DT, int NOISE, bool PE, bool IP>
