@@ -494,8 +494,9 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
   if (e == cudaSuccess) e = cudaMemsetAsync(c->d_sync, 0, sizeof(int32_t) * sync_words(n_tensors), stream);
   c->wide = rel && cfg->alpha_mode != SMAT_ALPHA_PER_ELEMENT && cfg->noise != SMAT_NOISE_LAPLACE && !c->any_inplace;
   if (e == cudaSuccess && c->fused) {
-    // lead of about two grid widths of the bf16 forward
-    const int64_t lead = 2 * (int64_t)c->sm_count *
+    // lead of about one grid width of the bf16 forward (one, two and four
+    // measured on the 7B list: one is fastest)
+    const int64_t lead = (int64_t)c->sm_count *
                          (c->wide ? fused_wide_ctas_per_sm(cfg->noise, c->rounds)
                                   : streaming_ctas_per_sm(SMAT_BF16, cfg->noise,
                                                           cfg->alpha_mode == SMAT_ALPHA_PER_ELEMENT, c->rounds));

@@ -233,7 +233,7 @@ __device__ __forceinline__ void sim_chunk_noise(const KArgs& a, const TView& v, 
 // A persistent kernel that takes work items in list order from a counter:
 // statistics items (a2, one chunk each) and forward items (a3). Every
 // statistics item of a tensor precedes its forward items in the list (with a
-// lead of about two grid widths), so the bandwidth-bound statistics of later
+// lead of about one grid width), so the bandwidth-bound statistics of later
 // tensors run beside the compute-bound forward of earlier ones. The CTA that
 // finishes a tensor's last statistics chunk sums the chunk partials in chunk
 // order, publishes sigma_t and releases the tensor's ready flag; forward items
