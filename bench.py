@@ -72,6 +72,8 @@ def parse():
                     help="where theta0 lives: its own HBM buffer (default); in-place (the sim buffer holds theta0 "
                          "and is refilled from pinned host memory every step, inside the timed region); pinned "
                          "host memory read directly by the kernels")
+    ap.add_argument("--chunk-log2", type=int, default=0,
+                    help="force the work-chunk size to 2^k elements (12..18; 0: the per-list rule)")
     ap.add_argument("--philox-rounds", type=int, choices=[7, 10], default=10,
                     help="Philox-4x32 rounds of the random streams (10 is the default stream definition)")
     ap.add_argument("--sweep", metavar="PATH", default=None,
@@ -557,7 +559,8 @@ def run_smat(args):
         return S.SmatSession(th, t0, sim, [t.keep_prob for t in ts], [t.sigma for t in ts],
                              [t.sigma_rel for t in ts], tensor_ids=idx, seed=w.seed, alpha_min=w.alpha_min,
                              alpha_max=w.alpha_max, alpha_mode=w.alpha_mode, noise=w.noise,
-                             philox_rounds=args.philox_rounds)
+                             philox_rounds=args.philox_rounds,
+                             flags=S.SMAT_FLAG_CHUNK_LOG2(args.chunk_log2) if args.chunk_log2 else 0)
 
     th, t0, sim, gs, go = W.generate(w, device=dev)
     host_t0 = None
