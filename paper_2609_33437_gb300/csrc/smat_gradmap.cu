@@ -103,16 +103,28 @@ __device__ __forceinline__ void grad_chunk(const KArgs& a, const TView& v, const
       }
     }
   }
-#pragma unroll
+#pragma unroll 1
   for (int k = 0; k < 4; ++k) {
     if (k < tl.n) {
       const int64_t gb = ch.begin + 16 * (int64_t)tl.at(k);
-      uint32_t tb = group_ties16<R, J0>(a, v.tid, v.t_hi, (uint64_t)(v.off + gb));
-      while (tb) {
-        const int e = __ffs(tb) - 1;
-        tb &= tb - 1u;
-        if (tie_kept<R, J0>(a, v.tid, v.t_lo, (uint64_t)(v.off + gb + e)))
-          grad_elem_as<R, GDT, PE, ACC>(a, v, G, gb + e, true);
+      if (PE) {
+        // the group again, ties decided at once (g~ is still intact: no
+        // accumulation, g_out != g_sim); cheaper than element by element,
+        // where each tie element would draw its packed alpha field again
+        Raw16<GDT> gs1, go1;
+        load16<GDT>(G.g_sim, gb, gs1);
+        float out[16];
+        TieList none;
+        grad_compute16<R, GDT, PE, ACC, J0>(a, v, (uint64_t)(v.off + gb), (uint32_t)(gb - ch.begin), false, none, gs1, go1, out);
+        store16<GDT>(G.g_out, gb, out);
+      } else {
+        uint32_t tb = group_ties16<R, J0>(a, v.tid, v.t_hi, (uint64_t)(v.off + gb));
+        while (tb) {
+          const int e = __ffs(tb) - 1;
+          tb &= tb - 1u;
+          if (tie_kept<R, J0>(a, v.tid, v.t_lo, (uint64_t)(v.off + gb + e)))
+            grad_elem_as<R, GDT, PE, ACC>(a, v, G, gb + e, true);
+        }
       }
     }
   }
