@@ -392,6 +392,32 @@ __device__ __forceinline__ bool tie_kept(const KArgs& a, uint32_t tid, uint32_t 
   return (pick(l, (unsigned)(gidx & 3)) >> 8) < t_lo;
 }
 
+// Decide the ties of the group whose MASK block is w now (set their flags in kw).
+template <int R, bool J0>
+__device__ __forceinline__ void resolve_block_ties(const KArgs& a, uint32_t tid, uint32_t t_hi, uint32_t t_lo,
+                                                   const uint4& w, uint64_t gidx0, uint32_t (&kw)[4]) {
+  uint32_t tb = tie_bits16(w, t_hi);
+  while (tb) {
+    const int e = __ffs(tb) - 1;
+    tb &= tb - 1u;
+    if (tie_kept<R, J0>(a, tid, t_lo, gidx0 + (uint64_t)e)) set_kept(kw, e);
+  }
+}
+
+// Set the flags of every tie element of the group whose MASK block is w.
+__device__ __forceinline__ void set_tie_flags(const uint4& w, uint32_t t_hi, uint32_t (&kw)[4]) {
+  const uint32_t words[4] = {w.x, w.y, w.z, w.w};
+  const uint32_t tt = t_hi * 0x01010101u;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const uint32_t e = words[q] ^ tt;
+    kw[q] |= ~(((e & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | e) & 0x80808080u;  // exact per byte
+  }
+}
+
+// Whether a tie element is kept with probability at least 1/2 (t_lo / 2^24).
+__device__ __forceinline__ bool tie_mostly_kept(uint32_t t_lo) { return t_lo >= (1u << 23); }
+
 // Decide the group's ties now (set their flags in kw).
 template <int R, bool J0>
 __device__ __forceinline__ void resolve_group_ties(const KArgs& a, uint32_t tid, uint32_t t_hi, uint32_t t_lo,

@@ -6,17 +6,24 @@ namespace {
 
 // ---------------------------------------------------------- a5: gradient map ---
 // When `defer` (no accumulation and g_out distinct from g_sim, so the
-// incoming gradient can be re-read), tie elements are written as dropped (+0)
-// and queued; otherwise they are resolved at once.
+// incoming gradient can be re-read), tie elements are written with their
+// likelier outcome (kept when P(kept | tie) >= 1/2, else dropped) and the group
+// is queued: the pass after the chunk rewrites only the ties that went the
+// other way. Otherwise the ties are resolved at once.
 template <int R, int GDT, bool PE, bool ACC, bool J0>
 __device__ __forceinline__ void grad_compute16(const KArgs& a, const TView& v, uint64_t g0, uint32_t off,
                                                bool defer, TieList& tl, const Raw16<GDT>& gs,
                                                const Raw16<GDT>& go, float (&out)[16]) {
   uint32_t kw[4] = {0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u};
   if (v.flags & TF_MASK) {
-    const bool tie = group_keep16<R, J0>(a, v.tid, v.t_hi, g0, kw);
-    if (v.t_lo != 0u && tie && (ACC || !defer || !tl.push(off >> 4)))
-      resolve_group_ties<R, J0>(a, v.tid, v.t_hi, v.t_lo, g0, kw);
+    const uint4 mb = stream_block<R, J0>(a, S_MASK, v.tid, g0 >> 4);
+    const bool tie = keep_bytes16(mb, v.t_hi, kw);
+    if (v.t_lo != 0u && tie) {
+      if (ACC || !defer || !tl.push(off >> 4))
+        resolve_block_ties<R, J0>(a, v.tid, v.t_hi, v.t_lo, mb, g0, kw);
+      else if (tie_mostly_kept(v.t_lo))
+        set_tie_flags(mb, v.t_hi, kw);
+    }
   }
   // per-element alpha: three ALPHA_E blocks per group, three words per quad
   uint4 ab0 = make_uint4(0u, 0u, 0u, 0u), ab1 = ab0, ab2 = ab0;
@@ -103,14 +110,26 @@ __device__ __forceinline__ void grad_chunk(const KArgs& a, const TView& v, const
       }
     }
   }
+  // Queued groups (no accumulation here): each tie element whose decision
+  // differs from the outcome written for it. Rewriting a dropped tie needs no
+  // read of g~, so with P(kept | tie) >= 1/2 most of these passes read nothing.
+  const bool major = tie_mostly_kept(v.t_lo);
 #pragma unroll 1
   for (int k = 0; k < 4; ++k) {
     if (k < tl.n) {
       const int64_t gb = ch.begin + 16 * (int64_t)tl.at(k);
-      if (PE) {
+      uint32_t tb = group_ties16<R, J0>(a, v.tid, v.t_hi, (uint64_t)(v.off + gb));
+      uint32_t flip = 0u;
+      while (tb) {
+        const int e = __ffs(tb) - 1;
+        tb &= tb - 1u;
+        if (tie_kept<R, J0>(a, v.tid, v.t_lo, (uint64_t)(v.off + gb + e)) != major) flip |= 1u << e;
+      }
+      if (flip == 0u) continue;
+      if (PE && !major) {
         // the group again, ties decided at once (g~ is still intact: no
         // accumulation, g_out != g_sim); cheaper than element by element,
-        // where each tie element would draw its packed alpha field again
+        // where each kept tie would draw its packed alpha field again
         Raw16<GDT> gs1, go1;
         load16<GDT>(G.g_sim, gb, gs1);
         float out[16];
@@ -118,11 +137,12 @@ __device__ __forceinline__ void grad_chunk(const KArgs& a, const TView& v, const
         grad_compute16<R, GDT, PE, ACC, J0>(a, v, (uint64_t)(v.off + gb), (uint32_t)(gb - ch.begin), false, none, gs1, go1, out);
         store16<GDT>(G.g_out, gb, out);
       } else {
-        uint32_t tb = group_ties16<R, J0>(a, v.tid, v.t_hi, (uint64_t)(v.off + gb));
-        while (tb) {
-          const int e = __ffs(tb) - 1;
-          tb &= tb - 1u;
-          if (tie_kept<R, J0>(a, v.tid, v.t_lo, (uint64_t)(v.off + gb + e)))
+        while (flip) {
+          const int e = __ffs(flip) - 1;
+          flip &= flip - 1u;
+          if (major)
+            store1<GDT>(G.g_out, gb + e, 0.0f);  // dropped: +0
+          else
             grad_elem_as<R, GDT, PE, ACC>(a, v, G, gb + e, true);
         }
       }
