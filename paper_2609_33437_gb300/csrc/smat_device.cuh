@@ -169,6 +169,16 @@ __device__ __forceinline__ float2 add2_rn(float2 a, float2 b) {
   return d;
 }
 
+__device__ __forceinline__ float2 sub2_rn(float2 a, float2 b) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+      "sub.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+
 __device__ __forceinline__ float2 fma2_rn(float2 a, float2 b, float2 c) {
   float2 d;
   asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
@@ -614,7 +624,7 @@ __device__ __forceinline__ void delta_group(const Raw16<DT>& th, const Raw16<DT>
 #pragma unroll
   for (int m = 0; m < 8; ++m) {
     const float2 a = th.pair(m), b = t0.pair(m);
-    const float2 d = add2_rn(a, make_float2(-b.x, -b.y));
+    const float2 d = sub2_rn(a, b);
     s2 = add2_rn(s2, d);
     q2 = fma2_rn(d, d, q2);
   }

@@ -80,7 +80,7 @@ __device__ __forceinline__ void merge_acc16(float c, uint32_t keep, const Raw16<
 #pragma unroll
   for (int h = 0; h < 8; ++h) {
     const float2 b = t0.pair(h);
-    const float2 d = add2_rn(x.pair(h), make_float2(-b.x, -b.y));
+    const float2 d = sub2_rn(x.pair(h), b);
     const float2 f = fma2_rn(c2, d, acc[h]);
     acc[h] = make_float2(((keep >> (2 * h)) & 1u) ? f.x : acc[h].x, ((keep >> (2 * h + 1)) & 1u) ? f.y : acc[h].y);
   }
@@ -233,8 +233,7 @@ __device__ __forceinline__ void dare_acc16_blend(float c, const uint4& km, const
     const uint32_t lm = __byte_perm(kmw[h >> 1], 0u, (h & 1) ? 0x3322u : 0x1100u);
     const uint32_t xw = (x.r[h] & lm) | (t0.r[h] & ~lm);
     const float2 b = t0.pair(h);
-    const float2 d = add2_rn(make_float2(__uint_as_float(xw << 16), __uint_as_float(xw & 0xFFFF0000u)),
-                             make_float2(-b.x, -b.y));
+    const float2 d = sub2_rn(make_float2(__uint_as_float(xw << 16), __uint_as_float(xw & 0xFFFF0000u)), b);
     acc[h] = fma2_rn(c2, d, acc[h]);
   }
 }
@@ -249,7 +248,7 @@ __device__ __forceinline__ void dare_acc16_select(float c, const uint4& km, cons
 #pragma unroll
   for (int h = 0; h < 8; ++h) {
     const float2 b = t0.pair(h);
-    const float2 d = add2_rn(x.pair(h), make_float2(-b.x, -b.y));
+    const float2 d = sub2_rn(x.pair(h), b);
     const float2 f = fma2_rn(c2, d, acc[h]);
     acc[h] = make_float2(kept_of(kw, 2 * h) ? f.x : acc[h].x, kept_of(kw, 2 * h + 1) ? f.y : acc[h].y);
   }
@@ -320,7 +319,7 @@ __device__ __forceinline__ void merge_ties16(const MArgs& m, const MTensor& T, i
 #pragma unroll
     for (int h = 0; h < 8; ++h) {
       const float2 b = t0.pair(h);
-      const float2 d = add2_rn(x.pair(h), make_float2(-b.x, -b.y));
+      const float2 d = sub2_rn(x.pair(h), b);
       if (abs_key(d.x) >= thr) sum[2 * h] = __fadd_rn(sum[2 * h], d.x);
       if (abs_key(d.y) >= thr) sum[2 * h + 1] = __fadd_rn(sum[2 * h + 1], d.y);
     }
@@ -354,7 +353,7 @@ __device__ __forceinline__ void merge_ties16(const MArgs& m, const MTensor& T, i
 #pragma unroll
     for (int h = 0; h < 8; ++h) {
       const float2 b = t0.pair(h);
-      const float2 d = add2_rn(x.pair(h), make_float2(-b.x, -b.y));
+      const float2 d = sub2_rn(x.pair(h), b);
       if (agree(d.x, lo, 2 * h)) {
         part[2 * h] = __fadd_rn(part[2 * h], d.x);
         cnt[h >> 1] += 1u << (16 * (h & 1));

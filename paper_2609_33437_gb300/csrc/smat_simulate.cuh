@@ -75,12 +75,12 @@ __device__ __forceinline__ uint32_t sim_group16(const KArgs& a, const TView& v, 
       if (PE) {
         const float2 cc = make_float2(__fmul_rn(alpha_of24(a, ua[2 * h]), v.inv_keep),
                                       __fmul_rn(alpha_of24(a, ua[2 * h + 1]), v.inv_keep));
-        const float2 f = fma2_rn(cc, add2_rn(th2, make_float2(-t02.x, -t02.y)), t02);
+        const float2 f = fma2_rn(cc, sub2_rn(th2, t02), t02);
         kv = make_float2(cc.x == 1.0f ? th2.x : f.x, cc.y == 1.0f ? th2.y : f.y);
       } else if (IDENT) {
         kv = th2;
       } else {
-        kv = fma2_rn(c2, add2_rn(th2, make_float2(-t02.x, -t02.y)), t02);
+        kv = fma2_rn(c2, sub2_rn(th2, t02), t02);
       }
       float x0 = kept_of(kw, e0) ? kv.x : t02.x;
       float x1 = kept_of(kw, e0 + 1) ? kv.y : t02.y;

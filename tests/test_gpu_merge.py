@@ -138,6 +138,18 @@ def test_merge_dare_seven_rounds():
         assert np.array_equal(to_host(out).view(np.uint16), ref.view(np.uint16)), k
 
 
+@pytest.mark.parametrize("K", [1, 2, 8, 9, 15, 16])
+def test_merge_dare_expert_counts(K):
+    """DARE with one to sixteen experts (the kernel loads experts in batches
+    of four, so every remainder occurs) equals the oracle."""
+    t0s, exs = _experts([17, 4096, 65_536 + 33], K, O.BF16, seed=40 + K)
+    outs = [torch.empty_like(t) for t in t0s]
+    kw = dict(gamma=0.6, p_drop=0.3, seed=5)
+    S.merge(t0s, exs, outs, S.SMAT_MERGE_DARE_TA, **kw)
+    torch.cuda.synchronize()
+    _check(t0s, exs, outs, O.BF16, S.SMAT_MERGE_DARE_TA, kw)
+
+
 @pytest.mark.parametrize("method", list(METHODS))
 @pytest.mark.parametrize("dtype", [O.F32, O.BF16])
 def test_merge_special_values(method, dtype):
