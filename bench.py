@@ -345,10 +345,11 @@ class PinnedHost:
     """Pinned host buffers for the end-to-end leg. Each one is an anonymous
     mapping advised for transparent huge pages (madvise(MADV_HUGEPAGE)),
     faulted in and registered with cudaHostRegister: the copy engines then
-    translate a few hundred large pages instead of about a million 64 KB ones,
-    which on this machine keeps a step's 67 GB of copies at about 240 GB/s
-    instead of 165. Falls back to torch's pinned allocator where any step
-    fails. close() unregisters them."""
+    translate a few hundred large pages instead of about a million 64 KB ones
+    (measured: a step's 67 GB of copies at about 240 GB/s instead of 165 when
+    the kernel had huge pages free; where it has none the mapping keeps base
+    pages, see huge_page_fraction()). Falls back to torch's pinned allocator
+    where any step fails. close() unregisters them."""
 
     def __init__(self):
         self._maps, self._registered = [], []
@@ -375,6 +376,22 @@ class PinnedHost:
                 pass
             self.huge = False
         return torch.empty(n, dtype=dtype, pin_memory=True)
+
+    def huge_page_fraction(self):
+        """Share of this process's anonymous memory backed by transparent huge
+        pages (AnonHugePages / Anonymous in /proc/self/smaps_rollup), or None:
+        where the kernel had no free huge pages the buffers fall back to base
+        pages and the copies slow down."""
+        try:
+            vals = {}
+            with open("/proc/self/smaps_rollup") as f:
+                for line in f:
+                    k, _, rest = line.partition(":")
+                    if k in ("AnonHugePages", "Anonymous"):
+                        vals[k] = int(rest.split()[0])
+            return vals["AnonHugePages"] / vals["Anonymous"] if vals.get("Anonymous") else None
+        except Exception:
+            return None
 
     def close(self):
         for raw in self._registered:
@@ -615,6 +632,7 @@ def e2e_run(w, sess_factory, steps, warmup, world, groups=8, keep_outputs=False,
     if saved:
         os.sched_setaffinity(0, saved)
     huge = pinned.huge
+    huge_frac = pinned.huge_page_fraction() if huge else None
     pinned.close()
     host_gbs = (h2d + d2h) * steps / el / 1e9
     return {"value": world * bytes_step * steps / el / 1e9, "unit": UNIT, "h2d_bytes_per_step": h2d,
@@ -623,6 +641,7 @@ def e2e_run(w, sess_factory, steps, warmup, world, groups=8, keep_outputs=False,
                         f"one compute and {copy_streams} copy-out streams",
             "host_numa_node": local[0] if local else None,
             "host_buffers": "huge-page mappings registered with cudaHostRegister" if huge else "torch pinned memory",
+            "host_huge_page_fraction": huge_frac,
             "host_link_gbs": host_gbs, "link_roof_gbs": roof,
             "frac_of_link_roof": host_gbs / roof["step_copies"] if roof["step_copies"] > 0 else None}
 
