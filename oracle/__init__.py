@@ -28,7 +28,7 @@ class OrcConfig(ctypes.Structure):
     _fields_ = [("seed", ctypes.c_uint64), ("step", ctypes.c_uint32),
                 ("rounds", ctypes.c_int32), ("alpha_mode", ctypes.c_int32),
                 ("noise", ctypes.c_int32), ("alpha_min", ctypes.c_float),
-                ("alpha_max", ctypes.c_float)]
+                ("alpha_max", ctypes.c_float), ("draw_bits", ctypes.c_int32)]
 
 
 class OrcTensor(ctypes.Structure):
@@ -88,8 +88,8 @@ def _c(a, dtype):
 
 
 def config(seed=0, step=0, rounds=10, alpha_mode=ALPHA_PER_TENSOR, noise=NOISE_UNIFORM,
-           alpha_min=0.3, alpha_max=1.0):
-    return OrcConfig(seed, step, rounds, alpha_mode, noise, alpha_min, alpha_max)
+           alpha_min=0.3, alpha_max=1.0, draw_bits=32):
+    return OrcConfig(seed, step, rounds, alpha_mode, noise, alpha_min, alpha_max, draw_bits)
 
 
 def tensor(tensor_id, numel, dtype=F32, keep_prob=0.9, sigma=0.0, sigma_rel=0.0, elem_offset=0):

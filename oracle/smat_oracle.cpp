@@ -50,6 +50,16 @@
 //           t_a = 0x0FFFFFFF (one alpha for all tensors) or the tensor id;
 //           per element alpha = fma(amax - amin, F(ALPHA_E, tid, gidx) 2^-24, amin)
 //
+//   The 16-bit draw option (draw_bits = 16; the layout above is draw_bits = 32):
+//   each per-element draw is the 16-bit value
+//     D(stream, tid, gidx) = half (gidx & 1), low half first, of word
+//                            (gidx & 7) >> 1 of W(stream, tid, gidx >> 3)
+//   (eight elements per block, no packing): Mask U16 = D(MASK, tid, gidx),
+//   kept <=> U16 < T16 = floor(p_keep * 2^16) (no MASK_LO part); noise
+//   v = sym16(D(NOISE, tid, gidx)) = (2u + 1 - 2^16) 2^-16 in place of sym24 in
+//   every law; per element alpha = fma(amax - amin, D(ALPHA_E, tid, gidx) 2^-16,
+//   amin). The per-tensor alpha is unchanged.
+//
 // Merging (the evaluation side, Eq. merged-state): theta_merge = theta0 +
 // sum_j alpha_j (.) m_j (.) Delta_j over K experts, Delta_j = theta_j - theta0
 // (one fp32 subtraction), accumulated over j = 0 .. K-1 in that order:
@@ -129,6 +139,7 @@ struct OrcConfig {
   int32_t noise;       // NOISE_UNIFORM / NOISE_GAUSSIAN / NOISE_LAPLACE
   float alpha_min;
   float alpha_max;
+  int32_t draw_bits;   // 32 (the packed layout; 0 reads as 32) or 16 (the 16-bit draw option)
 };
 
 struct OrcTensor {
@@ -156,6 +167,16 @@ uint32_t stream_word(const OrcConfig& cfg, uint32_t stream, uint32_t tid,
 }
 
 const float kTwoPow24Inv = 5.9604644775390625e-08f;  // 2^-24, exact
+const float kTwoPow16Inv = 1.52587890625e-05f;       // 2^-16, exact
+
+bool draws16(const OrcConfig& cfg) { return cfg.draw_bits == 16; }
+
+// 16-bit draw of element gidx in a per-element stream (the 16-bit option):
+// half gidx & 1 (low half first) of word (gidx & 7) >> 1 of block gidx >> 3.
+uint32_t draw16(const OrcConfig& cfg, uint32_t stream, uint32_t tid, uint64_t gidx) {
+  const uint32_t w = stream_word(cfg, stream, tid, gidx >> 3, (unsigned)((gidx & 7) >> 1));
+  return (gidx & 1) ? (w >> 16) : (w & 0xFFFFu);
+}
 
 float u01(uint32_t u) { return (float)(u >> 8) * kTwoPow24Inv; }
 
@@ -202,7 +223,7 @@ struct Scalars {
   float alpha;        // per-tensor alpha (unused in per-element mode)
   float inv_keep;     // 1 / p_keep  (Eq. smat-mask: 1 / (1 - p))
   float c;            // alpha * inv_keep
-  uint64_t T;         // keep threshold on the 32-bit mask uniform
+  uint64_t T;         // keep threshold on the 32-bit mask uniform (16-bit option: on U16)
   float sigma;        // Perturb RMS for this call
   float noise_scale;  // fl(sqrt3 sigma) (uniform), fl(sqrt2 sigma) (Gaussian), fl(sigma / sqrt2) (Laplace)
 };
@@ -250,7 +271,7 @@ Scalars make_scalars(const OrcConfig& cfg, const OrcTensor& t, float sigma) {
   }
   s.inv_keep = (t.keep_prob > 0.0f) ? (float)(1.0 / (double)t.keep_prob) : 0.0f;
   s.c = s.alpha * s.inv_keep;
-  s.T = (uint64_t)std::floor((double)t.keep_prob * 4294967296.0);
+  s.T = (uint64_t)std::floor((double)t.keep_prob * (draws16(cfg) ? 65536.0 : 4294967296.0));
   s.sigma = sigma;
   s.noise_scale = (float)(std::sqrt(cfg.noise == NOISE_UNIFORM ? 3.0 : cfg.noise == NOISE_GAUSSIAN ? 2.0 : 0.5) *
                           (double)sigma);
@@ -259,6 +280,7 @@ Scalars make_scalars(const OrcConfig& cfg, const OrcTensor& t, float sigma) {
 
 // ------------------------------------------------------- element values ---
 bool is_kept(const OrcConfig& cfg, const OrcTensor& t, const Scalars& s, uint64_t gidx) {
+  if (draws16(cfg)) return (uint64_t)draw16(cfg, S_MASK, t.tensor_id, gidx) < s.T;
   const uint32_t hw = stream_word(cfg, S_MASK, t.tensor_id, gidx >> 4, (unsigned)((gidx >> 2) & 3));
   const uint32_t hi = (hw >> (8u * (unsigned)(gidx & 3))) & 0xFFu;
   const uint32_t lo = stream_word(cfg, S_MASK_LO, t.tensor_id, gidx >> 2, (unsigned)(gidx & 3)) >> 8;
@@ -282,12 +304,14 @@ uint32_t field24(const OrcConfig& cfg, uint32_t stream, uint32_t tid, uint64_t g
 }
 
 // Scale per coordinate: alpha ~ U[alpha_min, alpha_max) from the element's
-// 24-bit ALPHA_E field, then c = alpha / p_keep (Eq. smat-mask rescale).
+// 24-bit ALPHA_E field (16-bit option: its 16-bit draw), then c = alpha /
+// p_keep (Eq. smat-mask rescale).
 float element_c(const OrcConfig& cfg, const OrcTensor& t, const Scalars& s, uint64_t gidx) {
   if (cfg.alpha_mode != ALPHA_PER_ELEMENT) return s.c;
   const float width = cfg.alpha_max - cfg.alpha_min;
-  const uint32_t u = field24(cfg, S_ALPHA_E, t.tensor_id, gidx);
-  const float alpha = std::fma(width, (float)u * kTwoPow24Inv, cfg.alpha_min);
+  const float u01e = draws16(cfg) ? (float)draw16(cfg, S_ALPHA_E, t.tensor_id, gidx) * kTwoPow16Inv
+                                  : (float)field24(cfg, S_ALPHA_E, t.tensor_id, gidx) * kTwoPow24Inv;
+  const float alpha = std::fma(width, u01e, cfg.alpha_min);
   return alpha * s.inv_keep;
 }
 
@@ -321,8 +345,16 @@ uint32_t noise_field(const OrcConfig& cfg, const OrcTensor& t, uint64_t gidx) {
   return field24(cfg, S_NOISE, t.tensor_id, gidx);
 }
 
-float sym24(uint32_t u24) { return (float)(2 * (int32_t)u24 + 1 - (1 << 24)) * kTwoPow24Inv; }
 double sym24_d(uint32_t u24) { return (double)(2 * (int64_t)u24 + 1 - (1 << 24)) * 0x1p-24; }
+double sym16_d(uint32_t u16) { return (double)(2 * (int64_t)u16 + 1 - (1 << 16)) * 0x1p-16; }
+
+// The symmetric uniform v in (-1, 1) of element gidx's noise draw: sym24 of its
+// 24-bit field, or sym16 of its 16-bit draw. Exact in fp32 and double (an odd
+// multiple of 2^-24 or 2^-16 below 1 in magnitude).
+double noise_v(const OrcConfig& cfg, const OrcTensor& t, uint64_t gidx) {
+  if (draws16(cfg)) return sym16_d(draw16(cfg, S_NOISE, t.tensor_id, gidx));
+  return sym24_d(noise_field(cfg, t, gidx));
+}
 
 // Laplace(0, 1) variate of v in (-1, 1) by the inverse CDF: -sign(v) ln(1 - |v|).
 double laplace_d(double v) {
@@ -330,16 +362,16 @@ double laplace_d(double v) {
   return v < 0.0 ? -z : z;
 }
 
-// Unit-variance normal variate of element gidx: sqrt2 erfinv(sym24(u)).
+// Unit-variance normal variate of element gidx: sqrt2 erfinv(v).
 double gauss_z(const OrcConfig& cfg, const OrcTensor& t, uint64_t gidx) {
-  return std::sqrt(2.0) * erfinv_d(sym24_d(noise_field(cfg, t, gidx)));
+  return std::sqrt(2.0) * erfinv_d(noise_v(cfg, t, gidx));
 }
 
 float noise_eps(const OrcConfig& cfg, const OrcTensor& t, const Scalars& s, uint64_t gidx) {
-  const uint32_t u = noise_field(cfg, t, gidx);
-  if (cfg.noise == NOISE_UNIFORM) return s.noise_scale * sym24(u);
-  if (cfg.noise == NOISE_LAPLACE) return s.noise_scale * (float)laplace_d(sym24_d(u));
-  return s.noise_scale * (float)erfinv_d(sym24_d(u));
+  const double v = noise_v(cfg, t, gidx);
+  if (cfg.noise == NOISE_UNIFORM) return s.noise_scale * (float)v;
+  if (cfg.noise == NOISE_LAPLACE) return s.noise_scale * (float)laplace_d(v);
+  return s.noise_scale * (float)erfinv_d(v);
 }
 
 // Eq. smat-state for one element, fp32 arithmetic, before the storage rounding.
@@ -397,11 +429,11 @@ void orc_laplace(const double* v, int64_t n, double* out) {
 }
 
 // Unit-variance variate of each element's noise under the config's law:
-// sqrt3 sym24(u) (uniform), sqrt2 erfinv(sym24(u)) (Gaussian),
-// laplace(sym24(u)) / sqrt2 (Laplace).
+// sqrt3 v (uniform), sqrt2 erfinv(v) (Gaussian), laplace(v) / sqrt2 (Laplace),
+// v the element's symmetric uniform (noise_v).
 void orc_noise_z(const OrcConfig* cfg, const OrcTensor* t, const uint64_t* gidx, int64_t n, double* z) {
   for (int64_t k = 0; k < n; ++k) {
-    const double v = sym24_d(noise_field(*cfg, *t, gidx[k]));
+    const double v = noise_v(*cfg, *t, gidx[k]);
     z[k] = cfg->noise == NOISE_UNIFORM    ? std::sqrt(3.0) * v
            : cfg->noise == NOISE_GAUSSIAN ? std::sqrt(2.0) * erfinv_d(v)
                                           : laplace_d(v) / std::sqrt(2.0);
@@ -508,13 +540,13 @@ void orc_simulate_f64(const OrcConfig* cfg, const OrcTensor* t, float sigma_t, c
       x = t0[i] + c * (th[i] - t0[i]);
     }
     if (s.sigma > 0.0f) {
-      const uint32_t u = noise_field(*cfg, *t, gidx);
+      const double v = noise_v(*cfg, *t, gidx);
       if (cfg->noise == NOISE_UNIFORM)
-        x += (double)s.noise_scale * (double)sym24(u);
+        x += (double)s.noise_scale * v;
       else if (cfg->noise == NOISE_LAPLACE)
-        x += (double)s.noise_scale * laplace_d(sym24_d(u));
+        x += (double)s.noise_scale * laplace_d(v);
       else
-        x += (double)s.noise_scale * erfinv_d(sym24_d(u));
+        x += (double)s.noise_scale * erfinv_d(v);
     }
     out[i] = x;
   }
@@ -643,6 +675,7 @@ void orc_merge(const OrcMerge* m, uint32_t tensor_id, int32_t dtype, int64_t n, 
           cfg.noise = NOISE_UNIFORM;
           cfg.alpha_min = 0.0f;
           cfg.alpha_max = 1.0f;
+          cfg.draw_bits = 32;  // DARE masks use the packed mask layout
           Scalars s;
           s.T = (uint64_t)std::floor((double)keep * 4294967296.0);
           if (is_kept(cfg, mt, s, gidx)) acc = std::fma(c_dare, d, acc);

@@ -46,6 +46,14 @@ def main():
              O.f32_to_bf16(gs), O.BF16),
         case("f32_laplace_per_tensor", O.config(seed=11, step=5, noise=O.NOISE_LAPLACE, alpha_min=0.3),
              O.tensor(6, n, O.F32, keep_prob=0.7, sigma=2e-3), th, t0, gs, O.F32),
+        case("bf16_gauss_per_element_draw16", O.config(seed=19, step=4, noise=O.NOISE_GAUSSIAN,
+                                                       alpha_mode=O.ALPHA_PER_ELEMENT, alpha_min=0.1,
+                                                       draw_bits=16),
+             O.tensor(12, n, O.BF16, keep_prob=0.3, sigma=1e-4, elem_offset=5), O.f32_to_bf16(th),
+             O.f32_to_bf16(t0), O.f32_to_bf16(gs), O.BF16),
+        case("f32_uniform_per_tensor_draw16", O.config(seed=23, step=0, noise=O.NOISE_UNIFORM, alpha_min=0.4,
+                                                       draw_bits=16),
+             O.tensor(14, n, O.F32, keep_prob=0.7, sigma=2e-3), th, t0, gs, O.F32),
     ]
     doc = {"about": "CPU-oracle outputs on fixed inputs; regression guard for the oracle "
                     "(written by tests/golden/make_golden.py, oracle/ only)",

@@ -885,3 +885,101 @@ def test_merge_ties_degenerate_cases():
     inf = np.array([np.inf, 2, 2, 2], np.float32)
     out, _ = O.merge(O.MERGE_TIES, z4, [inf, np.ones(4, np.float32)], gamma=0.5, retention=1.0)
     assert np.array_equal(out, np.array([np.inf, 0.75, 0.75, 0.75], np.float32))
+
+
+# ------------------------------------------------------- 16-bit draw option ---
+
+def _draw16(words4, gidx):
+    """Element gidx's 16-bit draw from the four words of block gidx >> 3:
+    half gidx & 1 (low half first) of word (gidx & 7) >> 1."""
+    w = int(words4[(gidx & 7) >> 1])
+    return (w >> 16) if gidx & 1 else (w & 0xFFFF)
+
+
+def test_draw16_layout_matches_triton_library():
+    """The 16-bit draw option (draw_bits = 16, the 16-bit layout of the
+    hot-path contract): element gidx's draw in the MASK, NOISE and ALPHA_E
+    streams is half gidx & 1 (low half first) of word (gidx & 7) >> 1 of
+    Triton's Philox block j = gidx >> 3 of that stream. Checked through the
+    oracle's outputs: the keep bits (kept iff the draw is below floor(p 2^16)),
+    uniform noise (eps / (sqrt3 sigma) = (2D + 1 - 2^16) 2^-16) and per-element
+    alpha ((alpha - alpha_min) / (alpha_max - alpha_min) = D 2^-16), each up to
+    fp32 rounding; element offsets with block indices at and above 2^32."""
+    seed, step, tid, p, sigma, amin, amax = 0x5EED5EED12345678, 9, 0x0345678, 0.37, 1e-3, 0.2, 0.9
+    cases = [(0, 40), (5, 11), ((1 << 35) - 7, 16), (5 << 35, 8)]
+    need = sorted({(s, (off + i) >> 3) for s in (0, 1, 2) for off, n in cases for i in range(n)})
+    assert any(j >> 32 for _, j in need)
+    words = _triton_philox([[j & 0xFFFFFFFF, j >> 32, (s << 28) | tid, step] for s, j in need],
+                           [seed] * len(need), 10)
+    W = {key: words[k] for k, key in enumerate(need)}
+    T16 = math.floor(p * 65536)
+    for off, n in cases:
+        gid = [off + i for i in range(n)]
+        cfg = O.config(seed=seed, step=step, draw_bits=16, noise=O.NOISE_UNIFORM)
+        t = O.tensor(tid, n, keep_prob=p, elem_offset=off)
+        kept = O.unpack_bits(O.mask_bits(cfg, t), n).astype(bool)
+        assert np.array_equal(kept, [_draw16(W[(0, g >> 3)], g) < T16 for g in gid]), off
+        # every coordinate dropped and theta0 = 0: theta~ = eps
+        t0 = O.tensor(tid, n, keep_prob=0.0, sigma=sigma, elem_offset=off)
+        z = np.zeros(n, np.float32)
+        eps = O.simulate(cfg, t0, z, z).astype(np.float64) / (math.sqrt(3.0) * float(np.float32(sigma)))
+        v = np.array([(2 * _draw16(W[(1, g >> 3)], g) + 1 - 65536) * 2.0**-16 for g in gid])
+        assert np.all(np.abs(eps - v) <= 4e-7 * np.abs(v)), (off, np.max(np.abs(eps - v)))
+        v_nb = np.array([(2 * _draw16(W[(1, (g ^ 1) >> 3)], g ^ 1) + 1 - 65536) * 2.0**-16 for g in gid])
+        assert np.mean(np.abs(eps - v_nb) <= 4e-7 * np.abs(v_nb)) < 0.2
+        # the threshold itself: p = D_k / 2^16 (exact in fp32) drops element k
+        # (the compare is strict) and keeps every draw below D_k
+        dk = _draw16(W[(0, gid[3] >> 3)], gid[3])
+        te = O.tensor(tid, n, keep_prob=float(np.float32(dk / 65536)), elem_offset=off)
+        ke = O.unpack_bits(O.mask_bits(cfg, te), n).astype(bool)
+        assert not ke[3]
+        assert np.array_equal(ke, [_draw16(W[(0, g >> 3)], g) < dk for g in gid])
+        assert O.unpack_bits(O.mask_bits(cfg, O.tensor(tid, n, keep_prob=1.0, elem_offset=off)), n).all()
+        cfa = O.config(seed=seed, step=step, draw_bits=16, alpha_mode=O.ALPHA_PER_ELEMENT,
+                       alpha_min=amin, alpha_max=amax)
+        back = (_alpha_per_element(cfa, tid, n, elem_offset=off) - amin) / (amax - amin)
+        d = np.array([_draw16(W[(2, g >> 3)], g) * 2.0**-16 for g in gid])
+        assert np.all(np.abs(back - d) <= 2.0**-22), (off, np.max(np.abs(back - d)))
+
+
+@pytest.mark.parametrize("p", [0.3, 0.25, 0.9])
+def test_draw16_keep_rate_and_gradient_support(p):
+    """16-bit draws: the keep rate is floor(p 2^16) / 2^16 (a binomial 5-sigma
+    bound over 2^18 coordinates), the 32-bit layout's keep decisions are a
+    different, independent draw, and the gradient map (Eq. smat-gradient) is
+    zero exactly on the dropped coordinates."""
+    n = 1 << 18
+    cfg16 = O.config(seed=41, step=2, draw_bits=16)
+    t = O.tensor(77, n, keep_prob=p)
+    k16 = O.unpack_bits(O.mask_bits(cfg16, t), n).astype(bool)
+    q = math.floor(p * 65536) / 65536
+    assert abs(k16.mean() - q) < 5 * math.sqrt(q * (1 - q) / n)
+    k32 = O.unpack_bits(O.mask_bits(O.config(seed=41, step=2), t), n).astype(bool)
+    agree = np.mean(k16 == k32)
+    assert abs(agree - (q * q + (1 - q) * (1 - q))) < 5 * math.sqrt(0.25 / n)
+    g = O.gradmap(cfg16, t, np.ones(n, np.float32))
+    assert np.array_equal(g != 0, k16)
+
+
+def test_draw16_gaussian_and_alpha_laws():
+    """16-bit draws: Gaussian Perturb is N(0, sigma^2) up to the 2^-16 grid
+    (KS against N(0, 1), unit variance, symmetric, |z| at most
+    sqrt2 erfinv(1 - 2^-16)); per-element alpha is U[alpha_min, alpha_max)
+    (KS) and independent of the neighbouring coordinate."""
+    from scipy.special import erfinv as sp_erfinv
+    n, sigma = 200_000, 1e-4
+    t = O.tensor(8, n, keep_prob=0.0, sigma=sigma)
+    z = np.zeros(n, np.float32)
+    eps = O.simulate(O.config(seed=6, noise=O.NOISE_GAUSSIAN, draw_bits=16), t, z, z).astype(np.float64) / sigma
+    assert stats.kstest(eps, "norm").pvalue > 1e-4
+    assert abs(eps.var() - 1) < 5 * math.sqrt(2.0 / n)
+    assert abs(eps.mean()) < 5 / math.sqrt(n)
+    assert np.max(np.abs(eps)) <= math.sqrt(2.0) * sp_erfinv(1 - 2.0**-16) * (1 + 1e-6)
+    eps32 = O.simulate(O.config(seed=6, noise=O.NOISE_GAUSSIAN), t, z, z).astype(np.float64) / sigma
+    assert abs(np.corrcoef(eps, eps32)[0, 1]) < 5 / math.sqrt(n)
+    amin, amax = 0.3, 0.8
+    cfa = O.config(seed=32, step=1, draw_bits=16, alpha_mode=O.ALPHA_PER_ELEMENT, alpha_min=amin, alpha_max=amax)
+    a = _alpha_per_element(cfa, 90, n)
+    assert np.all((a >= amin) & (a < amax))
+    assert stats.kstest((a - amin) / (amax - amin), "uniform").pvalue > 1e-4
+    assert abs(np.corrcoef(a[:-1], a[1:])[0, 1]) < 5 / math.sqrt(n)
