@@ -76,6 +76,9 @@ def parse():
                     help="force the work-chunk size to 2^k elements (12..18; 0: the per-list rule)")
     ap.add_argument("--philox-rounds", type=int, choices=[7, 10], default=10,
                     help="Philox-4x32 rounds of the random streams (10 is the default stream definition)")
+    ap.add_argument("--draw-bits", type=int, choices=[32, 16], default=32,
+                    help="per-element draw width: 32 (the default stream definition) or 16 (the 16-bit draw "
+                         "option: eight elements per Philox block, no mask-tie path; a different stream)")
     ap.add_argument("--sweep", metavar="PATH", default=None,
                     help="run the flat-tensor sweep, one JSON line per point to PATH")
     ap.add_argument("--sweep-max-log2n", type=int, default=32)
@@ -660,7 +663,7 @@ def run_smat(args):
         return S.SmatSession(th, t0, sim, [t.keep_prob for t in ts], [t.sigma for t in ts],
                              [t.sigma_rel for t in ts], tensor_ids=idx, seed=w.seed, alpha_min=w.alpha_min,
                              alpha_max=w.alpha_max, alpha_mode=w.alpha_mode, noise=w.noise,
-                             philox_rounds=args.philox_rounds,
+                             philox_rounds=args.philox_rounds, draw_bits=args.draw_bits,
                              flags=S.SMAT_FLAG_CHUNK_LOG2(args.chunk_log2) if args.chunk_log2 else 0)
 
     th, t0, sim, gs, go = W.generate(w, device=dev)
@@ -755,7 +758,7 @@ def run_smat(args):
                           "param_dtype": "bf16" if w.dtype == W.BF16 else "f32",
                           "grad_dtype": "bf16" if w.gdtype == W.BF16 else "f32",
                           "noise": NOISE_NAME[w.noise], "alpha": f"per-tensor U[{w.alpha_min}, {w.alpha_max})",
-                          "philox_rounds": args.philox_rounds,
+                          "philox_rounds": args.philox_rounds, "draw_bits": args.draw_bits,
                           "bytes_per_step": bytes_step,
                           "l2": ("256 MB written before each timed step (the step's data would fit in L2)" if small
                                  else "inputs larger than L2 (no flush needed)"),
@@ -830,7 +833,7 @@ def run_sweep(args):
                             w = W.flat_sweep(log2n, dt, keep, am, sig)
                             sess = S.SmatSession(th, t0, sim, [keep], [sig], [0.0], seed=w.seed,
                                                  alpha_min=w.alpha_min, alpha_max=w.alpha_max, alpha_mode=am,
-                                                 noise=w.noise)
+                                                 noise=w.noise, draw_bits=args.draw_bits)
 
                             def fwd(s):
                                 sess.simulate_multi(s)

@@ -114,6 +114,19 @@ typedef struct {
 #define SMAT_FLAG_CHUNK_LOG2(k) ((k) << 8)
 #define SMAT_FLAG_CHUNK_LOG2_MASK 0x1F00
 
+/* The random draws (the paper fixes only their laws, Sec. 4.1): Philox-4x32
+ * with philox_rounds rounds, key = seed, counter = (draw index, stream << 28 |
+ * tensor_id, step), one sub-stream each for Mask, Perturb, per-element and
+ * per-tensor Scale. draw_bits = 32 (default): the keep test is on a 32-bit
+ * uniform (a high byte per element from the Mask stream, its low 24 bits only
+ * when the byte ties the threshold's), Perturb and per-element Scale on
+ * 24-bit fields packed three words per four elements. draw_bits = 16 (the
+ * 16-bit draw option): every per-element draw is one 16-bit half word, eight
+ * elements per Philox block; keep iff draw < floor(p_keep 2^16), and a noise
+ * draw u maps to (2u + 1 - 2^16) 2^-16 before the law's transform. Fewer
+ * Philox words per element and no tie path, for a coarser keep threshold and
+ * noise grid; a different stream, so results differ from draw_bits = 32. The
+ * per-tensor Scale draw and the merge (DARE) masks are the same in both. */
 typedef struct {
   uint64_t seed;         /* Philox key */
   float alpha_min;       /* Scale: alpha ~ U[alpha_min, alpha_max); paper: alpha_max = 1 */
@@ -122,6 +135,7 @@ typedef struct {
   int32_t noise;         /* smat_noise */
   int32_t philox_rounds; /* 10 (default) or 7 */
   int32_t flags;         /* SMAT_FLAG_*; 0 = defaults */
+  int32_t draw_bits;     /* 32 (default; 0 reads as 32) or 16: the 16-bit draw option (below) */
 } smat_config;
 
 /* Bytes of device workspace smat_init needs for this tensor list (0 on

@@ -19,6 +19,11 @@ SOURCES = ["smat_fused_bf16.cu", "smat_fused_f32.cu", "smat_sim_bf16.cu", "smat_
            "smat_inplace_bf16.cu", "smat_inplace_f32.cu", "smat_inplace_sim_bf16.cu", "smat_inplace_sim_f32.cu",
            "smat_laplace_bf16.cu", "smat_laplace_f32.cu", "smat_merge.cu", "smat_gradmap.cu", "smat_aux.cu", "smat_noalloc.cu",
            "smat_host.cpp"]
+# The forward and gradient-map units are compiled a second time with
+# SMAT_DRAW16 defined: the launchers of the 16-bit draw option (suffix _d16).
+DRAW16_SOURCES = ["smat_fused_bf16.cu", "smat_fused_f32.cu", "smat_sim_bf16.cu", "smat_sim_f32.cu",
+                  "smat_inplace_bf16.cu", "smat_inplace_f32.cu", "smat_inplace_sim_bf16.cu",
+                  "smat_inplace_sim_f32.cu", "smat_laplace_bf16.cu", "smat_laplace_f32.cu", "smat_gradmap.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-fmad=false", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "--expt-relaxed-constexpr", "-I", INCLUDE, "-I", CSRC]
@@ -48,19 +53,24 @@ def build(force: bool = False, verbose_ptxas: bool = False) -> str:
     os.makedirs(BUILD, exist_ok=True)
     cc = nvcc()
 
-    def compile_one(src):
-        obj = os.path.join(BUILD, os.path.splitext(src)[0] + ".o")
+    def compile_one(job):
+        src, d16 = job
+        obj = os.path.join(BUILD, os.path.splitext(src)[0] + ("_d16" if d16 else "") + ".o")
         cmd = [cc] + ARCH + FLAGS + (["-Xptxas", "-v"] if verbose_ptxas and src.endswith(".cu") else [])
+        if d16:
+            cmd += ["-DSMAT_DRAW16"]
         if src.endswith(".cpp"):
             cmd += ["-x", "cu"]
         cmd += ["-c", os.path.join(CSRC, src), "-o", obj]
         p = subprocess.run(cmd, capture_output=True, text=True)
         if p.returncode != 0:
-            raise RuntimeError("nvcc failed on %s:\n%s" % (src, p.stderr))
+            raise RuntimeError("nvcc failed on %s%s:\n%s" % (src, " (SMAT_DRAW16)" if d16 else "", p.stderr))
         return obj, p.stderr
 
-    with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
-        results = list(ex.map(compile_one, SOURCES))
+    # the slowest units first, so the pool ends together
+    jobs = [(s, True) for s in DRAW16_SOURCES] + [(s, False) for s in SOURCES]
+    with cf.ThreadPoolExecutor(max_workers=min(len(jobs), os.cpu_count() or 8)) as ex:
+        results = list(ex.map(compile_one, jobs))
     if verbose_ptxas:
         for _, err in results:
             sys.stderr.write(err)

@@ -130,34 +130,51 @@ __global__ void debug_noise_unit_kernel(const uint32_t* words, int64_t n, int no
 
 }  // namespace
 
+// The launcher family (packed draws, or _d16 for the 16-bit draw option) of
+// a launch is chosen here from the variant code `rounds`.
+#define SMAT_BY_FAMILY(call) ((rounds & kDraw16) ? call##_d16 : call)
+
 cudaError_t launch_simulate(const KArgs& a, int grid, int dtype, int noise, bool per_elem_alpha,
                             int rounds, bool inplace, cudaStream_t s) {
   if (noise == NOISE_LAPLACE)  // built for 10 rounds (the host refuses 7 with Laplace)
-    return dtype == DT_BF16 ? launch_laplace_bf16(a, grid, false, per_elem_alpha, inplace, s)
-                            : launch_laplace_f32(a, grid, false, per_elem_alpha, inplace, s);
+    return dtype == DT_BF16 ? SMAT_BY_FAMILY(launch_laplace_bf16)(a, grid, false, per_elem_alpha, inplace, s)
+                            : SMAT_BY_FAMILY(launch_laplace_f32)(a, grid, false, per_elem_alpha, inplace, s);
   if (inplace)
-    return dtype == DT_BF16 ? launch_simulate_inplace_bf16(a, grid, noise, per_elem_alpha, rounds, s)
-                            : launch_simulate_inplace_f32(a, grid, noise, per_elem_alpha, rounds, s);
-  return dtype == DT_BF16 ? launch_simulate_bf16(a, grid, noise, per_elem_alpha, rounds, s)
-                          : launch_simulate_f32(a, grid, noise, per_elem_alpha, rounds, s);
+    return dtype == DT_BF16 ? SMAT_BY_FAMILY(launch_simulate_inplace_bf16)(a, grid, noise, per_elem_alpha, rounds, s)
+                            : SMAT_BY_FAMILY(launch_simulate_inplace_f32)(a, grid, noise, per_elem_alpha, rounds, s);
+  return dtype == DT_BF16 ? SMAT_BY_FAMILY(launch_simulate_bf16)(a, grid, noise, per_elem_alpha, rounds, s)
+                          : SMAT_BY_FAMILY(launch_simulate_f32)(a, grid, noise, per_elem_alpha, rounds, s);
 }
 
 cudaError_t launch_stats_simulate(const KArgs& a, int grid, int dtype, int noise, bool per_elem_alpha,
                                   int rounds, bool inplace, bool wide, cudaStream_t s) {
   if (noise == NOISE_LAPLACE)
-    return dtype == DT_BF16 ? launch_laplace_bf16(a, grid, true, per_elem_alpha, inplace, s)
-                            : launch_laplace_f32(a, grid, true, per_elem_alpha, inplace, s);
+    return dtype == DT_BF16 ? SMAT_BY_FAMILY(launch_laplace_bf16)(a, grid, true, per_elem_alpha, inplace, s)
+                            : SMAT_BY_FAMILY(launch_laplace_f32)(a, grid, true, per_elem_alpha, inplace, s);
   if (inplace)
-    return dtype == DT_BF16 ? launch_stats_simulate_inplace_bf16(a, grid, noise, per_elem_alpha, rounds, s)
-                            : launch_stats_simulate_inplace_f32(a, grid, noise, per_elem_alpha, rounds, s);
-  return dtype == DT_BF16 ? launch_stats_simulate_bf16(a, grid, noise, per_elem_alpha, rounds, wide, s)
-                          : launch_stats_simulate_f32(a, grid, noise, per_elem_alpha, rounds, s);
+    return dtype == DT_BF16
+               ? SMAT_BY_FAMILY(launch_stats_simulate_inplace_bf16)(a, grid, noise, per_elem_alpha, rounds, s)
+               : SMAT_BY_FAMILY(launch_stats_simulate_inplace_f32)(a, grid, noise, per_elem_alpha, rounds, s);
+  return dtype == DT_BF16 ? SMAT_BY_FAMILY(launch_stats_simulate_bf16)(a, grid, noise, per_elem_alpha, rounds, wide, s)
+                          : SMAT_BY_FAMILY(launch_stats_simulate_f32)(a, grid, noise, per_elem_alpha, rounds, s);
 }
 
 int streaming_ctas_per_sm(int dtype, int noise, bool pe, int rounds) {
-  return dtype == DT_BF16 ? simulate_ctas_per_sm_bf16(noise, pe, rounds)
-                          : simulate_ctas_per_sm_f32(noise, pe, rounds);
+  return dtype == DT_BF16 ? SMAT_BY_FAMILY(simulate_ctas_per_sm_bf16)(noise, pe, rounds)
+                          : SMAT_BY_FAMILY(simulate_ctas_per_sm_f32)(noise, pe, rounds);
 }
+
+int fused_wide_occ(int noise, int rounds) { return SMAT_BY_FAMILY(fused_wide_ctas_per_sm)(noise, rounds); }
+
+cudaError_t launch_grad_map(const KArgs& a, int grid, int gdtype, bool per_elem_alpha, bool accumulate, int rounds,
+                            cudaStream_t s) {
+  return SMAT_BY_FAMILY(launch_gradmap)(a, grid, gdtype, per_elem_alpha, accumulate, rounds, s);
+}
+
+int grad_map_occ(int gdtype, bool per_elem_alpha, bool accumulate, int rounds) {
+  return SMAT_BY_FAMILY(gradmap_ctas_per_sm)(gdtype, per_elem_alpha, accumulate, rounds);
+}
+#undef SMAT_BY_FAMILY
 
 cudaError_t launch_delta_stats(const KArgs& a, int grid, int dtype, cudaStream_t s) {
   if (a.chunk_end <= a.chunk_begin) return cudaSuccess;
@@ -170,7 +187,7 @@ cudaError_t launch_delta_stats(const KArgs& a, int grid, int dtype, cudaStream_t
 
 cudaError_t launch_scalars(const KArgs& a, int noise, int rounds, cudaStream_t s) {
   if (a.n_tensors <= 0) return cudaSuccess;
-  if (rounds == 7) {
+  if ((rounds & 0xFF) == 7) {  // the per-tensor Scale draw is the same in both draw families
     if (noise == NOISE_GAUSSIAN) scalars_kernel<7, NOISE_GAUSSIAN><<<a.n_tensors, 32, 0, s>>>(a);
     else if (noise == NOISE_LAPLACE) scalars_kernel<7, NOISE_LAPLACE><<<a.n_tensors, 32, 0, s>>>(a);
     else scalars_kernel<7, NOISE_UNIFORM><<<a.n_tensors, 32, 0, s>>>(a);
@@ -187,10 +204,12 @@ cudaError_t launch_mask_bits(const KArgs& a, int64_t numel, int rounds, cudaStre
   if (nwords <= 0) return cudaSuccess;
   int64_t blocks = (nwords + kBlock - 1) / kBlock;
   if (blocks > 65535) blocks = 65535;
-  if (rounds == 7)
-    mask_bits_kernel<7><<<(int)blocks, kBlock, 0, s>>>(a, numel);
-  else
-    mask_bits_kernel<10><<<(int)blocks, kBlock, 0, s>>>(a, numel);
+  switch (rounds) {
+    case 7: mask_bits_kernel<7><<<(int)blocks, kBlock, 0, s>>>(a, numel); break;
+    case 7 | kDraw16: mask_bits_kernel<7 | kDraw16><<<(int)blocks, kBlock, 0, s>>>(a, numel); break;
+    case 10 | kDraw16: mask_bits_kernel<10 | kDraw16><<<(int)blocks, kBlock, 0, s>>>(a, numel); break;
+    default: mask_bits_kernel<10><<<(int)blocks, kBlock, 0, s>>>(a, numel); break;
+  }
   return cudaGetLastError();
 }
 

@@ -51,14 +51,26 @@ __device__ __forceinline__ float noise_scale_of(float sigma) {
 constexpr int DT_F32 = 0;
 constexpr int DT_BF16 = 1;
 
-// One Philox-4x32-R block with round keys precomputed from the seed. Each
-// round takes the full 64-bit products of words 0 and 2 with the round
-// multipliers (one wide multiply each).
+// Stream variants. The `int R` template parameter of every kernel and helper
+// that draws from the streams is a stream variant: the Philox rounds in its
+// low byte (10, or 7 for the reduced-round option) and kDraw16 set for the
+// 16-bit draw option, in which every per-element draw (Mask, Perturb,
+// per-element Scale) is one 16-bit half of a Philox word: element gidx takes
+// half gidx & 1 (low half first) of word (gidx & 7) >> 1 of block gidx >> 3,
+// eight elements per block; the keep test is draw < floor(p_keep 2^16), with
+// no low-bits part, and the noise draw u maps to (2u + 1 - 2^16) 2^-16.
+template <int R>
+constexpr bool draws16() { return (R & kDraw16) != 0; }  // kDraw16: smat_internal.h
+
+// One Philox-4x32 block (the variant's rounds) with round keys precomputed
+// from the seed. Each round takes the full 64-bit products of words 0 and 2
+// with the round multipliers (one wide multiply each).
 template <int R>
 __device__ __forceinline__ uint4 philox(uint32_t c0, uint32_t c1, uint32_t c2, uint32_t c3,
                                         const RoundKeys& k) {
+  constexpr int kRounds = R & 0xFF;
 #pragma unroll
-  for (int r = 0; r < R; ++r) {
+  for (int r = 0; r < kRounds; ++r) {
     const uint64_t pA = (uint64_t)c0 * kMulA;
     const uint64_t pB = (uint64_t)c2 * kMulB;
     c0 = (uint32_t)(pB >> 32) ^ c1 ^ k.k0[r];
@@ -202,6 +214,24 @@ __device__ __forceinline__ float2 sym2(uint32_t u0, uint32_t u1) {
   return mul2_rn(m, splat(5.9604644775390625e-08f));
 }
 
+// 16-bit option: (2u + 1 - 2^16) 2^-16 of two 16-bit draws as one conversion
+// and one fused multiply-add, u 2^-15 - (1 - 2^-16): u 2^-15 is exact and so
+// is the sum (a multiple of 2^-16 below 1 in magnitude).
+constexpr float kSym16Scale = 3.0517578125e-05f;     // 2^-15
+constexpr float kSym16Shift = -0.9999847412109375f;  // -(1 - 2^-16)
+__device__ __forceinline__ float2 sym2_16(uint32_t u0, uint32_t u1) {
+  return fma2_rn(make_float2(__uint2float_rn(u0), __uint2float_rn(u1)), splat(kSym16Scale), splat(kSym16Shift));
+}
+__device__ __forceinline__ float sym16(uint32_t u) {
+  return __fmaf_rn(__uint2float_rn(u), kSym16Scale, kSym16Shift);
+}
+// The symmetric uniform of two draws of the variant (sym24 or sym16).
+template <bool D16, bool FMA_FORM>
+__device__ __forceinline__ float2 sym2v(uint32_t u0, uint32_t u1) {
+  if constexpr (D16) return sym2_16(u0, u1);
+  else return sym2<FMA_FORM>(u0, u1);
+}
+
 // The four 24-bit noise fields of a quad from its three noise words A, B, C:
 // the top 24 bits of each word, and the three low bytes combined.
 __device__ __forceinline__ void quad_fields(uint32_t A, uint32_t B, uint32_t C, uint32_t (&u)[4]) {
@@ -210,6 +240,17 @@ __device__ __forceinline__ void quad_fields(uint32_t A, uint32_t B, uint32_t C, 
   u[2] = C >> 8;
   // bytes [x, A0, B0, C0] then drop x
   u[3] = __byte_perm(__byte_perm(A, B, 0x0400u), C, 0x4210u) >> 8;
+}
+
+// 16-bit option: the four draws of quad q (elements 4q .. 4q + 3) of a group,
+// from the group's block q / 2 (its elements 8 (q / 2) .. 8 (q / 2) + 7):
+// words 2 (q & 1) and 2 (q & 1) + 1, low half first (`hi` = q & 1).
+__device__ __forceinline__ void halves_of(const uint4& b, int hi, uint32_t (&u)[4]) {
+  const uint32_t w0 = hi ? b.z : b.x, w1 = hi ? b.w : b.y;
+  u[0] = w0 & 0xFFFFu;
+  u[1] = w0 >> 16;
+  u[2] = w1 & 0xFFFFu;
+  u[3] = w1 >> 16;
 }
 
 __device__ __forceinline__ float lg2_approx(float t) {
@@ -269,13 +310,14 @@ __device__ __forceinline__ float2 erfinv_central2(float2 x, float& minL) {
   return mul2_rn(x, p);
 }
 
-// Group-path noise of a pair (see erfinv_central2 for minL).
-template <int NOISE>
+// Group-path noise of a pair (see erfinv_central2 for minL); D16: the two
+// draws are 16-bit.
+template <int NOISE, bool D16 = false>
 __device__ __forceinline__ float2 noise_group2(uint32_t n0, uint32_t n1, float2 scale, float& minL) {
-  if (NOISE == NOISE_UNIFORM) return mul2_rn(scale, sym2<false>(n0, n1));
-  if (NOISE == NOISE_GAUSSIAN) return mul2_rn(scale, erfinv_central2(sym2<true>(n0, n1), minL));
+  if (NOISE == NOISE_UNIFORM) return mul2_rn(scale, sym2v<D16, false>(n0, n1));
+  if (NOISE == NOISE_GAUSSIAN) return mul2_rn(scale, erfinv_central2(sym2v<D16, true>(n0, n1), minL));
   if (NOISE == NOISE_LAPLACE) {
-    const float2 v = sym2<true>(n0, n1);
+    const float2 v = sym2v<D16, true>(n0, n1);
     return mul2_rn(scale, make_float2(laplace_unit(v.x), laplace_unit(v.y)));
   }
   return splat(0.0f);
@@ -286,30 +328,35 @@ __device__ __forceinline__ float2 noise_group2(uint32_t n0, uint32_t n1, float2 
 // scale * erfinv(sym24(u)) with
 // scale = fl(sqrt2 sigma) (inverse-CDF transform: sqrt2 erfinv(v) is
 // N(0, 1) for v uniform on (-1, 1)).
-template <int NOISE>
+template <int NOISE, bool D16 = false>
 __device__ __forceinline__ float2 noise_of2(uint32_t n0, uint32_t n1, float2 scale) {
-  if (NOISE == NOISE_UNIFORM) return mul2_rn(scale, sym2<false>(n0, n1));
-  if (NOISE == NOISE_GAUSSIAN) return mul2_rn(scale, erfinv_poly2(sym2<true>(n0, n1)));
+  if (NOISE == NOISE_UNIFORM) return mul2_rn(scale, sym2v<D16, false>(n0, n1));
+  if (NOISE == NOISE_GAUSSIAN) return mul2_rn(scale, erfinv_poly2(sym2v<D16, true>(n0, n1)));
   if (NOISE == NOISE_LAPLACE) {
-    const float2 v = sym2<true>(n0, n1);
+    const float2 v = sym2v<D16, true>(n0, n1);
     return mul2_rn(scale, make_float2(laplace_unit(v.x), laplace_unit(v.y)));
   }
   return splat(0.0f);
 }
 
-template <int NOISE>
-__device__ __forceinline__ float noise_of(uint32_t u24, float scale) {
-  if (NOISE == NOISE_UNIFORM) return __fmul_rn(scale, sym24(u24));
-  if (NOISE == NOISE_GAUSSIAN) return __fmul_rn(scale, erfinv_poly(sym24(u24)));
-  if (NOISE == NOISE_LAPLACE) return __fmul_rn(scale, laplace_unit(sym24(u24)));
+template <int NOISE, bool D16 = false>
+__device__ __forceinline__ float noise_of(uint32_t u, float scale) {
+  const float v = D16 ? sym16(u) : sym24(u);
+  if (NOISE == NOISE_UNIFORM) return __fmul_rn(scale, v);
+  if (NOISE == NOISE_GAUSSIAN) return __fmul_rn(scale, erfinv_poly(v));
+  if (NOISE == NOISE_LAPLACE) return __fmul_rn(scale, laplace_unit(v));
   return 0.0f;
 }
 
-// The packed 24-bit field of one element (any alignment) in the NOISE or
-// ALPHA_E stream: its quad's three words come from one or two of the group's
-// three blocks.
+// The draw of one element (any alignment) in the NOISE or ALPHA_E stream: its
+// packed 24-bit field, whose quad's three words come from one or two of the
+// group's three blocks; or, with 16-bit draws, its half word.
 template <int R>
 __device__ __forceinline__ uint32_t field1(const KArgs& a, uint32_t stream, uint32_t tid, uint64_t gidx) {
+  if constexpr (draws16<R>()) {
+    const uint32_t w = pick(stream_block<R>(a, stream, tid, gidx >> 3), (unsigned)((gidx & 7) >> 1));
+    return (gidx & 1) ? (w >> 16) : (w & 0xFFFFu);
+  }
   const unsigned k = (unsigned)(gidx & 15), q = k >> 2, r = k & 3;
   const uint64_t j0 = 3 * (gidx >> 4);
   const unsigned s0 = 3 * q;  // first of the quad's words among the group's 12
@@ -369,9 +416,38 @@ __device__ __forceinline__ bool keep_bytes16(const uint4& w, uint32_t t_hi, uint
   }
   return anytie != 0u;
 }
+// 16-bit option: keep flags of the 16 elements gidx0 .. gidx0 + 15 (gidx0 %
+// 16 == 0) from the two MASK blocks gidx0 / 8 and gidx0 / 8 + 1 (half h of
+// word w serves element 2w + h), compared with T16 (< 2^16) two halves at a
+// time (SWAR on 16-bit lanes, no borrow between them); the flags land in the
+// byte layout of keep_bytes16 (bit 8b + 7 of kw[q] for element 4q + b).
+__device__ __forceinline__ void keep_halves16(const uint4& b0, const uint4& b1, uint32_t t16, uint32_t (&kw)[4]) {
+  const uint32_t words[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+  const uint32_t tt = t16 | (t16 << 16);
+  const uint32_t tl = tt & 0x7FFF7FFFu;
+  uint32_t f[8];
+#pragma unroll
+  for (int m = 0; m < 8; ++m) {
+    const uint32_t x = words[m];
+    // bit 15 of each half of d: low 15 bits of x >= low 15 bits of t
+    const uint32_t d = (x | 0x80008000u) - tl;
+    f[m] = ((~x & tt) | (~(x ^ tt) & ~d)) & 0x80008000u;  // x < t per half
+  }
+  // bytes 1 and 3 of words 2q and 2q + 1 carry elements 4q .. 4q + 3
+#pragma unroll
+  for (int q = 0; q < 4; ++q) kw[q] = __byte_perm(f[2 * q], f[2 * q + 1], 0x7531u);
+}
+
+// Keep flags of a group; true if some element's mask byte ties the
+// threshold's (never with 16-bit draws, whose compare is exact).
 template <int R, bool J0>
 __device__ __forceinline__ bool group_keep16(const KArgs& a, uint32_t tid, uint32_t t_hi, uint64_t gidx0,
                                              uint32_t (&kw)[4]) {
+  if constexpr (draws16<R>()) {
+    keep_halves16(stream_block<R, J0>(a, S_MASK, tid, gidx0 >> 3), stream_block<R, J0>(a, S_MASK, tid, (gidx0 >> 3) + 1),
+                  t_hi, kw);
+    return false;
+  }
   return keep_bytes16(stream_block<R, J0>(a, S_MASK, tid, gidx0 >> 4), t_hi, kw);
 }
 
@@ -468,6 +544,10 @@ struct TieList {
 template <int R>
 __device__ __forceinline__ bool elem_kept_at(const RoundKeys& key, uint32_t step, uint32_t tid, uint32_t t_hi,
                                              uint32_t t_lo, uint64_t gidx) {
+  if constexpr (draws16<R>()) {  // t_hi holds T16
+    const uint32_t w = pick(stream_block_at<R>(key, step, S_MASK, tid, gidx >> 3), (unsigned)((gidx & 7) >> 1));
+    return ((gidx & 1) ? (w >> 16) : (w & 0xFFFFu)) < t_hi;
+  }
   const uint4 w = stream_block_at<R>(key, step, S_MASK, tid, gidx >> 4);
   const uint32_t hi = (pick(w, (unsigned)((gidx >> 2) & 3)) >> (8u * (unsigned)(gidx & 3))) & 0xFFu;
   if (hi != t_hi) return hi < t_hi;
@@ -571,6 +651,14 @@ __device__ __forceinline__ float alpha_elem(const KArgs& a, uint32_t u) {
 // Scale per element from its packed 24-bit ALPHA_E field: u 2^-24 is exact.
 __device__ __forceinline__ float alpha_of24(const KArgs& a, uint32_t u24) {
   return __fmaf_rn(a.alpha_width, __fmul_rn(__uint2float_rn(u24), 5.9604644775390625e-08f), a.alpha_min);
+}
+// The same from a 16-bit draw (16-bit option): u 2^-16 is exact.
+__device__ __forceinline__ float alpha_of16(const KArgs& a, uint32_t u16) {
+  return __fmaf_rn(a.alpha_width, __fmul_rn(__uint2float_rn(u16), 1.52587890625e-05f), a.alpha_min);
+}
+template <bool D16>
+__device__ __forceinline__ float alpha_of(const KArgs& a, uint32_t u) {
+  return D16 ? alpha_of16(a, u) : alpha_of24(a, u);
 }
 
 // Per-chunk view of one tensor's constants.

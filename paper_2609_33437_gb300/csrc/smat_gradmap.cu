@@ -14,38 +14,48 @@ template <int R, int GDT, bool PE, bool ACC, bool J0>
 __device__ __forceinline__ void grad_compute16(const KArgs& a, const TView& v, uint64_t g0, uint32_t off,
                                                bool defer, TieList& tl, const Raw16<GDT>& gs,
                                                const Raw16<GDT>& go, float (&out)[16]) {
+  constexpr bool D16 = draws16<R>();
   uint32_t kw[4] = {0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u};
   if (v.flags & TF_MASK) {
-    const uint4 mb = stream_block<R, J0>(a, S_MASK, v.tid, g0 >> 4);
-    const bool tie = keep_bytes16(mb, v.t_hi, kw);
-    if (v.t_lo != 0u && tie) {
-      if (ACC || !defer || !tl.push(off >> 4))
-        resolve_block_ties<R, J0>(a, v.tid, v.t_hi, v.t_lo, mb, g0, kw);
-      else if (tie_mostly_kept(v.t_lo))
-        set_tie_flags(mb, v.t_hi, kw);
+    if constexpr (D16) {
+      group_keep16<R, J0>(a, v.tid, v.t_hi, g0, kw);  // exact 16-bit compare: no ties
+    } else {
+      const uint4 mb = stream_block<R, J0>(a, S_MASK, v.tid, g0 >> 4);
+      const bool tie = keep_bytes16(mb, v.t_hi, kw);
+      if (v.t_lo != 0u && tie) {
+        if (ACC || !defer || !tl.push(off >> 4))
+          resolve_block_ties<R, J0>(a, v.tid, v.t_hi, v.t_lo, mb, g0, kw);
+        else if (tie_mostly_kept(v.t_lo))
+          set_tie_flags(mb, v.t_hi, kw);
+      }
     }
   }
-  // per-element alpha: three ALPHA_E blocks per group, three words per quad
+  // per-element alpha: three ALPHA_E blocks per group, three words per quad;
+  // with 16-bit draws two blocks, one half word per element
   uint4 ab0 = make_uint4(0u, 0u, 0u, 0u), ab1 = ab0, ab2 = ab0;
   if (PE) {
-    const uint64_t jn = 3 * (g0 >> 4);
+    const uint64_t jn = D16 ? (g0 >> 3) : 3 * (g0 >> 4);
     ab0 = stream_block<R, J0>(a, S_ALPHA_E, v.tid, jn);
     ab1 = stream_block<R, J0>(a, S_ALPHA_E, v.tid, jn + 1);
-    ab2 = stream_block<R, J0>(a, S_ALPHA_E, v.tid, jn + 2);
+    if (!D16) ab2 = stream_block<R, J0>(a, S_ALPHA_E, v.tid, jn + 2);
   }
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     uint32_t ua[4] = {0u, 0u, 0u, 0u};
     if (PE) {
-      if (q == 0) quad_fields(ab0.x, ab0.y, ab0.z, ua);
-      if (q == 1) quad_fields(ab0.w, ab1.x, ab1.y, ua);
-      if (q == 2) quad_fields(ab1.z, ab1.w, ab2.x, ua);
-      if (q == 3) quad_fields(ab2.y, ab2.z, ab2.w, ua);
+      if (D16) {
+        halves_of(q < 2 ? ab0 : ab1, q & 1, ua);
+      } else {
+        if (q == 0) quad_fields(ab0.x, ab0.y, ab0.z, ua);
+        if (q == 1) quad_fields(ab0.w, ab1.x, ab1.y, ua);
+        if (q == 2) quad_fields(ab1.z, ab1.w, ab2.x, ua);
+        if (q == 3) quad_fields(ab2.y, ab2.z, ab2.w, ua);
+      }
     }
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
       const int e = 4 * q + k;
-      const float c = PE ? __fmul_rn(alpha_of24(a, ua[k]), v.inv_keep) : v.c;
+      const float c = PE ? __fmul_rn(alpha_of<D16>(a, ua[k]), v.inv_keep) : v.c;
       float g = kept_of(kw, e) ? __fmul_rn(c, gs.at(e)) : 0.0f;
       if (ACC) g = __fadd_rn(go.at(e), g);
       out[e] = g;
@@ -58,7 +68,7 @@ __device__ __forceinline__ void grad_elem_as(const KArgs& a, const TView& v, con
                                              bool kept) {
   const uint64_t g = (uint64_t)(v.off + e);
   float c = v.c;
-  if (PE) c = __fmul_rn(alpha_of24(a, field1<R>(a, S_ALPHA_E, v.tid, g)), v.inv_keep);
+  if (PE) c = __fmul_rn(alpha_of<draws16<R>()>(a, field1<R>(a, S_ALPHA_E, v.tid, g)), v.inv_keep);
   float r = kept ? __fmul_rn(c, load1<GDT>(G.g_sim, e)) : 0.0f;
   if (ACC) r = __fadd_rn(load1<GDT>(G.g_out, e), r);
   store1<GDT>(G.g_out, e, r);
@@ -199,18 +209,19 @@ cudaError_t grad_dt(const KArgs& a, int grid, int gdt, bool pe, bool acc, cudaSt
 
 }  // namespace
 
-cudaError_t launch_gradmap(const KArgs& a, int grid, int gdtype, bool per_elem_alpha, bool accumulate,
-                           int rounds, cudaStream_t s) {
+// This translation unit is compiled once per draw family (smat_internal.h).
+cudaError_t SMAT_FAMILY(launch_gradmap)(const KArgs& a, int grid, int gdtype, bool per_elem_alpha, bool accumulate,
+                                        int rounds, cudaStream_t s) {
   if (a.chunk_end <= a.chunk_begin) return cudaSuccess;
-  return rounds == 7 ? grad_dt<7>(a, grid, gdtype, per_elem_alpha, accumulate, s)
-                     : grad_dt<10>(a, grid, gdtype, per_elem_alpha, accumulate, s);
+  return (rounds & 0xFF) == 7 ? grad_dt<7 | kFamily>(a, grid, gdtype, per_elem_alpha, accumulate, s)
+                              : grad_dt<10 | kFamily>(a, grid, gdtype, per_elem_alpha, accumulate, s);
 }
 
-int gradmap_ctas_per_sm(int gdtype, bool pe, bool acc, int rounds) {
+int SMAT_FAMILY(gradmap_ctas_per_sm)(int gdtype, bool pe, bool acc, int rounds) {
 #define SMAT_GOCC(R, G) (pe ? (acc ? grad_occ<R, G, true, true>() : grad_occ<R, G, true, false>()) \
                            : (acc ? grad_occ<R, G, false, true>() : grad_occ<R, G, false, false>()))
-  if (rounds == 7) return gdtype == DT_BF16 ? SMAT_GOCC(7, DT_BF16) : SMAT_GOCC(7, DT_F32);
-  return gdtype == DT_BF16 ? SMAT_GOCC(10, DT_BF16) : SMAT_GOCC(10, DT_F32);
+  if ((rounds & 0xFF) == 7) return gdtype == DT_BF16 ? SMAT_GOCC(7 | kFamily, DT_BF16) : SMAT_GOCC(7 | kFamily, DT_F32);
+  return gdtype == DT_BF16 ? SMAT_GOCC(10 | kFamily, DT_BF16) : SMAT_GOCC(10 | kFamily, DT_F32);
 #undef SMAT_GOCC
 }
 

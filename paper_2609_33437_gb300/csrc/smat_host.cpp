@@ -90,6 +90,8 @@ smat_status check_config(const smat_config* cfg) {
     return fail(SMAT_ERR_UNSUPPORTED, "Laplace noise is built for 10 Philox rounds");
   if (cfg->philox_rounds != 0 && cfg->philox_rounds != 7 && cfg->philox_rounds != 10)
     return fail(SMAT_ERR_UNSUPPORTED, "philox_rounds %d not supported (7 or 10)", cfg->philox_rounds);
+  if (cfg->draw_bits != 0 && cfg->draw_bits != 16 && cfg->draw_bits != 32)
+    return fail(SMAT_ERR_UNSUPPORTED, "draw_bits %d not supported (32 or 16)", cfg->draw_bits);
   if (cfg->flags & ~(SMAT_FLAG_UNFUSED_STATS | SMAT_FLAG_CHUNK_LOG2_MASK))
     return fail(SMAT_ERR_UNSUPPORTED, "unknown flags 0x%x", cfg->flags);
   const int chunk_log2 = (cfg->flags & SMAT_FLAG_CHUNK_LOG2_MASK) >> 8;
@@ -414,7 +416,8 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
   smat_ctx* c = new smat_ctx();
   c->desc.assign(tensors, tensors + n_tensors);
   c->cfg = *cfg;
-  c->rounds = cfg->philox_rounds == 7 ? 7 : 10;
+  c->rounds = (cfg->philox_rounds == 7 ? 7 : 10) | (cfg->draw_bits == 16 ? kDraw16 : 0);
+  const bool d16 = cfg->draw_bits == 16;
   c->any_sigma_rel = rel;
   c->chunk_elems = cs;
   c->keys = make_keys(cfg->seed);
@@ -447,13 +450,17 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
       T.sigma = d.sigma;
       T.sigma_rel = d.sigma_rel;
       // Eq. smat-mask: keep with probability p_keep = 1 - p, rescale by 1 / p_keep.
-      const uint64_t thr = (uint64_t)std::floor((double)d.keep_prob * 4294967296.0);
+      // The threshold is on a 32-bit draw (its high byte, then on a tie the low
+      // 24 bits), or on a 16-bit draw with the 16-bit option (t_hi holds it;
+      // t_lo = 0, so there are no ties).
+      const int draw = d16 ? 16 : 32;
+      const uint64_t thr = (uint64_t)std::floor((double)d.keep_prob * (double)(uint64_t(1) << draw));
       T.inv_keep = d.keep_prob > 0.0f ? (float)(1.0 / (double)d.keep_prob) : 0.0f;
       uint32_t flags = 0;
-      if (thr < (uint64_t(1) << 32)) {
+      if (thr < (uint64_t(1) << draw)) {
         flags |= TF_MASK;
-        T.t_hi = (uint32_t)(thr >> 24);
-        T.t_lo = (uint32_t)(thr & 0xFFFFFFu);
+        T.t_hi = d16 ? (uint32_t)thr : (uint32_t)(thr >> 24);
+        T.t_lo = d16 ? 0u : (uint32_t)(thr & 0xFFFFFFu);
       }
       // 256-bit vector accesses need 32-byte aligned addresses; groups of 16
       // elements start at multiples of 16 elements from the base pointer.
@@ -497,7 +504,7 @@ smat_status smat_init(smat_ctx** out, const smat_tensor_desc* tensors, int32_t n
     // lead of about one grid width of the bf16 forward (one, two and four
     // measured on the 7B list: one is fastest)
     const int64_t lead = (int64_t)c->sm_count *
-                         (c->wide ? fused_wide_ctas_per_sm(cfg->noise, c->rounds)
+                         (c->wide ? fused_wide_occ(cfg->noise, c->rounds)
                                   : streaming_ctas_per_sm(SMAT_BF16, cfg->noise,
                                                           cfg->alpha_mode == SMAT_ALPHA_PER_ELEMENT, c->rounds));
     for (int dt = 0; dt < 2; ++dt) build_items(c, dt, lead);
@@ -542,7 +549,7 @@ smat_status smat_simulate_multi(smat_ctx* c, uint32_t step, smat_stream_t stream
       int grid = grid_for(c, c->range_end[dt] - c->range_begin[dt], dt);
       if (wide) {
         const int64_t chunks = c->range_end[dt] - c->range_begin[dt];
-        const int64_t resident = (int64_t)c->sm_count * fused_wide_ctas_per_sm(c->cfg.noise, c->rounds);
+        const int64_t resident = (int64_t)c->sm_count * fused_wide_occ(c->cfg.noise, c->rounds);
         grid = (int)(chunks < resident ? chunks : resident);
       }
       Timed t(c, 2, stream);
@@ -623,11 +630,11 @@ smat_status smat_grad_map_multi(smat_ctx* c, uint32_t step, const void* const* g
   a.chunk_begin = 0;
   a.chunk_end = (int64_t)c->h_chunks.size();
   const int64_t resident = (int64_t)c->sm_count *
-                           gradmap_ctas_per_sm(gdtype, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT, accumulate != 0, c->rounds);
+                           grad_map_occ(gdtype, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT, accumulate != 0, c->rounds);
   const int grid = (int)(a.chunk_end < resident ? a.chunk_end : resident);
   if (a.chunk_end <= 0) return SMAT_OK;
   Timed t(c, 3, stream);
-  const cudaError_t e = launch_gradmap(a, grid, gdtype, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT,
+  const cudaError_t e = launch_grad_map(a, grid, gdtype, c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT,
                                        accumulate != 0, c->rounds, stream);
   t.done();
   if (e != cudaSuccess) return cuda_fail(e, "gradient map launch");

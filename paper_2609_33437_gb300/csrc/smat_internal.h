@@ -23,6 +23,11 @@ constexpr uint32_t kGlobalAlphaTensor = 0x0FFFFFFFu;
 // forward work items are whole chunks; the gradient map, whose CTAs take
 // its units in a fixed grid-stride order, walks units of at most
 // kMaxGradUnitElems so its CTAs end closer together.
+// Stream variant code passed as `rounds` to the launchers below (and the `R`
+// template parameter of the kernels): the Philox rounds (10 or 7) in the low
+// byte, kDraw16 set for the 16-bit draw option (see smat_device.cuh).
+constexpr int kDraw16 = 0x100;
+
 constexpr int64_t kMinChunkElems = int64_t(1) << 12;
 constexpr int64_t kMaxChunkElems = int64_t(1) << 18;
 constexpr int64_t kMaxGradUnitElems = int64_t(1) << 17;
@@ -127,40 +132,68 @@ cudaError_t launch_simulate(const KArgs& a, int grid, int dtype, int noise, bool
 // in place, uniform or Gaussian noise: the four-CTA-per-SM build).
 cudaError_t launch_stats_simulate(const KArgs& a, int grid, int dtype, int noise, bool per_elem_alpha,
                                   int rounds, bool inplace, bool wide, cudaStream_t s);
-cudaError_t launch_gradmap(const KArgs& a, int grid, int gdtype, bool per_elem_alpha, bool accumulate,
-                           int rounds, cudaStream_t s);
-cudaError_t launch_simulate_f32(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
-                                cudaStream_t s);
-cudaError_t launch_simulate_bf16(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
-                                 cudaStream_t s);
-int simulate_ctas_per_sm_f32(int noise, bool per_elem_alpha, int rounds);
-int simulate_ctas_per_sm_bf16(int noise, bool per_elem_alpha, int rounds);
-cudaError_t launch_stats_simulate_f32(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
-                                      cudaStream_t s);
-cudaError_t launch_stats_simulate_bf16(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
-                                       bool wide, cudaStream_t s);
-// Resident CTAs per SM of the four-CTA build (bf16, uniform or Gaussian).
-int fused_wide_ctas_per_sm(int noise, int rounds);
-// Laplace noise (10 rounds; smat_laplace_*.cu): the work-list launch when
-// `fused`, else the grid-stride one; in-place instantiations when `inplace`.
-cudaError_t launch_laplace_f32(const KArgs& a, int grid, bool fused, bool per_elem_alpha, bool inplace, cudaStream_t s);
-cudaError_t launch_laplace_bf16(const KArgs& a, int grid, bool fused, bool per_elem_alpha, bool inplace, cudaStream_t s);
-// the same launches for lists with in-place tensors (smat_inplace_*.cu)
-cudaError_t launch_stats_simulate_inplace_f32(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
-                                              cudaStream_t s);
-cudaError_t launch_stats_simulate_inplace_bf16(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
-                                               cudaStream_t s);
-cudaError_t launch_simulate_inplace_f32(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
-                                        cudaStream_t s);
-cudaError_t launch_simulate_inplace_bf16(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
-                                         cudaStream_t s);
+// The forward launchers below exist twice: as declared (the packed draw
+// layout) and with the suffix _d16 (the 16-bit draw option). Each forward
+// translation unit is compiled once per family (SMAT_DRAW16 defined for the
+// second), so the default launches carry none of the option's code;
+// launch_simulate and launch_stats_simulate pick the family from `rounds`.
+#define SMAT_FORWARD_LAUNCHERS(sfx)                                                                           \
+  cudaError_t launch_simulate_f32##sfx(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,   \
+                                       cudaStream_t s);                                                       \
+  cudaError_t launch_simulate_bf16##sfx(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,  \
+                                        cudaStream_t s);                                                      \
+  int simulate_ctas_per_sm_f32##sfx(int noise, bool per_elem_alpha, int rounds);                              \
+  int simulate_ctas_per_sm_bf16##sfx(int noise, bool per_elem_alpha, int rounds);                             \
+  cudaError_t launch_stats_simulate_f32##sfx(const KArgs& a, int grid, int noise, bool per_elem_alpha,        \
+                                             int rounds, cudaStream_t s);                                     \
+  cudaError_t launch_stats_simulate_bf16##sfx(const KArgs& a, int grid, int noise, bool per_elem_alpha,       \
+                                              int rounds, bool wide, cudaStream_t s);                         \
+  /* Resident CTAs per SM of the four-CTA build (bf16, uniform or Gaussian). */                              \
+  int fused_wide_ctas_per_sm##sfx(int noise, int rounds);                                                     \
+  /* Laplace noise (10 rounds; smat_laplace_*.cu): the work-list launch when `fused`, else the grid-stride    \
+     one; in-place instantiations when `inplace`. */                                                          \
+  cudaError_t launch_laplace_f32##sfx(const KArgs& a, int grid, bool fused, bool per_elem_alpha, bool inplace, \
+                                      cudaStream_t s);                                                        \
+  cudaError_t launch_laplace_bf16##sfx(const KArgs& a, int grid, bool fused, bool per_elem_alpha,             \
+                                       bool inplace, cudaStream_t s);                                         \
+  /* the same launches for lists with in-place tensors (smat_inplace_*.cu) */                                \
+  cudaError_t launch_stats_simulate_inplace_f32##sfx(const KArgs& a, int grid, int noise, bool per_elem_alpha, \
+                                                     int rounds, cudaStream_t s);                             \
+  cudaError_t launch_stats_simulate_inplace_bf16##sfx(const KArgs& a, int grid, int noise,                    \
+                                                      bool per_elem_alpha, int rounds, cudaStream_t s);       \
+  cudaError_t launch_simulate_inplace_f32##sfx(const KArgs& a, int grid, int noise, bool per_elem_alpha,      \
+                                               int rounds, cudaStream_t s);                                   \
+  cudaError_t launch_simulate_inplace_bf16##sfx(const KArgs& a, int grid, int noise, bool per_elem_alpha,     \
+                                                int rounds, cudaStream_t s);                                  \
+  cudaError_t launch_gradmap##sfx(const KArgs& a, int grid, int gdtype, bool per_elem_alpha, bool accumulate, \
+                                  int rounds, cudaStream_t s);                                                \
+  int gradmap_ctas_per_sm##sfx(int gdtype, bool per_elem_alpha, bool accumulate, int rounds);
+SMAT_FORWARD_LAUNCHERS()
+SMAT_FORWARD_LAUNCHERS(_d16)
+#undef SMAT_FORWARD_LAUNCHERS
+
+// Family dispatch (smat_aux.cu): the four-CTA build's occupancy and the
+// gradient map for the variant code `rounds`.
+int fused_wide_occ(int noise, int rounds);
+cudaError_t launch_grad_map(const KArgs& a, int grid, int gdtype, bool per_elem_alpha, bool accumulate, int rounds,
+                            cudaStream_t s);
+int grad_map_occ(int gdtype, bool per_elem_alpha, bool accumulate, int rounds);
+
+// In the forward and gradient-map translation units: the family being
+// compiled (see above) and the name of its launchers.
+#ifdef SMAT_DRAW16
+#define SMAT_FAMILY(name) name##_d16
+constexpr int kFamily = kDraw16;
+#else
+#define SMAT_FAMILY(name) name
+constexpr int kFamily = 0;
+#endif
 cudaError_t launch_mask_bits(const KArgs& a, int64_t numel, int rounds, cudaStream_t s);
 cudaError_t launch_debug_philox(const uint32_t* ctr, int64_t n, const RoundKeys& key, int rounds,
                                 uint32_t* out, uint32_t* out_ref, cudaStream_t s);
 cudaError_t launch_debug_noise_unit(const uint32_t* words, int64_t n, int noise, float* out, cudaStream_t s);
 // Resident CTAs per SM of the streaming kernels (for grid sizing).
 int streaming_ctas_per_sm(int dtype, int noise, bool per_elem_alpha, int rounds);
-int gradmap_ctas_per_sm(int gdtype, bool per_elem_alpha, bool accumulate, int rounds);
 
 constexpr int kBlock = 256;
 

@@ -11,14 +11,14 @@ template <bool PE, bool IP>
 cudaError_t laplace_run(const KArgs& a, int grid, bool fused, cudaStream_t s) {
   if (fused) {
     if (a.n_items <= 0) return cudaSuccess;
-    return FusedVariant<10, DT_BF16, NOISE_LAPLACE, PE, IP>::run(a, grid, s);
+    return FusedVariant<10 | kFamily, DT_BF16, NOISE_LAPLACE, PE, IP>::run(a, grid, s);
   }
   if (a.chunk_end <= a.chunk_begin) return cudaSuccess;
-  return SimVariant<10, DT_BF16, NOISE_LAPLACE, PE, IP>::run(a, grid, s);
+  return SimVariant<10 | kFamily, DT_BF16, NOISE_LAPLACE, PE, IP>::run(a, grid, s);
 }
 }  // namespace
 
-cudaError_t launch_laplace_bf16(const KArgs& a, int grid, bool fused, bool per_elem_alpha, bool inplace,
+cudaError_t SMAT_FAMILY(launch_laplace_bf16)(const KArgs& a, int grid, bool fused, bool per_elem_alpha, bool inplace,
                                cudaStream_t s) {
   if (per_elem_alpha)
     return inplace ? laplace_run<true, true>(a, grid, fused, s) : laplace_run<true, false>(a, grid, fused, s);

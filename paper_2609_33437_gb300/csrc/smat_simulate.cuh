@@ -37,35 +37,45 @@ __device__ __forceinline__ uint32_t sim_group16(const KArgs& a, const TView& v, 
   const float2 c2 = splat(v.c);
   const float2 scale2 = splat(v.noise_scale);
   // noise and per-element alpha: three blocks per group each, three words per
-  // quad (see quad_fields)
+  // quad (see quad_fields); with 16-bit draws two blocks each, one half word
+  // per element
+  constexpr bool D16 = draws16<R>();
   uint4 nb0 = make_uint4(0u, 0u, 0u, 0u), nb1 = nb0, nb2 = nb0;
   uint4 ab0 = nb0, ab1 = nb0, ab2 = nb0;
-  const uint64_t jn = 3 * (g0 >> 4);
+  const uint64_t jn = D16 ? (g0 >> 3) : 3 * (g0 >> 4);
   if (NOISE != NOISE_NONE) {
     nb0 = stream_block<R, J0>(a, S_NOISE, v.tid, jn);
     nb1 = stream_block<R, J0>(a, S_NOISE, v.tid, jn + 1);
-    nb2 = stream_block<R, J0>(a, S_NOISE, v.tid, jn + 2);
+    if (!D16) nb2 = stream_block<R, J0>(a, S_NOISE, v.tid, jn + 2);
   }
   if (PE) {
     ab0 = stream_block<R, J0>(a, S_ALPHA_E, v.tid, jn);
     ab1 = stream_block<R, J0>(a, S_ALPHA_E, v.tid, jn + 1);
-    ab2 = stream_block<R, J0>(a, S_ALPHA_E, v.tid, jn + 2);
+    if (!D16) ab2 = stream_block<R, J0>(a, S_ALPHA_E, v.tid, jn + 2);
   }
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     uint32_t u[4] = {0u, 0u, 0u, 0u};
     if (NOISE != NOISE_NONE) {
-      if (q == 0) quad_fields(nb0.x, nb0.y, nb0.z, u);
-      if (q == 1) quad_fields(nb0.w, nb1.x, nb1.y, u);
-      if (q == 2) quad_fields(nb1.z, nb1.w, nb2.x, u);
-      if (q == 3) quad_fields(nb2.y, nb2.z, nb2.w, u);
+      if (D16) {
+        halves_of(q < 2 ? nb0 : nb1, q & 1, u);
+      } else {
+        if (q == 0) quad_fields(nb0.x, nb0.y, nb0.z, u);
+        if (q == 1) quad_fields(nb0.w, nb1.x, nb1.y, u);
+        if (q == 2) quad_fields(nb1.z, nb1.w, nb2.x, u);
+        if (q == 3) quad_fields(nb2.y, nb2.z, nb2.w, u);
+      }
     }
     uint32_t ua[4] = {0u, 0u, 0u, 0u};
     if (PE) {
-      if (q == 0) quad_fields(ab0.x, ab0.y, ab0.z, ua);
-      if (q == 1) quad_fields(ab0.w, ab1.x, ab1.y, ua);
-      if (q == 2) quad_fields(ab1.z, ab1.w, ab2.x, ua);
-      if (q == 3) quad_fields(ab2.y, ab2.z, ab2.w, ua);
+      if (D16) {
+        halves_of(q < 2 ? ab0 : ab1, q & 1, ua);
+      } else {
+        if (q == 0) quad_fields(ab0.x, ab0.y, ab0.z, ua);
+        if (q == 1) quad_fields(ab0.w, ab1.x, ab1.y, ua);
+        if (q == 2) quad_fields(ab1.z, ab1.w, ab2.x, ua);
+        if (q == 3) quad_fields(ab2.y, ab2.z, ab2.w, ua);
+      }
     }
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
@@ -73,8 +83,8 @@ __device__ __forceinline__ uint32_t sim_group16(const KArgs& a, const TView& v, 
       const float2 th2 = th.pair(e0 >> 1), t02 = t0.pair(e0 >> 1);
       float2 kv;
       if (PE) {
-        const float2 cc = make_float2(__fmul_rn(alpha_of24(a, ua[2 * h]), v.inv_keep),
-                                      __fmul_rn(alpha_of24(a, ua[2 * h + 1]), v.inv_keep));
+        const float2 cc = make_float2(__fmul_rn(alpha_of<D16>(a, ua[2 * h]), v.inv_keep),
+                                      __fmul_rn(alpha_of<D16>(a, ua[2 * h + 1]), v.inv_keep));
         const float2 f = fma2_rn(cc, sub2_rn(th2, t02), t02);
         kv = make_float2(cc.x == 1.0f ? th2.x : f.x, cc.y == 1.0f ? th2.y : f.y);
       } else if (IDENT) {
@@ -85,8 +95,8 @@ __device__ __forceinline__ uint32_t sim_group16(const KArgs& a, const TView& v, 
       float x0 = kept_of(kw, e0) ? kv.x : t02.x;
       float x1 = kept_of(kw, e0 + 1) ? kv.y : t02.y;
       if (NOISE != NOISE_NONE) {
-        const float2 eps = EXACT ? noise_of2<NOISE>(u[2 * h], u[2 * h + 1], scale2)
-                                 : noise_group2<NOISE>(u[2 * h], u[2 * h + 1], scale2, minL);
+        const float2 eps = EXACT ? noise_of2<NOISE, D16>(u[2 * h], u[2 * h + 1], scale2)
+                                 : noise_group2<NOISE, D16>(u[2 * h], u[2 * h + 1], scale2, minL);
         x0 = __fadd_rn(x0, eps.x);
         x1 = __fadd_rn(x1, eps.y);
       }
@@ -103,21 +113,26 @@ __device__ __forceinline__ uint32_t sim_group16(const KArgs& a, const TView& v, 
 // L = log2(1 - x^2) < -8), computed exactly as erfinv_central2 computes L.
 template <int R, bool J0>
 __device__ __forceinline__ uint32_t group_tails16(const KArgs& a, uint32_t tid, uint64_t gidx0) {
-  const uint64_t jn = 3 * (gidx0 >> 4);
+  constexpr bool D16 = draws16<R>();
+  const uint64_t jn = D16 ? (gidx0 >> 3) : 3 * (gidx0 >> 4);
   const uint4 b0 = stream_block<R, J0>(a, S_NOISE, tid, jn);
   const uint4 b1 = stream_block<R, J0>(a, S_NOISE, tid, jn + 1);
-  const uint4 b2 = stream_block<R, J0>(a, S_NOISE, tid, jn + 2);
+  const uint4 b2 = D16 ? b1 : stream_block<R, J0>(a, S_NOISE, tid, jn + 2);
   uint32_t bits = 0u;
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     uint32_t u[4];
-    if (q == 0) quad_fields(b0.x, b0.y, b0.z, u);
-    if (q == 1) quad_fields(b0.w, b1.x, b1.y, u);
-    if (q == 2) quad_fields(b1.z, b1.w, b2.x, u);
-    if (q == 3) quad_fields(b2.y, b2.z, b2.w, u);
+    if (D16) {
+      halves_of(q < 2 ? b0 : b1, q & 1, u);
+    } else {
+      if (q == 0) quad_fields(b0.x, b0.y, b0.z, u);
+      if (q == 1) quad_fields(b0.w, b1.x, b1.y, u);
+      if (q == 2) quad_fields(b1.z, b1.w, b2.x, u);
+      if (q == 3) quad_fields(b2.y, b2.z, b2.w, u);
+    }
 #pragma unroll
     for (int r = 0; r < 4; ++r) {
-      const float x = sym24(u[r]);
+      const float x = D16 ? sym16(u[r]) : sym24(u[r]);
       if (lg2_approx(__fmaf_rn(-x, x, 1.0f)) < -8.0f) bits |= 1u << (4 * q + r);
     }
   }
@@ -128,13 +143,14 @@ __device__ __forceinline__ uint32_t group_tails16(const KArgs& a, uint32_t tid, 
 template <int R, int DT, int NOISE, bool PE>
 __device__ __forceinline__ void sim_elem_as(const KArgs& a, const TView& v, const void* th_p,
                                             const void* t0_p, void* sim_p, int64_t e, bool kept) {
+  constexpr bool D16 = draws16<R>();
   const uint64_t g = (uint64_t)(v.off + e);
   float c = v.c;
-  if (PE) c = __fmul_rn(alpha_of24(a, field1<R>(a, S_ALPHA_E, v.tid, g)), v.inv_keep);
+  if (PE) c = __fmul_rn(alpha_of<D16>(a, field1<R>(a, S_ALPHA_E, v.tid, g)), v.inv_keep);
   const float x_th = load1<DT>(th_p, e), x_t0 = load1<DT>(t0_p, e);
   float x = x_t0;
   if (kept) x = (c == 1.0f) ? x_th : __fmaf_rn(c, __fsub_rn(x_th, x_t0), x_t0);
-  if (NOISE != NOISE_NONE) x = __fadd_rn(x, noise_of<NOISE>(field1<R>(a, S_NOISE, v.tid, g), v.noise_scale));
+  if (NOISE != NOISE_NONE) x = __fadd_rn(x, noise_of<NOISE, D16>(field1<R>(a, S_NOISE, v.tid, g), v.noise_scale));
   store1<DT>(sim_p, e, x);
 }
 

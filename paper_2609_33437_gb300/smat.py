@@ -47,7 +47,7 @@ class TensorDesc(ctypes.Structure):
 class Config(ctypes.Structure):
     _fields_ = [("seed", ctypes.c_uint64), ("alpha_min", ctypes.c_float), ("alpha_max", ctypes.c_float),
                 ("alpha_mode", ctypes.c_int32), ("noise", ctypes.c_int32), ("philox_rounds", ctypes.c_int32),
-                ("flags", ctypes.c_int32)]
+                ("flags", ctypes.c_int32), ("draw_bits", ctypes.c_int32)]
 
 
 SMAT_FLAG_UNFUSED_STATS = 1
@@ -139,8 +139,9 @@ class SmatSession:
     thetas / theta0s / sims: lists of contiguous CUDA tensors (theta read,
     theta0 read, sim = theta~ written), same dtype and numel per position.
     keep_probs, sigmas, sigma_rels: per-tensor p_keep (Eq. smat-mask, 1 - p),
-    Perturb RMS, relative Perturb RMS. The workspace is allocated here with
-    torch and handed to the library.
+    Perturb RMS, relative Perturb RMS. draw_bits: 32 (the default draw
+    layout) or 16 (the 16-bit draw option, include/smat.h). The workspace is
+    allocated here with torch and handed to the library.
     """
 
     def __init__(self, thetas: Sequence[torch.Tensor], theta0s: Sequence[torch.Tensor],
@@ -149,7 +150,7 @@ class SmatSession:
                  elem_offsets: Optional[Sequence[int]] = None, seed: int = 0, alpha_min: float = 0.0,
                  alpha_max: float = 1.0, alpha_mode: int = SMAT_ALPHA_GLOBAL,
                  noise: int = SMAT_NOISE_UNIFORM, philox_rounds: int = 10, flags: int = 0,
-                 stream: Optional[torch.cuda.Stream] = None):
+                 stream: Optional[torch.cuda.Stream] = None, draw_bits: int = 32):
         self._L = load_library()
         n = len(thetas)
         if not (len(theta0s) == n and len(sims) == n and len(keep_probs) == n and len(sigmas) == n):
@@ -180,7 +181,7 @@ class SmatSession:
             self.numels.append(th.numel())
         self._descs = descs
         self.config = Config(int(seed) & (2**64 - 1), float(alpha_min), float(alpha_max), int(alpha_mode),
-                             int(noise), int(philox_rounds), int(flags))
+                             int(noise), int(philox_rounds), int(flags), int(draw_bits))
         self.device = thetas[0].device if n else torch.device("cuda", torch.cuda.current_device())
         nbytes = self._L.smat_workspace_bytes(ctypes.byref(descs), n, ctypes.byref(self.config))
         if nbytes == 0 and n > 0:

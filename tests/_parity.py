@@ -38,9 +38,9 @@ def f32_of(bits: np.ndarray) -> np.ndarray:
     return bits.astype(np.float32)
 
 
-def orc_config(w: W.Workload, step: int, rounds: int = 10):
+def orc_config(w: W.Workload, step: int, rounds: int = 10, draw_bits: int = 32):
     return O.config(seed=w.seed, step=step, rounds=rounds, alpha_mode=w.alpha_mode, noise=w.noise,
-                    alpha_min=w.alpha_min, alpha_max=w.alpha_max)
+                    alpha_min=w.alpha_min, alpha_max=w.alpha_max, draw_bits=draw_bits)
 
 
 def orc_tensor(w: W.Workload, k: int, numel=None, elem_offset=0):
@@ -49,11 +49,12 @@ def orc_tensor(w: W.Workload, k: int, numel=None, elem_offset=0):
                     sigma_rel=t.sigma_rel, elem_offset=elem_offset)
 
 
-def session_for(w: W.Workload, th, t0, sim, rounds: int = 10, elem_offsets=None, flags: int = 0):
+def session_for(w: W.Workload, th, t0, sim, rounds: int = 10, elem_offsets=None, flags: int = 0,
+                draw_bits: int = 32):
     return S.SmatSession(th, t0, sim, [t.keep_prob for t in w.tensors], [t.sigma for t in w.tensors],
                          [t.sigma_rel for t in w.tensors], elem_offsets=elem_offsets, seed=w.seed,
                          alpha_min=w.alpha_min, alpha_max=w.alpha_max, alpha_mode=w.alpha_mode, noise=w.noise,
-                         philox_rounds=rounds, flags=flags)
+                         philox_rounds=rounds, flags=flags, draw_bits=draw_bits)
 
 
 def _ordered_bf16(b: np.ndarray) -> np.ndarray:
@@ -121,7 +122,8 @@ def compare(got_bits, ref_bits, dtype, noise, th=None, t0=None, what=""):
     assert not bad.any(), f"{what}: {int(bad.sum())} elements beyond 1e-6 relative (max ratio {float((err / scale).max())})"
 
 
-def run_and_check_full(w: W.Workload, steps=(0, 1, 2), rounds=10, accumulate=False, gdtype=None, flags=0):
+def run_and_check_full(w: W.Workload, steps=(0, 1, 2), rounds=10, accumulate=False, gdtype=None, flags=0,
+                       draw_bits=32):
     """Generate w on the GPU, run simulate + gradient map for each step through
     the C ABI and compare every element with the oracle."""
     dev = torch.device("cuda")
@@ -130,7 +132,7 @@ def run_and_check_full(w: W.Workload, steps=(0, 1, 2), rounds=10, accumulate=Fal
         gs = [g.to(W.torch_dtype(gdtype)) for g in gs]
         go = [torch.empty_like(g) for g in gs]
     gdt = w.gdtype if gdtype is None else gdtype
-    sess = session_for(w, th, t0, sim, rounds=rounds, flags=flags)
+    sess = session_for(w, th, t0, sim, rounds=rounds, flags=flags, draw_bits=draw_bits)
     hth = [to_host(x) for x in th]
     ht0 = [to_host(x) for x in t0]
     hgs = [to_host(x) for x in gs]
@@ -145,7 +147,7 @@ def run_and_check_full(w: W.Workload, steps=(0, 1, 2), rounds=10, accumulate=Fal
         sess.swap()
         scal = sess.tensor_scalars(step).cpu().numpy()
         torch.cuda.synchronize()
-        cfg = orc_config(w, step, rounds)
+        cfg = orc_config(w, step, rounds, draw_bits)
         for k in range(len(w.tensors)):
             t = orc_tensor(w, k)
             ref = O.simulate(cfg, t, hth[k], ht0[k])

@@ -138,7 +138,7 @@ def test_init_rejects_invalid_tensor(L, bad, code):
     (dict(noise=S.SMAT_NOISE_LAPLACE, philox_rounds=7), 2),
     (dict(alpha_min=0.9, alpha_max=0.5), 1), (dict(alpha_min=float("nan")), 1),
     (dict(flags=S.SMAT_FLAG_CHUNK_LOG2(11)), 2), (dict(flags=S.SMAT_FLAG_CHUNK_LOG2(19)), 2), (dict(flags=1 << 14), 2),
-    (dict(flags=2), 2),
+    (dict(flags=2), 2), (dict(draw_bits=8), 2), (dict(draw_bits=24), 2),
 ])
 def test_init_rejects_invalid_config(L, bad, code):
     ctx = ctypes.c_void_p()
@@ -277,3 +277,15 @@ def test_binding_matches_header_layout(tmp_path):
             continue
         n = 0 if params.strip() in ("", "void") else params.count(",") + 1
         assert len(argtypes) == n, name
+
+
+def test_draw_bits_option_sizes_like_the_default(L):
+    """draw_bits 16 (the 16-bit draw option) and 32 are accepted and need the
+    same workspace (the option changes the draws, not the tables); 0 reads as
+    32."""
+    d = [desc()]
+    base = ws_bytes(L, d, cfg())
+    assert base > 0
+    assert ws_bytes(L, d, cfg(draw_bits=16)) == base
+    assert ws_bytes(L, d, cfg(draw_bits=32)) == base
+    assert ws_bytes(L, d, cfg(draw_bits=7)) == 0
