@@ -5,15 +5,16 @@
 
 namespace smat {
 
-cudaError_t SMAT_FAMILY(launch_stats_simulate_bf16)(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
-                                      bool wide, cudaStream_t s) {
+cudaError_t SMAT_FAMILY(launch_stats_simulate_bf16)(const KArgs& a, int grid, int noise, bool per_elem_alpha,
+                                                    int rounds, bool wide, cudaStream_t s) {
   if (a.n_items <= 0) return cudaSuccess;
   return (rounds & 0xFF) == 7 ? fused_run<7 | kFamily, DT_BF16, false>(a, grid, noise, per_elem_alpha, wide, s)
-                     : fused_run<10 | kFamily, DT_BF16, false>(a, grid, noise, per_elem_alpha, wide, s);
+                              : fused_run<10 | kFamily, DT_BF16, false>(a, grid, noise, per_elem_alpha, wide, s);
 }
 
 int SMAT_FAMILY(fused_wide_ctas_per_sm)(int noise, int rounds) {
-  return (rounds & 0xFF) == 7 ? fused_occ<7 | kFamily, DT_BF16, false>(noise, false, true) : fused_occ<10 | kFamily, DT_BF16, false>(noise, false, true);
+  return (rounds & 0xFF) == 7 ? fused_occ<7 | kFamily, DT_BF16, false>(noise, false, true)
+                              : fused_occ<10 | kFamily, DT_BF16, false>(noise, false, true);
 }
 
 }  // namespace smat

@@ -210,8 +210,8 @@ cudaError_t grad_dt(const KArgs& a, int grid, int gdt, bool pe, bool acc, cudaSt
 }  // namespace
 
 // This translation unit is compiled once per draw family (smat_internal.h).
-cudaError_t SMAT_FAMILY(launch_gradmap)(const KArgs& a, int grid, int gdtype, bool per_elem_alpha, bool accumulate,
-                                        int rounds, cudaStream_t s) {
+cudaError_t SMAT_FAMILY(launch_gradmap)(const KArgs& a, int grid, int gdtype, bool per_elem_alpha,
+                                        bool accumulate, int rounds, cudaStream_t s) {
   if (a.chunk_end <= a.chunk_begin) return cudaSuccess;
   return (rounds & 0xFF) == 7 ? grad_dt<7 | kFamily>(a, grid, gdtype, per_elem_alpha, accumulate, s)
                               : grad_dt<10 | kFamily>(a, grid, gdtype, per_elem_alpha, accumulate, s);

@@ -7,11 +7,11 @@
 
 namespace smat {
 
-cudaError_t SMAT_FAMILY(launch_stats_simulate_inplace_f32)(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
-                                              cudaStream_t s) {
+cudaError_t SMAT_FAMILY(launch_stats_simulate_inplace_f32)(const KArgs& a, int grid, int noise,
+                                                           bool per_elem_alpha, int rounds, cudaStream_t s) {
   if (a.n_items <= 0) return cudaSuccess;
   return (rounds & 0xFF) == 7 ? fused_run<7 | kFamily, DT_F32, true>(a, grid, noise, per_elem_alpha, false, s)
-                     : fused_run<10 | kFamily, DT_F32, true>(a, grid, noise, per_elem_alpha, false, s);
+                              : fused_run<10 | kFamily, DT_F32, true>(a, grid, noise, per_elem_alpha, false, s);
 }
 
 }  // namespace smat

@@ -5,11 +5,11 @@
 
 namespace smat {
 
-cudaError_t SMAT_FAMILY(launch_simulate_inplace_bf16)(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
-                                        cudaStream_t s) {
+cudaError_t SMAT_FAMILY(launch_simulate_inplace_bf16)(const KArgs& a, int grid, int noise,
+                                                      bool per_elem_alpha, int rounds, cudaStream_t s) {
   if (a.chunk_end <= a.chunk_begin) return cudaSuccess;
   return (rounds & 0xFF) == 7 ? sim_run<7 | kFamily, DT_BF16, true>(a, grid, noise, per_elem_alpha, s)
-                     : sim_run<10 | kFamily, DT_BF16, true>(a, grid, noise, per_elem_alpha, s);
+                              : sim_run<10 | kFamily, DT_BF16, true>(a, grid, noise, per_elem_alpha, s);
 }
 
 }  // namespace smat

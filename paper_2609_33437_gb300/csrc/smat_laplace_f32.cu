@@ -18,8 +18,8 @@ cudaError_t laplace_run(const KArgs& a, int grid, bool fused, cudaStream_t s) {
 }
 }  // namespace
 
-cudaError_t SMAT_FAMILY(launch_laplace_f32)(const KArgs& a, int grid, bool fused, bool per_elem_alpha, bool inplace,
-                               cudaStream_t s) {
+cudaError_t SMAT_FAMILY(launch_laplace_f32)(const KArgs& a, int grid, bool fused, bool per_elem_alpha,
+                                            bool inplace, cudaStream_t s) {
   if (per_elem_alpha)
     return inplace ? laplace_run<true, true>(a, grid, fused, s) : laplace_run<true, false>(a, grid, fused, s);
   return inplace ? laplace_run<false, true>(a, grid, fused, s) : laplace_run<false, false>(a, grid, fused, s);

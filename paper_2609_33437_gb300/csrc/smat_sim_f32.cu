@@ -3,15 +3,16 @@
 
 namespace smat {
 
-cudaError_t SMAT_FAMILY(launch_simulate_f32)(const KArgs& a, int grid, int noise, bool per_elem_alpha, int rounds,
-                                  cudaStream_t s) {
+cudaError_t SMAT_FAMILY(launch_simulate_f32)(const KArgs& a, int grid, int noise, bool per_elem_alpha,
+                                             int rounds, cudaStream_t s) {
   if (a.chunk_end <= a.chunk_begin) return cudaSuccess;
   return (rounds & 0xFF) == 7 ? sim_run<7 | kFamily, DT_F32, false>(a, grid, noise, per_elem_alpha, s)
-                     : sim_run<10 | kFamily, DT_F32, false>(a, grid, noise, per_elem_alpha, s);
+                              : sim_run<10 | kFamily, DT_F32, false>(a, grid, noise, per_elem_alpha, s);
 }
 
 int SMAT_FAMILY(simulate_ctas_per_sm_f32)(int noise, bool per_elem_alpha, int rounds) {
-  return (rounds & 0xFF) == 7 ? sim_occ<7 | kFamily, DT_F32>(noise, per_elem_alpha) : sim_occ<10 | kFamily, DT_F32>(noise, per_elem_alpha);
+  return (rounds & 0xFF) == 7 ? sim_occ<7 | kFamily, DT_F32>(noise, per_elem_alpha)
+                              : sim_occ<10 | kFamily, DT_F32>(noise, per_elem_alpha);
 }
 
 }  // namespace smat
