@@ -668,11 +668,24 @@ def run_smat(args):
 
     th, t0, sim, gs, go = W.generate(w, device=dev)
     host_t0 = None
-    if args.theta0 == "host":
-        t0 = [x.cpu().pin_memory() for x in t0]
-    elif args.theta0 == "inplace":
-        host_t0 = [x.cpu().pin_memory() for x in t0]
-        sim = t0  # one buffer per tensor: theta0, overwritten by theta~, refilled every step
+    pinned = None
+    if args.theta0 in ("host", "inplace"):
+        # theta0 in pinned host memory: one huge-page mapping registered with
+        # cudaHostRegister (see PinnedHost), one view per tensor
+        pinned = PinnedHost()
+        pad = lambda n: (n + 15) // 16 * 16  # noqa: E731  (32-byte aligned views: the vector path)
+        flat = pinned.empty(sum(pad(x.numel()) for x in t0), t0[0].dtype if t0 else torch.bfloat16)
+        views, off = [], 0
+        for x in t0:
+            v = flat[off:off + x.numel()].view(x.shape)
+            v.copy_(x)
+            views.append(v)
+            off += pad(x.numel())
+        if args.theta0 == "host":
+            t0 = views
+        else:
+            host_t0 = views
+            sim = t0  # one buffer per tensor: theta0, overwritten by theta~, refilled every step
     sess = make_session(th, t0, sim)
 
     def step(s):
@@ -746,6 +759,9 @@ def run_smat(args):
             per_kernel[k]["frac_of_measured_peak"] = per_kernel[k]["gbs"] / peak
     launches = int(sum(v[1] for v in kern.values()))
     del sess
+    if pinned is not None:
+        del t0, host_t0, views, flat
+        pinned.close()
     out = None
     if rank == 0:
         out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
