@@ -396,6 +396,29 @@ class PinnedHost:
         except Exception:
             return None
 
+    def numa_pages(self):
+        """Pages of this process's anonymous mappings per NUMA node (summed
+        N<node>=<pages> fields of /proc/self/numa_maps), or None: host buffers
+        that did not fit on the GPU's node land on another one, behind a
+        slower path."""
+        try:
+            nodes = {}
+            with open("/proc/self/numa_maps") as f:
+                for line in f:
+                    if "anon" not in line:
+                        continue
+                    kb = 4
+                    for tok in line.split():
+                        if tok.startswith("kernelpagesize_kB="):
+                            kb = int(tok.split("=")[1])
+                    for tok in line.split():
+                        if tok.startswith("N") and "=" in tok and tok[1:tok.index("=")].isdigit():
+                            node = tok[1:tok.index("=")]
+                            nodes[node] = nodes.get(node, 0) + int(tok.split("=")[1]) * kb * 1024
+            return {k: v for k, v in sorted(nodes.items())} or None
+        except Exception:
+            return None
+
     def close(self):
         for raw in self._registered:
             torch.cuda.cudart().cudaHostUnregister(raw.data_ptr())
@@ -636,6 +659,7 @@ def e2e_run(w, sess_factory, steps, warmup, world, groups=8, keep_outputs=False,
         os.sched_setaffinity(0, saved)
     huge = pinned.huge
     huge_frac = pinned.huge_page_fraction() if huge else None
+    numa = pinned.numa_pages()
     pinned.close()
     host_gbs = (h2d + d2h) * steps / el / 1e9
     return {"value": world * bytes_step * steps / el / 1e9, "unit": UNIT, "h2d_bytes_per_step": h2d,
@@ -645,6 +669,7 @@ def e2e_run(w, sess_factory, steps, warmup, world, groups=8, keep_outputs=False,
             "host_numa_node": local[0] if local else None,
             "host_buffers": "huge-page mappings registered with cudaHostRegister" if huge else "torch pinned memory",
             "host_huge_page_fraction": huge_frac,
+            "host_bytes_per_numa_node": numa,
             "host_link_gbs": host_gbs, "link_roof_gbs": roof,
             "frac_of_link_roof": host_gbs / roof["step_copies"] if roof["step_copies"] > 0 else None}
 
