@@ -357,7 +357,7 @@ def gpu_local_cpus(device_index: int):
         return None
 
 
-HUGE_PAGE = 512 << 20  # transparent huge page size of the GPU machine's 64 KB-page kernel
+HUGE_PAGE = 512 << 20  # transparent huge page size of an arm64 kernel with 64 KB base pages
 
 
 class PinnedHost:
@@ -446,7 +446,7 @@ def step_copy_roof(h_ins, h_outs, d_ins, d_outs, groups=8, reps=2):
     """The end-to-end step's copies alone, in the pipeline's pattern: the
     arrays cut into `groups` consecutive ranges; for each range every input
     array is copied in on one stream while the output arrays are copied out
-    on another, no kernels (the roof of the end-to-end leg on this box's link
+    on another, no kernels (the roof of the end-to-end leg on this machine's link
     and these host buffers). Returns GB/s of host traffic."""
     s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
     nbytes = sum(h.numel() * h.element_size() for h in h_ins + h_outs)
@@ -470,7 +470,7 @@ def step_copy_roof(h_ins, h_outs, d_ins, d_outs, groups=8, reps=2):
 
 
 def link_roof(h_in, h_out, nbytes=4 << 30, reps=3, max_streams=4):
-    """Host-link copy roof on this box: pinned-host-to-device and
+    """Host-link copy roof on this machine: pinned-host-to-device and
     device-to-pinned-host cudaMemcpyAsync (torch copy_, non_blocking) of
     `nbytes` in each direction, split over 1, 2 or 4 streams at once (several
     copy engines), alone and both directions together; best of `reps` for each,
