@@ -28,21 +28,21 @@ def _popcount(words: torch.Tensor) -> int:
     return int(c.sum())
 
 
-def _check_workload(w: W.Workload, step: int = 0):
+def _check_workload(w: W.Workload, step: int = 0, draw_bits: int = 32):
     dev = torch.device("cuda")
     free, total = torch.cuda.mem_get_info()
     need = (2 if w.dtype == O.BF16 else 4) * w.numel * 3 + (2 if w.gdtype == O.BF16 else 4) * w.numel * 2
     if need > free * 0.9:
         pytest.skip(f"needs {need / 1e9:.1f} GB of device memory, {free / 1e9:.1f} GB free")
     th, t0, sim, gs, go = W.generate(w, device=dev)
-    sess = session_for(w, th, t0, sim)
+    sess = session_for(w, th, t0, sim, draw_bits=draw_bits)
     sess.simulate_multi(step)
     sess.swap()
     sess.grad_map_multi(step, gs, go)
     sess.swap()
     scal = sess.tensor_scalars(step).cpu().numpy()
     torch.cuda.synchronize()
-    cfg = orc_config(w, step)
+    cfg = orc_config(w, step, draw_bits=draw_bits)
     rng = np.random.default_rng(77)
     for k, spec in enumerate(w.tensors):
         n = spec.numel
@@ -68,6 +68,8 @@ def _check_workload(w: W.Workload, step: int = 0):
         gbits = (wh[idx >> 5] >> (idx & 31).astype(np.uint32)) & 1
         assert np.array_equal(gbits.astype(np.uint8), kept), f"tensor {k} mask bits"
         p = float(np.float32(spec.keep_prob))
+        if draw_bits == 16:
+            p = math.floor(p * 65536) / 65536  # the 16-bit threshold
         if 0.0 < p < 1.0:
             kcount = _popcount(words)
             assert abs(kcount - n * p) <= 5 * math.sqrt(n * p * (1 - p)) + 1, f"tensor {k} keep rate"
@@ -90,3 +92,12 @@ def test_flat_2_32_plus_ragged_bf16_sampled():
     w = W.flat_sweep(32, O.BF16, 0.3, 2, 1e-4)
     w.tensors[0].shape = ((1 << 32) + 17,)
     _check_workload(w, step=1)
+
+
+def test_full_size_7b_list_draw16_sampled():
+    """The 7B list with the 16-bit draw option, in the launch configuration
+    `bench.py --draw-bits 16` times (the four-CTA work-list build with the
+    statistics items), sampled against the oracle with the same option."""
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    _check_workload(W.llama_7b(), step=3, draw_bits=16)
