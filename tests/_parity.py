@@ -88,7 +88,10 @@ def compare(got_bits, ref_bits, dtype, noise, th=None, t0=None, what=""):
     r = f32_of(ref_bits) if dtype == O.BF16 else ref_bits.view(np.float32)
     nan_g, nan_r = np.isnan(g), np.isnan(r)
     assert np.array_equal(nan_g, nan_r), f"{what}: NaN pattern differs"
-    ok = ~nan_r
+    # an infinity on either side must be the same infinity on both
+    inf = np.isinf(g) | np.isinf(r)
+    assert np.array_equal(g[inf], r[inf]), f"{what}: {int((g[inf] != r[inf]).sum())} infinities differ"
+    ok = ~nan_r & ~inf
     if noise == O.NOISE_UNIFORM:
         bad = np.nonzero(got_bits[ok] != ref_bits[ok])[0]
         assert bad.size == 0, f"{what}: {bad.size} elements differ (exact expected); first {np.nonzero(ok)[0][bad[:5]]}"

@@ -347,3 +347,74 @@ def test_parameter_switching_toy_mlp_step():
         sim_ref = O.simulate(cfg, t, to_host(theta_before[k]).ravel(), to_host(theta0[k]).ravel())
         assert np.array_equal(to_host(sp.sims[k]).ravel().view(np.uint32), sim_ref.view(np.uint32))
     torch.optim.SGD(params, lr=0.1).step()
+
+
+def _sprinkle(x: np.ndarray, rng, dtype, frac=0.01):
+    """Signed zeros, infinities, NaN, subnormals and the largest finite values
+    written over a fraction of the elements (as storage bits)."""
+    n = x.size
+    idx = rng.choice(n, size=max(8, int(frac * n)), replace=False)
+    if dtype == O.BF16:
+        specials = np.array([0x0000, 0x8000, 0x7F80, 0xFF80, 0x7FC0, 0x0001, 0x8003, 0x7F7F, 0xFF7F], np.uint16)
+        xv = x.view(np.uint16)
+    else:
+        specials = np.array([0x00000000, 0x80000000, 0x7F800000, 0xFF800000, 0x7FC00000, 0x00000001, 0x80000005,
+                             0x7F7FFFFF, 0xFF7FFFFF], np.uint32)
+        xv = x.view(np.uint32)
+    xv[idx] = specials[rng.integers(0, len(specials), size=len(idx))]
+    return x
+
+
+@pytest.mark.parametrize("alpha_mode", [O.ALPHA_PER_TENSOR, O.ALPHA_PER_ELEMENT])
+@pytest.mark.parametrize("noise", [O.NOISE_UNIFORM, O.NOISE_GAUSSIAN])
+@pytest.mark.parametrize("dtype", [O.BF16, O.F32])
+def test_special_values_in_theta_theta0_and_gradients(dtype, noise, alpha_mode):
+    """Signed zeros, infinities, NaN, subnormals and the largest finite values
+    in theta, theta0 and g~ (vector and element paths): the forward follows
+    the same IEEE operations as the oracle (NaN wherever the oracle's is NaN;
+    otherwise the usual tolerances) and the gradient map equals the oracle's
+    with any NaN equal to any NaN (dropped coordinates are +0 whatever g~)."""
+    rng = np.random.default_rng(1000 + 10 * dtype + noise + 100 * alpha_mode)
+    dev = torch.device("cuda")
+    sizes = [70_001, 4099]
+    tdt = torch.bfloat16 if dtype == O.BF16 else torch.float32
+    hs = []
+    for n in sizes:
+        t0 = (rng.standard_normal(n) * 0.02).astype(np.float32)
+        th = (t0 + rng.standard_normal(n) * 1e-3).astype(np.float32)
+        g = rng.standard_normal(n).astype(np.float32)
+        if dtype == O.BF16:
+            t0, th, g = O.f32_to_bf16(t0), O.f32_to_bf16(th), O.f32_to_bf16(g)
+        hs.append((_sprinkle(th, rng, dtype), _sprinkle(t0, rng, dtype), _sprinkle(g, rng, dtype)))
+
+    def dev_t(a):
+        t = torch.from_numpy(a.view(np.int16) if dtype == O.BF16 else a).to(dev)
+        return t.view(tdt)
+
+    th = [dev_t(h[0]) for h in hs]
+    t0 = [dev_t(h[1]) for h in hs]
+    gs = [dev_t(h[2]) for h in hs]
+    sim = [torch.empty_like(x) for x in th]
+    go = [torch.empty_like(x) for x in th]
+    keeps, sig = [0.7, 0.3], 2e-3
+    sess = S.SmatSession(th, t0, sim, keeps, [sig, sig], seed=321, alpha_min=0.3, alpha_max=1.0,
+                         alpha_mode=alpha_mode, noise=noise)
+    sess.simulate_multi(2)
+    sess.swap()
+    sess.grad_map_multi(2, gs, go)
+    sess.swap()
+    torch.cuda.synchronize()
+    cfg = O.config(seed=321, step=2, alpha_mode=alpha_mode, noise=noise, alpha_min=0.3, alpha_max=1.0)
+    sv = np.uint16 if dtype == O.BF16 else np.uint32
+    for k, n in enumerate(sizes):
+        t = O.tensor(k, n, dtype=dtype, keep_prob=keeps[k], sigma=sig)
+        ref = O.simulate(cfg, t, hs[k][0], hs[k][1])
+        compare(to_host(sim[k]), ref.view(sv), dtype, noise, f32_of(hs[k][0]), f32_of(hs[k][1]),
+                what=f"special values tensor {k}")
+        gref = f32_of(O.gradmap(cfg, t, hs[k][2], gdtype=dtype))
+        gg = f32_of(to_host(go[k]))
+        assert np.array_equal(np.isnan(gg), np.isnan(gref)), f"tensor {k}: gradient NaN pattern"
+        ok = ~np.isnan(gref)
+        assert np.array_equal(gg[ok].view(np.uint32), gref[ok].view(np.uint32)), f"tensor {k}: gradient bits"
+    assert sess.poll_errors() == 0
+    sess.close()
