@@ -18,8 +18,9 @@
 // order. Each thread owns 16 consecutive elements at a time (one 256-bit load
 // per bf16 input, two per fp32 input), which is exactly one Philox block of
 // the mask stream (16 high bytes) and three blocks of the noise stream (24
-// bits per element). The random words stay in registers; masks and noise are
-// never written to memory.
+// bits per element); with the 16-bit draw option, two blocks of each. The
+// random words stay in registers; masks and noise are never written to
+// memory.
 //
 // The path is elementwise and bound by HBM bandwidth or by the integer
 // pipeline (Philox): there is no contraction, so no tensor-core work.

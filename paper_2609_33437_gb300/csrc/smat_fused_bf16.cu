@@ -1,6 +1,8 @@
 // Rows a2 + a3 (the persistent work-list forward, with the delta statistics of
 // sigma_rel tensors) for bf16 parameters. A translation unit of its own so the
 // forward kernels compile in parallel.
+// Compiled once per draw family (the packed layout, and with SMAT_DRAW16
+// the 16-bit draw option: the _d16 launchers; smat_internal.h).
 #include "smat_simulate.cuh"
 
 namespace smat {

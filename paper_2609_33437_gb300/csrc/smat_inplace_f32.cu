@@ -3,6 +3,8 @@
 // with the in-place path (flagged groups are recomputed whole after the chunk
 // instead of rewritten element by element, since their theta0 is still
 // needed), so the launches of other lists carry none of its code.
+// Compiled once per draw family (the packed layout, and with SMAT_DRAW16
+// the 16-bit draw option: the _d16 launchers; smat_internal.h).
 #include "smat_simulate.cuh"
 
 namespace smat {

@@ -1,6 +1,8 @@
 // Row a3 (grid-stride launch, SMAT_FLAG_UNFUSED_STATS) for bf16 parameters in
 // lists with in-place tensors: the launch of smat_sim_bf16.cu instantiated with
 // the in-place path (see smat_inplace_bf16.cu).
+// Compiled once per draw family (the packed layout, and with SMAT_DRAW16
+// the 16-bit draw option: the _d16 launchers; smat_internal.h).
 #include "smat_simulate.cuh"
 
 namespace smat {

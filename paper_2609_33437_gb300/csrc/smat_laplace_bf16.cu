@@ -2,6 +2,8 @@
 // Perturb (Sec. 4.1, "Perturb": the matched-RMS comparison of uniform,
 // Gaussian and Laplace noise), 10 Philox rounds: the forward launches
 // instantiated with the Laplace transform, in a translation unit of their own.
+// Compiled once per draw family (the packed layout, and with SMAT_DRAW16
+// the 16-bit draw option: the _d16 launchers; smat_internal.h).
 #include "smat_simulate.cuh"
 
 namespace smat {

@@ -1,4 +1,6 @@
 // Row a3 (forward, grid-stride launch with SMAT_FLAG_UNFUSED_STATS) for f32 parameters.
+// Compiled once per draw family (the packed layout, and with SMAT_DRAW16
+// the 16-bit draw option: the _d16 launchers; smat_internal.h).
 #include "smat_simulate.cuh"
 
 namespace smat {
