@@ -38,6 +38,11 @@ class OrcTensor(ctypes.Structure):
                 ("sigma_rel", ctypes.c_float)]
 
 
+class OrcAdamW(ctypes.Structure):
+    _fields_ = [("lr", ctypes.c_float), ("beta1", ctypes.c_float), ("beta2", ctypes.c_float),
+                ("eps", ctypes.c_float), ("weight_decay", ctypes.c_float), ("step", ctypes.c_int32)]
+
+
 class OrcMerge(ctypes.Structure):
     _fields_ = [("seed", ctypes.c_uint64), ("rounds", ctypes.c_int32), ("method", ctypes.c_int32),
                 ("n_experts", ctypes.c_int32), ("gamma", ctypes.c_float), ("p_drop", ctypes.c_float),
@@ -64,6 +69,7 @@ def lib():
         L.orc_gradmap.argtypes = [P, P, ctypes.c_int32, ctypes.c_int32, P, P]
         L.orc_gradmap_at.argtypes = [P, P, ctypes.c_int32, ctypes.c_int32, P, ctypes.c_int64, P, P, P]
         L.orc_mask_bits.argtypes = [P, P, P]
+        L.orc_gradmap_adamw.argtypes = [P, P, ctypes.c_int32, P, P, P, P, P]
         L.orc_gauss_z.argtypes = [P, P, P, ctypes.c_int64, P]
         L.orc_noise_z.argtypes = [P, P, P, ctypes.c_int64, P]
         L.orc_laplace.argtypes = [P, ctypes.c_int64, P]
@@ -73,7 +79,7 @@ def lib():
         for name in ("orc_philox", "orc_stream_words", "orc_f32_to_bf16", "orc_erfinv", "orc_scalars",
                      "orc_delta_stats", "orc_simulate", "orc_simulate_at", "orc_gradmap",
                      "orc_gradmap_at", "orc_mask_bits", "orc_gauss_z", "orc_simulate_f64",
-                     "orc_gradmap_f64", "orc_noise_z", "orc_laplace", "orc_merge"):
+                     "orc_gradmap_f64", "orc_noise_z", "orc_laplace", "orc_merge", "orc_gradmap_adamw"):
             getattr(L, name).restype = None
         _lib = L
     return _lib
@@ -202,6 +208,20 @@ def gradmap_at(cfg, t, idx, gsim_vals, gdtype=F32, accumulate=False, gold_vals=N
     lib().orc_gradmap_at(ctypes.byref(cfg), ctypes.byref(t), gdtype, int(bool(accumulate)), _p(idx),
                          idx.shape[0], _p(gs), _p(go), _p(out))
     return out
+
+
+def gradmap_adamw(cfg, t, g_sim, theta, m1, m2, lr, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.0,
+                  adam_step=1, gdtype=F32):
+    """The gradient map fused with an AdamW step (see orc_gradmap_adamw):
+    returns new (theta, m1, m2); the inputs are not modified."""
+    gs = _c(g_sim, _store_dtype(gdtype))
+    th = np.array(theta, dtype=_store_dtype(t.dtype), copy=True)
+    a = np.array(m1, dtype=np.float32, copy=True)
+    b = np.array(m2, dtype=np.float32, copy=True)
+    o = OrcAdamW(lr, beta1, beta2, eps, weight_decay, adam_step)
+    lib().orc_gradmap_adamw(ctypes.byref(cfg), ctypes.byref(t), gdtype, _p(gs), _p(th), _p(a), _p(b),
+                            ctypes.byref(o))
+    return th, a, b
 
 
 def mask_bits(cfg, t):

@@ -142,6 +142,16 @@ struct OrcConfig {
   int32_t draw_bits;   // 32 (the packed layout; 0 reads as 32) or 16 (the 16-bit draw option)
 };
 
+// AdamW hyperparameters of the fused gradient map + optimizer step.
+struct OrcAdamW {
+  float lr;
+  float beta1;
+  float beta2;
+  float eps;
+  float weight_decay;
+  int32_t step;  // t >= 1: the optimizer's own step count (bias corrections)
+};
+
 struct OrcTensor {
   uint32_t tensor_id;  // < 0x0FFFFFFF
   int32_t dtype;       // parameter storage dtype
@@ -493,6 +503,44 @@ void orc_gradmap(const OrcConfig* cfg, const OrcTensor* t, int32_t gdtype, int32
     const float gold = accumulate ? load_elem(g_out, gdtype, i) : 0.0f;
     const float v = gradmap_value(*cfg, *t, s, gidx, load_elem(g_sim, gdtype, i), accumulate, gold);
     store_elem(g_out, gdtype, i, v);
+  }
+}
+
+// Gradient map fused with the optimizer step of the simulated-loss step
+// (Sec. 4.3: the mapped gradient updates the original storage theta), here
+// AdamW with decoupled weight decay (Loshchilov and Hutter, ICLR 2019) and
+// fp32 moments. Per element, one IEEE binary32 operation at a time:
+//   g   = the value the gradient map stores (Eq. smat-gradient, rounded to the
+//         gradient dtype), so the fused step equals the gradient map followed
+//         by the update
+//   th  = th * decay,                 decay = fl(1 - lr wd)
+//   m1  = b1 m1 + omb1 g,             omb1  = fl(1 - b1)
+//   m2  = b2 m2 + omb2 (g g),         omb2  = fl(1 - b2)
+//   den = sqrt(m2) / bc2 + eps,       bc2   = fl(sqrt(1 - b2^t))
+//   th  = th - step (m1 / den),       step  = fl(lr / (1 - b1^t))
+// with the per-call constants computed in double and rounded once; theta is
+// then rounded to its storage dtype. theta is updated in place (dtype of the
+// tensor), m1 and m2 are fp32 arrays updated in place.
+void orc_gradmap_adamw(const OrcConfig* cfg, const OrcTensor* t, int32_t gdtype, const void* g_sim,
+                       void* theta, float* m1, float* m2, const OrcAdamW* o) {
+  const Scalars s = make_scalars(*cfg, *t, 0.0f);
+  const double b1 = o->beta1, b2 = o->beta2, tt = (double)o->step;
+  const float decay = (float)(1.0 - (double)o->lr * (double)o->weight_decay);
+  const float omb1 = (float)(1.0 - b1), omb2 = (float)(1.0 - b2);
+  const float bc2 = (float)std::sqrt(1.0 - std::pow(b2, tt));
+  const float step = (float)((double)o->lr / (1.0 - std::pow(b1, tt)));
+  for (int64_t i = 0; i < t->numel; ++i) {
+    const uint64_t gidx = (uint64_t)(t->elem_offset + i);
+    // the stored gradient: rounded to the gradient dtype and read back
+    float g = gradmap_value(*cfg, *t, s, gidx, load_elem(g_sim, gdtype, i), 0, 0.0f);
+    if (gdtype == DT_BF16) g = bf16_bits_to_f32(f32_to_bf16_bits(g));
+    float th = load_elem(theta, t->dtype, i);
+    th = th * decay;
+    m1[i] = o->beta1 * m1[i] + omb1 * g;
+    m2[i] = o->beta2 * m2[i] + omb2 * (g * g);
+    const float den = std::sqrt(m2[i]) / bc2 + o->eps;
+    th = th - step * (m1[i] / den);
+    store_elem(theta, t->dtype, i, th);
   }
 }
 

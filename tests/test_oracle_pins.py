@@ -983,3 +983,61 @@ def test_draw16_gaussian_and_alpha_laws():
     assert np.all((a >= amin) & (a < amax))
     assert stats.kstest((a - amin) / (amax - amin), "uniform").pvalue > 1e-4
     assert abs(np.corrcoef(a[:-1], a[1:])[0, 1]) < 5 / math.sqrt(n)
+
+
+# ------------------------------------- gradient map fused with AdamW (Sec. 4.3) ---
+
+def test_gradmap_adamw_matches_torch_adamw_on_the_mapped_gradient():
+    """The fused step equals torch.optim.AdamW (a library routine, float64)
+    applied with the gradient the gradient map stores (Eq. smat-gradient:
+    alpha m (.) g~, dropped coordinates 0), step after step, within fp32
+    rounding; moments likewise. Per-element alpha, a Mask, weight decay, bf16
+    gradients."""
+    n, steps = 4096, 5
+    lr, b1, b2, eps, wd = 1e-3, 0.9, 0.95, 1e-8, 0.1
+    rg = rng(70)
+    t = O.tensor(12, n, dtype=O.F32, keep_prob=0.7)
+    th = (rg.standard_normal(n) * 0.02).astype(np.float32)
+    m1 = np.zeros(n, np.float32)
+    m2 = np.zeros(n, np.float32)
+    p = torch.tensor(th.astype(np.float64), requires_grad=True)
+    f = lambda v: float(np.float32(v))  # noqa: E731  (the hyperparameters cross the ABI as fp32)
+    opt = torch.optim.AdamW([p], lr=f(lr), betas=(f(b1), f(b2)), eps=f(eps), weight_decay=f(wd))
+    for k in range(1, steps + 1):
+        cfg = O.config(seed=8, step=10 + k, alpha_mode=O.ALPHA_PER_ELEMENT, alpha_min=0.3)
+        gs = O.f32_to_bf16((rg.standard_normal(n) * 0.5).astype(np.float32))
+        g = O.bf16_to_f32(O.gradmap(cfg, t, gs, gdtype=O.BF16)).astype(np.float64)
+        th, m1, m2 = O.gradmap_adamw(cfg, t, gs, th, m1, m2, lr, b1, b2, eps, wd, adam_step=k, gdtype=O.BF16)
+        p.grad = torch.tensor(g)
+        opt.step()
+        st = opt.state[p]
+        ref = p.detach().numpy()
+        # fp32 rounding, step after step: m1 may cancel towards 0 (an absolute
+        # floor at fp32 resolution of its terms), m2 is a sum of positives
+        assert np.allclose(m1, st["exp_avg"].numpy(), rtol=2e-6, atol=1e-7), k
+        assert np.allclose(m2, st["exp_avg_sq"].numpy(), rtol=1e-6, atol=0), k
+        # theta: a few fp32 ulps of theta per step, and of the update near 0
+        assert np.all(np.abs(th.astype(np.float64) - ref) <= 2e-6 * np.abs(ref) + 5e-5 * lr), k
+
+
+def test_gradmap_adamw_first_step_and_weight_decay_closed_forms():
+    """Step 1 from zero moments without weight decay moves each coordinate by
+    -lr g / (|g| + eps) (the bias corrections cancel); with g~ = 0 the step is
+    the decoupled decay theta (1 - lr wd) alone and the moments stay 0."""
+    n, lr, eps = 2048, 3e-4, 1e-8
+    rg = rng(71)
+    t = O.tensor(13, n, dtype=O.F32, keep_prob=1.0)
+    cfg = O.config(seed=9, step=1, alpha_mode=O.ALPHA_GLOBAL, alpha_min=1.0, alpha_max=1.0)  # alpha = 1: g = g~
+    th = (rg.standard_normal(n) * 0.02).astype(np.float32)
+    gs = (rg.standard_normal(n)).astype(np.float32)
+    z = np.zeros(n, np.float32)
+    b1, b2 = 0.875, 0.984375  # exact in fp32
+    th1, m1, m2 = O.gradmap_adamw(cfg, t, gs, th, z, z, lr, b1, b2, eps, 0.0, adam_step=1)
+    g = gs.astype(np.float64)
+    exp = th.astype(np.float64) - np.float64(np.float32(lr)) * g / (np.abs(g) + eps)
+    assert np.all(np.abs(th1 - exp) <= 2e-7 * np.abs(exp) + 1e-6 * lr)
+    assert np.allclose(m1, (1 - b1) * g, rtol=1e-7) and np.allclose(m2, (1 - b2) * g * g, rtol=3e-7)
+    wd = 0.05
+    th2, a, b = O.gradmap_adamw(cfg, t, z, th, z, z, lr, 0.9, 0.999, eps, wd, adam_step=3)
+    assert np.array_equal(th2, th * np.float32(1.0 - lr * wd))
+    assert not a.any() and not b.any()
