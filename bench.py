@@ -88,6 +88,8 @@ def parse():
     ap.add_argument("--experts", type=int, default=8)
     ap.add_argument("--ref-sample", type=int, default=0,
                     help="elements per step of the oracle sample in --impl reference (0: sized for about 150 s)")
+    ap.add_argument("--adamw", action="store_true",
+                    help="time the gradient map fused with an AdamW step on the chosen list, beside the plain map")
     ap.add_argument("--schedule", action="store_true",
                     help="training-loop overhead of periodic SMAT (Sec. 4.3) over plain fine-tuning, synthetic model")
     return ap.parse_args()
@@ -1083,10 +1085,90 @@ def run_merge(args):
     return 0
 
 
+def run_adamw(args):
+    """The gradient map fused with an AdamW step (smat_grad_map_adamw_multi)
+    on the chosen list, beside the plain gradient map into a separate buffer.
+    Each timed call follows a forward of its own SMAT step (new mask), as in
+    training; the moments start warm (m1 ~ N(0, 1e-6), m2 ~ U[0, 1e-6), as
+    after earlier optimizer steps). A second series times the first optimizer
+    step, from zero moments (reset outside the timed region) on one mask.
+    Algorithmic bytes per element of the fused call: read g~, theta, m1, m2
+    and write theta, m1, m2, g + 2 b + 16 (22 for bf16 gradients and
+    parameters); the plain map moves 2 g, and an update after it would move
+    g + 2 b + 16 again (26 in all). Inputs are larger than L2, so no flush
+    between calls."""
+    from paper_2609_33437_gb300 import smat as S
+    S.load_library()
+    dev = torch.device("cuda")
+    w = workload(args)
+    th, t0, sim, gs, go = W.generate(w, device=dev)
+    gen = torch.Generator(device=dev).manual_seed(w.data_seed + 17)
+    m1 = [torch.randn(t.numel, generator=gen, device=dev) * 1e-3 for t in w.tensors]
+    m2 = [torch.rand(t.numel, generator=gen, device=dev) * 1e-6 for t in w.tensors]
+    sess = S.SmatSession(th, t0, sim, [t.keep_prob for t in w.tensors], [t.sigma for t in w.tensors],
+                         [t.sigma_rel for t in w.tensors], seed=w.seed, alpha_min=w.alpha_min,
+                         alpha_max=w.alpha_max, alpha_mode=w.alpha_mode, noise=w.noise,
+                         philox_rounds=args.philox_rounds, draw_bits=args.draw_bits)
+    hp = dict(lr=1e-5, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.01)
+
+    def ev():
+        return torch.cuda.Event(enable_timing=True)
+
+    fused, plain = [], []
+    n_iter = max(3, args.warmup) + args.steps
+    for i in range(n_iter):
+        sess.simulate_multi(i)
+        e = [ev() for _ in range(4)]
+        e[0].record()
+        sess.grad_map_adamw_multi(i, gs, m1, m2, adam_step=i + 1, **hp)
+        e[1].record()
+        e[2].record()
+        sess.grad_map_multi(i, gs, go)
+        e[3].record()
+        e[3].synchronize()
+        if i >= n_iter - args.steps:
+            fused.append(e[0].elapsed_time(e[1]))
+            plain.append(e[2].elapsed_time(e[3]))
+    cold = []
+    for i in range(max(3, args.warmup) + args.steps):
+        for x in m1 + m2:
+            x.zero_()
+        e = [ev() for _ in range(2)]
+        e[0].record()
+        sess.grad_map_adamw_multi(n_iter - 1, gs, m1, m2, adam_step=1, **hp)
+        e[1].record()
+        e[1].synchronize()
+        if i >= max(3, args.warmup):
+            cold.append(e[0].elapsed_time(e[1]))
+    n = w.numel
+    gb = 2 if w.gdtype == W.BF16 else 4
+    pb = 2 if w.dtype == W.BF16 else 4
+    fused_bytes = (gb + 2 * pb + 16) * n
+    map_bytes = 2 * gb * n
+    ms_f, ms_m, ms_c = statistics.median(fused), statistics.median(plain), statistics.median(cold)
+    peak, peak_kind = measured_peaks()
+    gbs = fused_bytes / (ms_f * 1e-3) / 1e9
+    rec = recorded_traffic("gradmap_adamw", w.name)
+    assert sess.poll_errors() == 0
+    print(json.dumps({"adamw": True, "workload": w.name, "elements": n, "fused_ms": ms_f,
+                      "fused_gbs": gbs, "fused_frac": gbs / peak, "peak_gbs": peak, "peak_kind": peak_kind,
+                      "fused_bytes_per_elem": fused_bytes / n, "first_step_ms": ms_c,
+                      "first_step_gbs": fused_bytes / (ms_c * 1e-3) / 1e9, "grad_map_ms": ms_m,
+                      "grad_map_gbs": map_bytes / (ms_m * 1e-3) / 1e9,
+                      "separate_bytes_per_elem": 3 * gb + 2 * pb + 16,
+                      "traffic": rec["dram_bytes_per_launch"] if rec else None,
+                      "runs_ms": {"fused": fused, "first_step": cold, "grad_map": plain}, "hyper": hp,
+                      "draw_bits": args.draw_bits, "philox_rounds": args.philox_rounds}))
+    sess.close()
+    return 0
+
+
 def main():
     args = parse()
     if args.merge:
         return run_merge(args)
+    if args.adamw:
+        return run_adamw(args)
     if args.impl == "reference":
         return run_reference(args)
     if args.sweep:

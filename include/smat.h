@@ -188,6 +188,43 @@ smat_status smat_grad_map_multi(smat_ctx* ctx, uint32_t step, const void* const*
                                 void* const* g_out, int32_t gdtype, int32_t accumulate,
                                 smat_stream_t stream);
 
+/* AdamW hyperparameters of smat_grad_map_adamw_multi (decoupled weight
+ * decay). step is the optimizer's own step count t >= 1, used in the bias
+ * corrections 1 - beta1^t and 1 - beta2^t. */
+typedef struct {
+  float lr;            /* finite, >= 0 */
+  float beta1, beta2;  /* in [0, 1) */
+  float eps;           /* finite, > 0 */
+  float weight_decay;  /* finite, >= 0 */
+  int32_t step;        /* >= 1 */
+} smat_adamw;
+
+/* Gradient map fused with the optimizer's update (Sec. 4.3: with the original
+ * storage restored, theta is updated with the mapped gradient of Eq.
+ * smat-gradient). For every element i of tensor k, with
+ * g = alpha m_i g_sim[k][i] rounded to gdtype (the value smat_grad_map_multi
+ * would store; it is not written anywhere), one AdamW step in fp32, each
+ * operation rounded in this order:
+ *   theta *= fl(1 - lr wd);
+ *   m1 = beta1 m1 + fl(1 - beta1) g;  m2 = beta2 m2 + fl(1 - beta2) (g g);
+ *   theta -= fl(lr / (1 - beta1^t)) (m1 / (sqrt(m2) / fl(sqrt(1 - beta2^t)) + eps))
+ * then theta is rounded to the tensor's dtype and stored in place into the
+ * descriptor's theta (which this call writes). The constants fl(...) are
+ * computed in double and rounded to fp32 once. g_sim, m1, m2 are HOST arrays
+ * of n_tensors DEVICE pointers: g_sim[k] numel elements of gdtype, m1[k] and
+ * m2[k] numel fp32 moments each, updated in place; none may overlap another
+ * or theta (SMAT_ERR_INVALID_ARG); misaligned elements (SMAT_ERR_ALIGNMENT);
+ * an entry may be NULL only if numel == 0. The mask rule is
+ * smat_grad_map_multi's (`step` must be the step of the last forward), and the
+ * original storage must be active (SMAT_ERR_STATE otherwise). One pass reads
+ * g_sim, theta, m1, m2 and writes theta, m1, m2: the separate gradient map and
+ * update would also write and re-read the mapped gradient. The pointer table
+ * shares its workspace region with smat_grad_map_multi's, so alternating the
+ * two calls re-uploads it each time. */
+smat_status smat_grad_map_adamw_multi(smat_ctx* ctx, uint32_t step, const void* const* g_sim,
+                                      float* const* m1, float* const* m2, int32_t gdtype,
+                                      const smat_adamw* opt, smat_stream_t stream);
+
 /* Parameter storage switch (Sec. 4.3): flips the active storage and returns
  * it in *active_out (0 = theta, the original storage; 1 = sim, theta~).
  * Host only: no device work, no copy. */

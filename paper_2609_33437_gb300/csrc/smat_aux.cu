@@ -174,6 +174,15 @@ cudaError_t launch_grad_map(const KArgs& a, int grid, int gdtype, bool per_elem_
 int grad_map_occ(int gdtype, bool per_elem_alpha, bool accumulate, int rounds) {
   return SMAT_BY_FAMILY(gradmap_ctas_per_sm)(gdtype, per_elem_alpha, accumulate, rounds);
 }
+
+cudaError_t launch_grad_map_adamw(const KArgs& a, int grid, int gdtype, int pdtype, bool per_elem_alpha, int rounds,
+                                  cudaStream_t s) {
+  return SMAT_BY_FAMILY(launch_gradmap_adamw)(a, grid, gdtype, pdtype, per_elem_alpha, rounds, s);
+}
+
+int grad_map_adamw_occ(int gdtype, int pdtype, bool per_elem_alpha, int rounds) {
+  return SMAT_BY_FAMILY(gradmap_adamw_ctas_per_sm)(gdtype, pdtype, per_elem_alpha, rounds);
+}
 #undef SMAT_BY_FAMILY
 
 cudaError_t launch_delta_stats(const KArgs& a, int grid, int dtype, cudaStream_t s) {

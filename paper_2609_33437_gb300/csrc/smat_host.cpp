@@ -71,7 +71,8 @@ Layout layout_for(int32_t n, int64_t n_chunks, bool any_sigma_rel) {
   L.chunks = off;  off = align_up(off + sizeof(Chunk) * (size_t)n_chunks);
   L.scal = off;    off = align_up(off + sizeof(DevScalars) * (size_t)n);
   L.partials = off; off = align_up(off + (any_sigma_rel ? sizeof(StatPartial) * (size_t)n_chunks : 0));
-  L.grads = off;   off = align_up(off + sizeof(GradPtr) * (size_t)n);
+  // the gradient-map and fused-AdamW pointer tables share this region
+  L.grads = off;   off = align_up(off + std::max(sizeof(GradPtr), sizeof(AdamPtr)) * (size_t)n);
   L.items = off;   off = align_up(off + sizeof(int32_t) * (any_sigma_rel ? 2 : 1) * (size_t)n_chunks);
   L.sync = off;    off = align_up(off + sizeof(int32_t) * sync_words(n));
   L.total = off;
@@ -243,6 +244,10 @@ struct smat_ctx {
   bool scalars_sigma = false; // the table's sigma_t are current
   std::vector<GradPtr> h_grads;
   bool grads_uploaded = false;
+  // the fused AdamW table lives in the same workspace region as the gradient
+  // table: uploading one invalidates the other
+  std::vector<AdamPtr> h_adams;
+  bool adams_uploaded = false;
   // work-list forward launch (with the statistics of sigma_rel tensors)
   bool fused = false;
   bool wide = false;  // the bf16 fused launch carries statistics items: its four-CTA build
@@ -304,6 +309,7 @@ KArgs base_args(const smat_ctx* c, uint32_t step) {
   a.scal = c->d_scal;
   a.partials = c->d_partials;
   a.grads = c->d_grads;
+  a.adams = reinterpret_cast<const AdamPtr*>(c->d_grads);
   a.key = c->keys;
   a.step = step;
   a.n_tensors = (int32_t)c->desc.size();
@@ -621,6 +627,7 @@ smat_status smat_grad_map_multi(smat_ctx* c, uint32_t step, const void* const* g
       if (e != cudaSuccess) return cuda_fail(e, "gradient table upload");
     }
     c->grads_uploaded = true;
+    c->adams_uploaded = false;
   }
   if (c->scalars_step != (int64_t)step) {
     const smat_status st = run_scalars(c, step, false, stream);
@@ -638,6 +645,105 @@ smat_status smat_grad_map_multi(smat_ctx* c, uint32_t step, const void* const* g
                                        accumulate != 0, c->rounds, stream);
   t.done();
   if (e != cudaSuccess) return cuda_fail(e, "gradient map launch");
+  return SMAT_OK;
+}
+
+smat_status smat_grad_map_adamw_multi(smat_ctx* c, uint32_t step, const void* const* g_sim, float* const* m1,
+                                      float* const* m2, int32_t gdtype, const smat_adamw* opt,
+                                      smat_stream_t stream) {
+  if (!c) return fail(SMAT_ERR_INVALID_ARG, "ctx is NULL");
+  if (!opt) return fail(SMAT_ERR_INVALID_ARG, "opt is NULL");
+  if (gdtype != SMAT_F32 && gdtype != SMAT_BF16)
+    return fail(SMAT_ERR_UNSUPPORTED, "gradient dtype %d not supported", gdtype);
+  if (!(std::isfinite(opt->lr) && opt->lr >= 0.0f))
+    return fail(SMAT_ERR_INVALID_ARG, "lr must be finite and >= 0");
+  if (!(opt->beta1 >= 0.0f && opt->beta1 < 1.0f) || !(opt->beta2 >= 0.0f && opt->beta2 < 1.0f))
+    return fail(SMAT_ERR_INVALID_ARG, "beta1 and beta2 must lie in [0, 1)");
+  if (!(std::isfinite(opt->eps) && opt->eps > 0.0f)) return fail(SMAT_ERR_INVALID_ARG, "eps must be finite and > 0");
+  if (!(std::isfinite(opt->weight_decay) && opt->weight_decay >= 0.0f))
+    return fail(SMAT_ERR_INVALID_ARG, "weight_decay must be finite and >= 0");
+  if (opt->step < 1) return fail(SMAT_ERR_INVALID_ARG, "optimizer step %d: must be >= 1", opt->step);
+  // same rule as the gradient map: the mask of the forward that produced the
+  // gradient's theta~ (App. D)
+  if (c->sim_step != (int64_t)step) {
+    if (c->sim_step < 0)
+      return fail(SMAT_ERR_STATE, "gradient map for step %u, but no forward has run on this context", step);
+    return fail(SMAT_ERR_STATE, "gradient map for step %u, but the last forward on this context was step %lld", step,
+                (long long)c->sim_step);
+  }
+  // the update writes theta, so the original storage must be the one the
+  // model reads (Sec. 4.3: the storage is switched back before the update)
+  if (c->active != 0) return fail(SMAT_ERR_STATE, "the simulated storage is active: switch back before the update");
+  const int32_t n = (int32_t)c->desc.size();
+  if (n > 0 && (!g_sim || !m1 || !m2)) return fail(SMAT_ERR_INVALID_ARG, "pointer arrays are NULL");
+  const size_t es = elem_size(gdtype);
+  std::vector<AdamPtr> t((size_t)n);
+  for (int32_t k = 0; k < n; ++k) {
+    const smat_tensor_desc& d = c->desc[k];
+    AdamPtr& p = t[k];
+    std::memset(&p, 0, sizeof(p));
+    p.g_sim = g_sim[k];
+    p.m1 = m1[k];
+    p.m2 = m2[k];
+    if (d.numel > 0) {
+      if (!p.g_sim || !p.m1 || !p.m2) return fail(SMAT_ERR_INVALID_ARG, "tensor %d: NULL pointer", k);
+      if ((uintptr_t)p.g_sim % es) return fail(SMAT_ERR_ALIGNMENT, "tensor %d: g_sim not aligned to %zu bytes", k, es);
+      if ((uintptr_t)p.m1 % 4 || (uintptr_t)p.m2 % 4)
+        return fail(SMAT_ERR_ALIGNMENT, "tensor %d: moment buffers not 4-byte aligned", k);
+      const size_t gb = es * (size_t)d.numel, mb = 4 * (size_t)d.numel;
+      const size_t tb = elem_size(d.dtype) * (size_t)d.numel;
+      if (overlaps(p.m1, mb, p.m2, mb) || overlaps(p.m1, mb, d.theta, tb) || overlaps(p.m2, mb, d.theta, tb) ||
+          overlaps(p.g_sim, gb, d.theta, tb) || overlaps(p.g_sim, gb, p.m1, mb) || overlaps(p.g_sim, gb, p.m2, mb))
+        return fail(SMAT_ERR_INVALID_ARG, "tensor %d: theta, g_sim, m1 and m2 must not overlap", k);
+    }
+    p.vec = ((uintptr_t)p.g_sim % 32 == 0 && (uintptr_t)p.m1 % 32 == 0 && (uintptr_t)p.m2 % 32 == 0 &&
+             (uintptr_t)d.theta % 32 == 0 && d.elem_offset % 16 == 0)
+                ? 1u
+                : 0u;
+  }
+  if (!c->adams_uploaded || t.size() != c->h_adams.size() ||
+      (n > 0 && std::memcmp(t.data(), c->h_adams.data(), sizeof(AdamPtr) * (size_t)n) != 0)) {
+    c->h_adams.swap(t);
+    if (n > 0) {
+      const cudaError_t e = cudaMemcpyAsync(c->d_grads, c->h_adams.data(), sizeof(AdamPtr) * (size_t)n,
+                                            cudaMemcpyHostToDevice, stream);
+      if (e != cudaSuccess) return cuda_fail(e, "optimizer table upload");
+    }
+    c->adams_uploaded = true;
+    c->grads_uploaded = false;
+  }
+  if (c->scalars_step != (int64_t)step) {
+    const smat_status st = run_scalars(c, step, false, stream);
+    if (st != SMAT_OK) return st;
+  }
+  KArgs a = base_args(c, step);
+  const double b1 = opt->beta1, b2 = opt->beta2, tt = (double)opt->step;
+  a.adam.decay = (float)(1.0 - (double)opt->lr * (double)opt->weight_decay);
+  a.adam.b1 = opt->beta1;
+  a.adam.omb1 = (float)(1.0 - b1);
+  a.adam.b2 = opt->beta2;
+  a.adam.omb2 = (float)(1.0 - b2);
+  a.adam.bc2 = (float)std::sqrt(1.0 - std::pow(b2, tt));
+  a.adam.step = (float)((double)opt->lr / (1.0 - std::pow(b1, tt)));
+  a.adam.eps = opt->eps;
+  a.chunk_begin = 0;
+  a.chunk_end = (int64_t)c->h_chunks.size();
+  if (a.chunk_end <= 0) return SMAT_OK;
+  // one launch per parameter dtype (the kernel is specialised on it)
+  const bool pe = c->cfg.alpha_mode == SMAT_ALPHA_PER_ELEMENT;
+  for (int dt = 0; dt < 2; ++dt) {
+    a.chunk_begin = c->range_begin[dt];
+    a.chunk_end = c->range_end[dt];
+    if (a.chunk_end <= a.chunk_begin) continue;
+    const int pdt = dt == 0 ? SMAT_F32 : SMAT_BF16;
+    const int64_t units = (a.chunk_end - a.chunk_begin) * (int64_t)a.grad_units;
+    const int64_t resident = (int64_t)c->sm_count * grad_map_adamw_occ(gdtype, pdt, pe, c->rounds);
+    const int grid = (int)(units < resident ? units : resident);
+    Timed tm(c, 3, stream);
+    const cudaError_t e = launch_grad_map_adamw(a, grid, gdtype, pdt, pe, c->rounds, stream);
+    tm.done();
+    if (e != cudaSuccess) return cuda_fail(e, "fused AdamW launch");
+  }
   return SMAT_OK;
 }
 

@@ -84,6 +84,25 @@ struct GradPtr {
   uint32_t pad;
 };
 
+// Gradient map fused with AdamW: the incoming gradient and the fp32 moment
+// buffers of one tensor (theta is the tensor's own theta).
+struct AdamPtr {  // 32 bytes
+  const void* g_sim;
+  float* m1;
+  float* m2;
+  uint32_t vec;  // theta, g_sim, m1, m2 32-byte aligned and elem_offset % 16 == 0
+  uint32_t pad;
+};
+
+// Per-call AdamW constants, computed in double on the host and rounded once.
+struct AdamScalars {
+  float decay;  // fl(1 - lr wd)
+  float b1, omb1, b2, omb2;  // beta1, fl(1 - beta1), beta2, fl(1 - beta2)
+  float bc2;    // fl(sqrt(1 - beta2^t))
+  float step;   // fl(lr / (1 - beta1^t))
+  float eps;
+};
+
 // Philox round keys, precomputed from the seed on the host.
 struct RoundKeys {
   uint32_t k0[kMaxRounds];
@@ -117,6 +136,9 @@ struct KArgs {
   uint32_t* ready;       // per tensor: epoch of the call whose sigma_t is published
   int32_t* error;        // device error flags (bit 0: a wait ran out)
   uint32_t epoch;        // this call's epoch (>= 1)
+  // gradient map fused with AdamW
+  const AdamPtr* adams;
+  AdamScalars adam;
 };
 
 constexpr uint32_t kItemForward = 0x80000000u;
@@ -167,7 +189,10 @@ cudaError_t launch_stats_simulate(const KArgs& a, int grid, int dtype, int noise
                                                 int rounds, cudaStream_t s);                                  \
   cudaError_t launch_gradmap##sfx(const KArgs& a, int grid, int gdtype, bool per_elem_alpha, bool accumulate, \
                                   int rounds, cudaStream_t s);                                                \
-  int gradmap_ctas_per_sm##sfx(int gdtype, bool per_elem_alpha, bool accumulate, int rounds);
+  int gradmap_ctas_per_sm##sfx(int gdtype, bool per_elem_alpha, bool accumulate, int rounds);                 \
+  cudaError_t launch_gradmap_adamw##sfx(const KArgs& a, int grid, int gdtype, int pdtype, bool per_elem_alpha, \
+                                        int rounds, cudaStream_t s);                                          \
+  int gradmap_adamw_ctas_per_sm##sfx(int gdtype, int pdtype, bool per_elem_alpha, int rounds);
 SMAT_FORWARD_LAUNCHERS()
 SMAT_FORWARD_LAUNCHERS(_d16)
 #undef SMAT_FORWARD_LAUNCHERS
@@ -178,6 +203,9 @@ int fused_wide_occ(int noise, int rounds);
 cudaError_t launch_grad_map(const KArgs& a, int grid, int gdtype, bool per_elem_alpha, bool accumulate, int rounds,
                             cudaStream_t s);
 int grad_map_occ(int gdtype, bool per_elem_alpha, bool accumulate, int rounds);
+cudaError_t launch_grad_map_adamw(const KArgs& a, int grid, int gdtype, int pdtype, bool per_elem_alpha, int rounds,
+                                  cudaStream_t s);
+int grad_map_adamw_occ(int gdtype, int pdtype, bool per_elem_alpha, int rounds);
 
 // In the forward and gradient-map translation units: the family being
 // compiled (see above) and the name of its launchers.

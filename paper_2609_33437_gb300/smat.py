@@ -6,6 +6,7 @@ no CPU fallback: if the library cannot be loaded the calls raise.
 
 Names follow the C ABI: smat_init -> SmatSession(...), smat_simulate_multi ->
 SmatSession.simulate_multi, smat_grad_map_multi -> SmatSession.grad_map_multi,
+smat_grad_map_adamw_multi -> SmatSession.grad_map_adamw_multi,
 smat_swap -> SmatSession.swap, smat_mask_bits -> SmatSession.mask_bits,
 smat_tensor_scalars -> SmatSession.tensor_scalars.
 """
@@ -27,7 +28,15 @@ EXPORTED = ("smat_workspace_bytes", "smat_init", "smat_simulate_multi", "smat_gr
             "smat_debug_philox", "smat_debug_noise_unit", "smat_debug_fused", "smat_poll_errors",
             "smat_delta_sigma_noalloc", "smat_timing_enable", "smat_timing_read", "smat_status_string",
             "smat_last_error", "smat_abi_version", "smat_refill_theta0", "smat_mark_theta0_resident",
-            "smat_merge_workspace_bytes", "smat_merge", "smat_merge_ties_thresholds")
+            "smat_merge_workspace_bytes", "smat_merge", "smat_merge_ties_thresholds",
+            "smat_grad_map_adamw_multi")
+
+
+class AdamW(ctypes.Structure):
+    """smat_adamw: AdamW hyperparameters (decoupled weight decay); step is the
+    optimizer's own step count t >= 1."""
+    _fields_ = [("lr", ctypes.c_float), ("beta1", ctypes.c_float), ("beta2", ctypes.c_float),
+                ("eps", ctypes.c_float), ("weight_decay", ctypes.c_float), ("step", ctypes.c_int32)]
 
 
 class SmatError(RuntimeError):
@@ -81,6 +90,7 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
     L.smat_init.argtypes = [ctypes.POINTER(P), P, I32, P, P, ctypes.c_size_t, P]
     L.smat_simulate_multi.argtypes = [P, U32, P]
     L.smat_grad_map_multi.argtypes = [P, U32, P, P, I32, I32, P]
+    L.smat_grad_map_adamw_multi.argtypes = [P, U32, P, P, P, I32, ctypes.POINTER(AdamW), P]
     L.smat_swap.argtypes = [P, ctypes.POINTER(I32)]
     L.smat_active.argtypes = [P, ctypes.POINTER(I32)]
     L.smat_mask_bits.argtypes = [P, U32, I32, P, P]
@@ -105,7 +115,8 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
     L.smat_last_error.argtypes = []
     L.smat_last_error.restype = ctypes.c_char_p
     L.smat_abi_version.restype = I32
-    for name in ("smat_init", "smat_simulate_multi", "smat_grad_map_multi", "smat_swap", "smat_active",
+    for name in ("smat_init", "smat_simulate_multi", "smat_grad_map_multi", "smat_grad_map_adamw_multi",
+                 "smat_swap", "smat_active",
                  "smat_mask_bits", "smat_tensor_scalars", "smat_destroy", "smat_debug_philox", "smat_debug_noise_unit",
                  "smat_poll_errors", "smat_debug_fused", "smat_timing_enable", "smat_timing_read",
                  "smat_refill_theta0", "smat_mark_theta0_resident", "smat_merge", "smat_merge_ties_thresholds"):
@@ -224,6 +235,38 @@ class SmatSession:
         check("smat_grad_map_multi",
               self._L.smat_grad_map_multi(self._ctx, int(step), ins, outs, SMAT_F32 if gd is None else gd,
                                           int(bool(accumulate)), _stream_handle(stream)))
+
+    def grad_map_adamw_multi(self, step: int, g_sims: Sequence[torch.Tensor], m1s: Sequence[torch.Tensor],
+                             m2s: Sequence[torch.Tensor], lr: float, beta1: float = 0.9, beta2: float = 0.999,
+                             eps: float = 1e-8, weight_decay: float = 0.0, adam_step: int = 1,
+                             stream: Optional[torch.cuda.Stream] = None):
+        """The gradient map fused with one AdamW step: theta (the descriptors'
+        own storage) and the fp32 moments m1s, m2s are updated in place."""
+        if len(g_sims) != self.n or len(m1s) != self.n or len(m2s) != self.n:
+            raise ValueError("one gradient and two moment buffers per tensor expected")
+        gd = None
+        gp = (ctypes.c_void_p * max(self.n, 1))()
+        p1 = (ctypes.c_void_p * max(self.n, 1))()
+        p2 = (ctypes.c_void_p * max(self.n, 1))()
+        for k in range(self.n):
+            g, a, b = g_sims[k], m1s[k], m2s[k]
+            if g.numel() != self.numels[k] or a.numel() != self.numels[k] or b.numel() != self.numels[k]:
+                raise ValueError(f"tensor {k}: numel mismatch")
+            if a.dtype != torch.float32 or b.dtype != torch.float32:
+                raise ValueError(f"tensor {k}: moments must be float32")
+            if not all(x.is_cuda and x.is_contiguous() for x in (g, a, b)):
+                raise ValueError(f"tensor {k}: must be contiguous CUDA tensors")
+            code = dtype_code(g.dtype)
+            if gd is None:
+                gd = code
+            elif gd != code:
+                raise ValueError("all gradients must share one dtype")
+            gp[k], p1[k], p2[k] = g.data_ptr(), a.data_ptr(), b.data_ptr()
+        self._gkeep = (list(g_sims), list(m1s), list(m2s))
+        opt = AdamW(float(lr), float(beta1), float(beta2), float(eps), float(weight_decay), int(adam_step))
+        check("smat_grad_map_adamw_multi",
+              self._L.smat_grad_map_adamw_multi(self._ctx, int(step), gp, p1, p2, SMAT_F32 if gd is None else gd,
+                                                ctypes.byref(opt), _stream_handle(stream)))
 
     def swap(self) -> int:
         a = ctypes.c_int32()

@@ -171,6 +171,8 @@ def test_init_rejects_duplicate_ids_overlap_and_workspace(L):
 def test_null_context_calls_fail_cleanly(L):
     assert L.smat_simulate_multi(None, 0, None) == 1
     assert L.smat_grad_map_multi(None, 0, None, None, 0, 0, None) == 1
+    opt = S.AdamW(1e-3, 0.9, 0.999, 1e-8, 0.0, 1)
+    assert L.smat_grad_map_adamw_multi(None, 0, None, None, None, 0, ctypes.byref(opt), None) == 1
     a = ctypes.c_int32()
     assert L.smat_swap(None, ctypes.byref(a)) == 1
     assert L.smat_mask_bits(None, 0, 0, None, None) == 1
@@ -240,7 +242,7 @@ def test_binding_matches_header_layout(tmp_path):
     if cc is None:
         pytest.skip("no host C compiler")
     structs = {"smat_tensor_desc": S.TensorDesc, "smat_config": S.Config,
-               "smat_merge_tensor": S.MergeTensor, "smat_merge_config": S.MergeConfig}
+               "smat_merge_tensor": S.MergeTensor, "smat_merge_config": S.MergeConfig, "smat_adamw": S.AdamW}
     consts = ["SMAT_F32", "SMAT_BF16", "SMAT_NOISE_UNIFORM", "SMAT_NOISE_GAUSSIAN", "SMAT_NOISE_LAPLACE",
               "SMAT_ALPHA_GLOBAL", "SMAT_ALPHA_PER_TENSOR", "SMAT_ALPHA_PER_ELEMENT", "SMAT_FLAG_UNFUSED_STATS",
               "SMAT_MERGE_WA", "SMAT_MERGE_TA", "SMAT_MERGE_DARE_TA", "SMAT_MERGE_TIES"]
