@@ -70,6 +70,7 @@ def lib():
         L.orc_gradmap_at.argtypes = [P, P, ctypes.c_int32, ctypes.c_int32, P, ctypes.c_int64, P, P, P]
         L.orc_mask_bits.argtypes = [P, P, P]
         L.orc_gradmap_adamw.argtypes = [P, P, ctypes.c_int32, P, P, P, P, P]
+        L.orc_gradmap_adamw_at.argtypes = [P, P, ctypes.c_int32, P, ctypes.c_int64, P, P, P, P, P, P]
         L.orc_gauss_z.argtypes = [P, P, P, ctypes.c_int64, P]
         L.orc_noise_z.argtypes = [P, P, P, ctypes.c_int64, P]
         L.orc_laplace.argtypes = [P, ctypes.c_int64, P]
@@ -79,7 +80,8 @@ def lib():
         for name in ("orc_philox", "orc_stream_words", "orc_f32_to_bf16", "orc_erfinv", "orc_scalars",
                      "orc_delta_stats", "orc_simulate", "orc_simulate_at", "orc_gradmap",
                      "orc_gradmap_at", "orc_mask_bits", "orc_gauss_z", "orc_simulate_f64",
-                     "orc_gradmap_f64", "orc_noise_z", "orc_laplace", "orc_merge", "orc_gradmap_adamw"):
+                     "orc_gradmap_f64", "orc_noise_z", "orc_laplace", "orc_merge", "orc_gradmap_adamw",
+                     "orc_gradmap_adamw_at"):
             getattr(L, name).restype = None
         _lib = L
     return _lib
@@ -222,6 +224,22 @@ def gradmap_adamw(cfg, t, g_sim, theta, m1, m2, lr, beta1=0.9, beta2=0.999, eps=
     lib().orc_gradmap_adamw(ctypes.byref(cfg), ctypes.byref(t), gdtype, _p(gs), _p(th), _p(a), _p(b),
                             ctypes.byref(o))
     return th, a, b
+
+
+def gradmap_adamw_at(cfg, t, idx, gsim_vals, theta_vals, m1_vals, m2_vals, lr, beta1=0.9, beta2=0.999, eps=1e-8,
+                     weight_decay=0.0, adam_step=1, gdtype=F32):
+    """gradmap_adamw at sampled local indices (g~ and theta as fp32 values):
+    returns (theta stored bits as uint32, m1, m2)."""
+    idx = _c(idx, np.int64)
+    gs = _c(gsim_vals, np.float32)
+    th = _c(theta_vals, np.float32)
+    a = np.array(m1_vals, dtype=np.float32, copy=True)
+    b = np.array(m2_vals, dtype=np.float32, copy=True)
+    out = np.zeros(idx.shape[0], np.uint32)
+    o = OrcAdamW(lr, beta1, beta2, eps, weight_decay, adam_step)
+    lib().orc_gradmap_adamw_at(ctypes.byref(cfg), ctypes.byref(t), gdtype, _p(idx), idx.shape[0], _p(gs), _p(th),
+                               _p(a), _p(b), ctypes.byref(o), _p(out))
+    return out, a, b
 
 
 def mask_bits(cfg, t):

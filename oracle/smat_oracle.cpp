@@ -521,26 +521,60 @@ void orc_gradmap(const OrcConfig* cfg, const OrcTensor* t, int32_t gdtype, int32
 // with the per-call constants computed in double and rounded once; theta is
 // then rounded to its storage dtype. theta is updated in place (dtype of the
 // tensor), m1 and m2 are fp32 arrays updated in place.
+namespace {
+struct AdamConsts {
+  float decay, omb1, omb2, bc2, step;
+};
+
+AdamConsts adam_consts(const OrcAdamW& o) {
+  const double b1 = o.beta1, b2 = o.beta2, tt = (double)o.step;
+  AdamConsts k;
+  k.decay = (float)(1.0 - (double)o.lr * (double)o.weight_decay);
+  k.omb1 = (float)(1.0 - b1);
+  k.omb2 = (float)(1.0 - b2);
+  k.bc2 = (float)std::sqrt(1.0 - std::pow(b2, tt));
+  k.step = (float)((double)o.lr / (1.0 - std::pow(b1, tt)));
+  return k;
+}
+
+// One element: the stored gradient (Eq. smat-gradient, rounded to the
+// gradient dtype and read back), then the update above; returns theta
+// before its rounding to the storage dtype.
+float adam_element(const OrcConfig& cfg, const OrcTensor& t, const Scalars& s, const OrcAdamW& o,
+                   const AdamConsts& k, int32_t gdtype, uint64_t gidx, float g_sim, float th, float& m1,
+                   float& m2) {
+  float g = gradmap_value(cfg, t, s, gidx, g_sim, 0, 0.0f);
+  if (gdtype == DT_BF16) g = bf16_bits_to_f32(f32_to_bf16_bits(g));
+  th = th * k.decay;
+  m1 = o.beta1 * m1 + k.omb1 * g;
+  m2 = o.beta2 * m2 + k.omb2 * (g * g);
+  const float den = std::sqrt(m2) / k.bc2 + o.eps;
+  return th - k.step * (m1 / den);
+}
+}  // namespace
+
 void orc_gradmap_adamw(const OrcConfig* cfg, const OrcTensor* t, int32_t gdtype, const void* g_sim,
                        void* theta, float* m1, float* m2, const OrcAdamW* o) {
   const Scalars s = make_scalars(*cfg, *t, 0.0f);
-  const double b1 = o->beta1, b2 = o->beta2, tt = (double)o->step;
-  const float decay = (float)(1.0 - (double)o->lr * (double)o->weight_decay);
-  const float omb1 = (float)(1.0 - b1), omb2 = (float)(1.0 - b2);
-  const float bc2 = (float)std::sqrt(1.0 - std::pow(b2, tt));
-  const float step = (float)((double)o->lr / (1.0 - std::pow(b1, tt)));
+  const AdamConsts k = adam_consts(*o);
   for (int64_t i = 0; i < t->numel; ++i) {
-    const uint64_t gidx = (uint64_t)(t->elem_offset + i);
-    // the stored gradient: rounded to the gradient dtype and read back
-    float g = gradmap_value(*cfg, *t, s, gidx, load_elem(g_sim, gdtype, i), 0, 0.0f);
-    if (gdtype == DT_BF16) g = bf16_bits_to_f32(f32_to_bf16_bits(g));
-    float th = load_elem(theta, t->dtype, i);
-    th = th * decay;
-    m1[i] = o->beta1 * m1[i] + omb1 * g;
-    m2[i] = o->beta2 * m2[i] + omb2 * (g * g);
-    const float den = std::sqrt(m2[i]) / bc2 + o->eps;
-    th = th - step * (m1[i] / den);
+    const float th = adam_element(*cfg, *t, s, *o, k, gdtype, (uint64_t)(t->elem_offset + i),
+                                  load_elem(g_sim, gdtype, i), load_elem(theta, t->dtype, i), m1[i], m2[i]);
     store_elem(theta, t->dtype, i, th);
+  }
+}
+
+// The same at sampled local indices: g~ and theta given as fp32 values, the
+// moments updated in place, theta returned as its stored bits.
+void orc_gradmap_adamw_at(const OrcConfig* cfg, const OrcTensor* t, int32_t gdtype, const int64_t* idx,
+                          int64_t n, const float* gsim_vals, const float* theta_vals, float* m1, float* m2,
+                          const OrcAdamW* o, uint32_t* theta_bits) {
+  const Scalars s = make_scalars(*cfg, *t, 0.0f);
+  const AdamConsts k = adam_consts(*o);
+  for (int64_t j = 0; j < n; ++j) {
+    const float th = adam_element(*cfg, *t, s, *o, k, gdtype, (uint64_t)(t->elem_offset + idx[j]), gsim_vals[j],
+                                  theta_vals[j], m1[j], m2[j]);
+    theta_bits[j] = stored_bits(t->dtype, th);
   }
 }
 

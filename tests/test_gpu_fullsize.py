@@ -101,3 +101,51 @@ def test_full_size_7b_list_draw16_sampled():
     if not torch.cuda.is_available():
         pytest.skip("needs a CUDA GPU")
     _check_workload(W.llama_7b(), step=3, draw_bits=16)
+
+
+@pytest.mark.parametrize("draw_bits", [32, 16])
+def test_full_size_7b_list_fused_adamw_sampled(draw_bits):
+    """The gradient map fused with AdamW on the whole 7B list in the launch
+    configuration `bench.py --adamw` times (one call per optimizer step after
+    the forward of its own SMAT step, warm moments): theta, m1 and m2 bit-exact
+    against the oracle at sampled elements (each tensor's first and last 16
+    and random ones), over two optimizer steps."""
+    w = W.llama_7b()
+    dev = torch.device("cuda")
+    free, total = torch.cuda.mem_get_info()
+    need = 2 * w.numel * 4 + 4 * w.numel * 2
+    if need > free * 0.9:
+        pytest.skip(f"needs {need / 1e9:.1f} GB of device memory, {free / 1e9:.1f} GB free")
+    th, t0, sim, gs, _ = W.generate(w, device=dev, with_grad=True)
+    gen = torch.Generator(device=dev).manual_seed(w.data_seed + 17)
+    m1 = [torch.randn(t.numel, generator=gen, device=dev) * 1e-3 for t in w.tensors]
+    m2 = [torch.rand(t.numel, generator=gen, device=dev) * 1e-6 for t in w.tensors]
+    sess = session_for(w, th, t0, sim, draw_bits=draw_bits)
+    rng = np.random.default_rng(91)
+    picks = []
+    for k, spec in enumerate(w.tensors):
+        n = spec.numel
+        idx = np.unique(np.concatenate([np.arange(min(n, 16)), np.arange(max(0, n - 16), n),
+                                        rng.integers(0, n, size=min(n, SAMPLES // 4))]))
+        it = torch.from_numpy(idx).to(dev)
+        picks.append((idx, it, f32_of(to_host(th[k][it])), to_host(m1[k][it]), to_host(m2[k][it]),
+                      f32_of(to_host(gs[k][it]))))
+    hp = dict(lr=1e-5, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.01)
+    for t_opt, step in enumerate((3, 4), start=1):
+        sess.simulate_multi(step)
+        sess.grad_map_adamw_multi(step, gs, m1, m2, adam_step=t_opt, **hp)
+        torch.cuda.synchronize()
+        cfg = orc_config(w, step, draw_bits=draw_bits)
+        for k in range(len(w.tensors)):
+            idx, it, thv, a, b, gv = picks[k]
+            bits, a, b = O.gradmap_adamw_at(cfg, orc_tensor(w, k), idx, gv, thv, a, b, adam_step=t_opt,
+                                            gdtype=w.gdtype, **hp)
+            got = to_host(th[k][it])
+            assert np.array_equal(got.astype(np.uint32) if w.dtype == O.BF16 else got.view(np.uint32), bits), \
+                f"step {step} tensor {k} theta"
+            assert np.array_equal(to_host(m1[k][it]).view(np.uint32), a.view(np.uint32)), f"tensor {k} m1"
+            assert np.array_equal(to_host(m2[k][it]).view(np.uint32), b.view(np.uint32)), f"tensor {k} m2"
+            thv = f32_of(got)
+            picks[k] = (idx, it, thv, a, b, gv)
+    assert sess.poll_errors() == 0
+    sess.close()

@@ -1041,3 +1041,30 @@ def test_gradmap_adamw_first_step_and_weight_decay_closed_forms():
     th2, a, b = O.gradmap_adamw(cfg, t, z, th, z, z, lr, 0.9, 0.999, eps, wd, adam_step=3)
     assert np.array_equal(th2, th * np.float32(1.0 - lr * wd))
     assert not a.any() and not b.any()
+
+
+@pytest.mark.parametrize("dtype,gdtype", [(O.BF16, O.BF16), (O.F32, O.F32), (O.BF16, O.F32)])
+def test_gradmap_adamw_at_equals_the_whole_tensor(dtype, gdtype):
+    """The sampled form (which the full-size GPU check uses) equals the
+    whole-tensor form at every sampled index: per-element alpha, a keep rate
+    just above a tie boundary, an element offset above 2^33, warm moments."""
+    n = 5000
+    rg = rng(83)
+    t = O.tensor(21, n, dtype=dtype, keep_prob=0.5 + 2**-10, elem_offset=2**33 + 7)
+    cfg = O.config(seed=4, step=6, alpha_mode=O.ALPHA_PER_ELEMENT, alpha_min=0.2)
+    th32 = (rg.standard_normal(n) * 0.02).astype(np.float32)
+    gs32 = rg.standard_normal(n).astype(np.float32)
+    th = O.f32_to_bf16(th32) if dtype == O.BF16 else th32
+    gs = O.f32_to_bf16(gs32) if gdtype == O.BF16 else gs32
+    m1 = (rg.standard_normal(n) * 1e-3).astype(np.float32)
+    m2 = (rg.random(n) * 1e-6).astype(np.float32)
+    hp = dict(lr=1e-3, weight_decay=0.01, adam_step=4, gdtype=gdtype)
+    th_all, m1_all, m2_all = O.gradmap_adamw(cfg, t, gs, th, m1, m2, **hp)
+    idx = np.sort(rg.choice(n, 700, replace=False))
+    thv = O.bf16_to_f32(th[idx]) if dtype == O.BF16 else th[idx]
+    gv = O.bf16_to_f32(gs[idx]) if gdtype == O.BF16 else gs[idx]
+    bits, a, b = O.gradmap_adamw_at(cfg, t, idx, gv, thv, m1[idx], m2[idx], **hp)
+    ref = th_all[idx].view(np.uint16).astype(np.uint32) if dtype == O.BF16 else th_all[idx].view(np.uint32)
+    assert np.array_equal(bits, ref)
+    assert np.array_equal(a.view(np.uint32), m1_all[idx].view(np.uint32))
+    assert np.array_equal(b.view(np.uint32), m2_all[idx].view(np.uint32))
