@@ -25,6 +25,13 @@ Usage (a training loop with any optimizer):
         loss_fn(model, batch).backward()
         sched.after_backward(step)
         opt.step(); opt.zero_grad()
+
+or, with torch.optim.AdamW on fp32 parameters, the gradient map folded into
+the optimizer's read of the gradient on simulated-loss steps:
+
+        sched.before_forward(step)
+        loss_fn(model, batch).backward()
+        sched.optimizer_step(step, opt); opt.zero_grad()
 """
 
 from typing import List, Optional, Sequence
@@ -103,6 +110,58 @@ class PeriodicSmat:
             return
         self.session.grad_map_multi(step, [p.grad for p in self.params], [p.grad for p in self.params])
         self._swap()
+        self._refill_after()
+
+    def _fusable(self, opt) -> bool:
+        """The fused path takes one AdamW parameter group holding exactly this
+        schedule's fp32 parameters, with a plain (non-capturable, non-fused,
+        non-amsgrad, non-maximising) update and one step count for all."""
+        if type(opt) is not torch.optim.AdamW or len(opt.param_groups) != 1:
+            return False
+        g = opt.param_groups[0]
+        if [id(p) for p in g["params"]] != [id(p) for p in self.params]:
+            return False
+        if g.get("amsgrad") or g.get("maximize") or g.get("capturable") or g.get("fused") or g.get("differentiable"):
+            return False
+        if torch.is_tensor(g["lr"]) or any(p.dtype != torch.float32 for p in self.params):
+            return False
+        steps = {float(opt.state[p]["step"]) if "step" in opt.state[p] else 0.0 for p in self.params}
+        return len(steps) == 1
+
+    def optimizer_step(self, step: int, opt):
+        """After the backward pass: on an ordinary step, opt.step(). On a
+        simulated-loss step with an AdamW the fused path accepts (see
+        _fusable), the storage is switched back and the gradient map and the
+        AdamW update run as one pass (smat_grad_map_adamw_multi) on the
+        optimizer's own moments; the mapped gradient is not written (p.grad
+        keeps g~). Otherwise after_backward, then opt.step()."""
+        if not self.is_smat_step(step):
+            opt.step()
+            return
+        if not self._fusable(opt):
+            self.after_backward(step)
+            opt.step()
+            return
+        g = opt.param_groups[0]
+        for p in self.params:
+            st = opt.state[p]
+            if "step" not in st:  # the optimizer's own lazy initialisation, done here first
+                st["step"] = torch.tensor(0.0, dtype=torch.float32)
+                st["exp_avg"] = torch.zeros_like(p, memory_format=torch.preserve_format)
+                st["exp_avg_sq"] = torch.zeros_like(p, memory_format=torch.preserve_format)
+        t = int(float(opt.state[self.params[0]]["step"])) + 1
+        grads = [p.grad for p in self.params]
+        self._swap()
+        beta1, beta2 = g["betas"]
+        self.session.grad_map_adamw_multi(step, grads, [opt.state[p]["exp_avg"] for p in self.params],
+                                          [opt.state[p]["exp_avg_sq"] for p in self.params], lr=g["lr"],
+                                          beta1=beta1, beta2=beta2, eps=g["eps"],
+                                          weight_decay=g["weight_decay"], adam_step=t)
+        for p in self.params:
+            opt.state[p]["step"] += 1
+        self._refill_after()
+
+    def _refill_after(self):
         if self.inplace:
             # the copy may start once this stream is past the gradient map
             ready = torch.cuda.Event()
