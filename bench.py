@@ -1046,7 +1046,8 @@ def run_merge(args):
     method: gamma 0.3 (TA, DARE, TIES), DARE drop 0.3, TIES retention 0.5 (the
     paper's calibrated settings, App. B). Algorithmic bytes per element: the
     merge reads theta0 and the K experts and writes the result, (K + 2) b; TIES
-    adds three radix-select passes reading theta0 and each expert, 6 K b."""
+    adds three radix-select passes that each read theta0 and every expert,
+    3 (K + 1) b: (4 K + 5) b in all."""
     from paper_2609_33437_gb300 import smat as S
     S.load_library()
     dev = torch.device("cuda")
@@ -1077,7 +1078,7 @@ def run_merge(args):
         times.append(e0.elapsed_time(e1))
     ms = statistics.median(times)
     b = 2 if w.dtype == W.BF16 else 4
-    nbytes = (K + 2) * b * w.numel + (6 * K * b * w.numel if method == S.SMAT_MERGE_TIES else 0)
+    nbytes = (K + 2) * b * w.numel + (3 * (K + 1) * b * w.numel if method == S.SMAT_MERGE_TIES else 0)
     peak, peak_kind = measured_peaks()
     print(json.dumps({"merge": args.merge, "experts": K, "workload": w.name, "elements": w.numel,
                       "ms": ms, "gbs": nbytes / (ms * 1e-3) / 1e9, "frac_of_measured_peak": nbytes / (ms * 1e-3) / 1e9 / peak,

@@ -488,12 +488,17 @@ __global__ void __launch_bounds__(kBlock, 2) dare_kernel(const __grid_constant__
 // one shared-memory histogram per expert, flushed into the 64-bit global bins.
 constexpr int kHistExperts = 4;
 
-template <int DT>
-__global__ void __launch_bounds__(kBlock) ties_hist_kernel(const __grid_constant__ MArgs m) {
+// The key is abs(Delta)'s bits: its sign bit is 0, so the prefix test and
+// the digit are taken on Delta's raw bits with bit 31 masked out of both
+// (one operation per key fewer). FIRST: the first pass, where no digit is
+// decided yet and every key counts.
+template <int DT, bool FIRST>
+__global__ void __launch_bounds__(kBlock, DT == DT_BF16 ? 4 : 1) ties_hist_kernel(const __grid_constant__ MArgs m) {
   __shared__ uint32_t h[kHistExperts * kHistBins];
   const int nbat = (m.K + kHistExperts - 1) / kHistExperts;
   const int64_t items = m.n_chunks * nbat;
-  const uint32_t digit = (1u << m.width) - 1u;
+  const uint32_t digit = ((1u << m.width) - 1u) & (0x7FFFFFFFu >> m.shift);
+  const uint32_t dm = m.decided & 0x7FFFFFFFu;
   for (int64_t w = blockIdx.x; w < items; w += gridDim.x) {
     const int64_t ci = w / nbat;
     const int e0 = (int)(w % nbat) * kHistExperts;
@@ -522,9 +527,11 @@ __global__ void __launch_bounds__(kBlock) ties_hist_kernel(const __grid_constant
         for (int b = 0; b < kHistExperts; ++b) {
           if (b < ne) {
 #pragma unroll
-            for (int k = 0; k < 16; ++k) {
-              const uint32_t key = abs_key(__fsub_rn(x[b].at(k), t0.at(k)));
-              if ((key & m.decided) == P[b]) atomicAdd(&h[b * kHistBins + ((key >> m.shift) & digit)], 1u);
+            for (int q = 0; q < 8; ++q) {
+              const float2 d = sub2_rn(x[b].pair(q), t0.pair(q));
+              const uint32_t k0 = __float_as_uint(d.x), k1 = __float_as_uint(d.y);
+              if (FIRST || (k0 & dm) == P[b]) atomicAdd(&h[b * kHistBins + ((k0 >> m.shift) & digit)], 1u);
+              if (FIRST || (k1 & dm) == P[b]) atomicAdd(&h[b * kHistBins + ((k1 >> m.shift) & digit)], 1u);
             }
           }
         }
@@ -714,7 +721,8 @@ cudaError_t merge_launch(MArgs m, int64_t slots, bool ties, int sms, cudaStream_
   if (ties) {
     const int64_t items = m.n_chunks * ((m.K + kHistExperts - 1) / kHistExperts);
     int occ = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, ties_hist_kernel<DT>, kBlock, 0) != cudaSuccess || occ < 1)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, ties_hist_kernel<DT, false>, kBlock, 0) != cudaSuccess ||
+        occ < 1)
       occ = 1;
     const int64_t resident = (int64_t)occ * sms;
     const int hgrid = (int)(items < resident ? items : resident);
@@ -723,7 +731,10 @@ cudaError_t merge_launch(MArgs m, int64_t slots, bool ties, int sms, cudaStream_
       m.width = kPassWidth[p];
       m.decided = (m.shift + m.width >= 32) ? 0u : ~((1u << (m.shift + m.width)) - 1u);
       m.last_pass = p == kPasses - 1;
-      ties_hist_kernel<DT><<<hgrid, kBlock, 0, s>>>(m);
+      if (p == 0)
+        ties_hist_kernel<DT, true><<<hgrid, kBlock, 0, s>>>(m);
+      else
+        ties_hist_kernel<DT, false><<<hgrid, kBlock, 0, s>>>(m);
       ties_select_kernel<<<(int)slots, kBlock, 0, s>>>(m);
     }
   }
