@@ -13,6 +13,9 @@
 //   gradient  g = alpha * m (.) g~                  Eq. smat-gradient (Sec. 4.2)
 //   the mask is regenerated for the gradient, never stored (App. D,
 //   "Implementation details").
+//   update    the stored gradient fed into one decoupled-weight-decay AdamW
+//             step of theta and fp32 moments (Sec. 4.3: theta updated with
+//             the mapped gradient once the storage is switched back).
 //
 // The paper does not say how the random draws are produced. The counter-based
 // stream layout below is this project's specification; every reading of the
